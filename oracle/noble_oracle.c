@@ -1,0 +1,339 @@
+/*
+ * NOBLE linear layer with the CosNet branch: plain fp64 CPU oracle.
+ *
+ * TEST INFRASTRUCTURE ONLY.  Nothing on the product path may call, link or
+ * load this file; only the tests, the smoke check and the CPU-baseline leg of
+ * the benchmark do.  It shares no source with the CUDA library.
+ *
+ * Orientation follows the paper's Eq. 1 (Section 3.1) with row vectors:
+ *
+ *     y = x W + bias + sigma(x W_down) W_up
+ *     W      : [d_in][d_out]
+ *     W_down : [d_in][r]
+ *     W_up   : [r][d_out]
+ *
+ * and sigma is CosNet, Eq. 2 (Section 3.2) / Eqs. 5-7 (Appendix A):
+ *
+ *     h  = x W_down                    (bottleneck input, r wide)
+ *     u1 = omega1 * h + phi1           (elementwise)
+ *     a  = cos(u1)
+ *     b  = a M        b_j = sum_i a_i M[i][j]   (reading of "M . cos(...)")
+ *     u2 = omega2 * b + phi2
+ *     c  = cos(u2)    = sigma(h)
+ *
+ * Two further sigma modes exist only to pin the oracle:
+ *   ORACLE_IDENTITY: sigma(h) = h, where the branch collapses to
+ *                    x (W + W_down W_up)   (the LoRA remark in Section 1 and 3.1)
+ *   ORACLE_COS1:     sigma(h) = cos(omega1 * h + phi1), the single-cosine
+ *                    activation of the ablation in Section 4.4 (Table 5).
+ *
+ * The backward pass is the chain rule applied to the definitions above; the
+ * paper trains with autograd and never writes it out.  For a scalar loss
+ * L = sum_t sum_o y[t][o] * dy[t][o]:
+ *
+ *     dc      = dy W_up^T
+ *     du2     = -sin(u2) * dc
+ *     dphi2   = sum_t du2          domega2 = sum_t du2 * b
+ *     db      = omega2 * du2
+ *     dM      = sum_t a^T db       (dM[i][j] = sum_t a_i db_j)
+ *     da      = db M^T             (da_i = sum_j db_j M[i][j])
+ *     du1     = -sin(u1) * da
+ *     dphi1   = sum_t du1          domega1 = sum_t du1 * h
+ *     dh      = omega1 * du1
+ *     dx      = dy W^T + dh W_down^T
+ *     dW      = x^T dy     dbias = sum_t dy
+ *     dW_up   = c^T dy     dW_down = x^T dh
+ *
+ * Every sum runs over its index in ascending order.  Rows (tokens) are
+ * independent in the forward pass, so the only parallelism is over tokens for
+ * per-token outputs and over output rows for weight gradients; neither changes
+ * the order of any individual sum.
+ *
+ * Parity status: pinned (see the oracle tests): W_up = 0 reduction, identity
+ * collapse, linear-limit CosNet with random frequencies (fixes the orientation
+ * of M and where each omega/phi enters), closed-form cosine values,
+ * 2*pi periodicity in the phases, token permutation, and central finite
+ * differences for every gradient.
+ */
+#include <math.h>
+#include <stdint.h>
+#include <stdlib.h>
+#include <string.h>
+
+#define ORACLE_COSNET 0
+#define ORACLE_IDENTITY 1
+#define ORACLE_COS1 2
+
+/* sigma for one token, Eq. 2 / Eqs. 5-7.  Writes a, b, c (each [r]).  In the
+ * identity and single-cosine modes b is set equal to a (there is no M).      */
+static void sigma_token(int mode, int64_t r, const double *h,
+                        const double *om1, const double *ph1, const double *M,
+                        const double *om2, const double *ph2,
+                        double *a, double *b, double *c)
+{
+    int64_t i, j;
+    if (mode == ORACLE_IDENTITY) {
+        for (i = 0; i < r; ++i) { a[i] = h[i]; b[i] = h[i]; c[i] = h[i]; }
+        return;
+    }
+    for (i = 0; i < r; ++i) a[i] = cos(om1[i] * h[i] + ph1[i]);
+    if (mode == ORACLE_COS1) {
+        for (i = 0; i < r; ++i) { b[i] = a[i]; c[i] = a[i]; }
+        return;
+    }
+    for (j = 0; j < r; ++j) {
+        double s = 0.0;
+        for (i = 0; i < r; ++i) s += a[i] * M[i * r + j];
+        b[j] = s;
+    }
+    for (j = 0; j < r; ++j) c[j] = cos(om2[j] * b[j] + ph2[j]);
+}
+
+/*
+ * Forward pass, Eq. 1 with sigma from Eq. 2.
+ * x [T][d_in]; W [d_in][d_out]; bias [d_out] or NULL; W_down [d_in][r];
+ * om1, ph1, om2, ph2 [r]; M [r][r]; W_up [r][d_out].
+ * Outputs: y [T][d_out]; h, b, c [T][r] each (any may be NULL).
+ * r == 0 gives the plain layer x W + bias.
+ */
+void oracle_fwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
+                const double *x, const double *W, const double *bias,
+                const double *W_down, const double *om1, const double *ph1,
+                const double *M, const double *om2, const double *ph2,
+                const double *W_up, double *y, double *h_out, double *b_out,
+                double *c_out)
+{
+    int64_t t;
+#pragma omp parallel for schedule(static)
+    for (t = 0; t < T; ++t) {
+        const double *xt = x + t * d_in;
+        double *h = NULL, *a = NULL, *b = NULL, *c = NULL;
+        int64_t i, k, o;
+        if (r > 0) {
+            h = (double *)malloc(sizeof(double) * 4 * r);
+            a = h + r; b = a + r; c = b + r;
+            /* h = x W_down */
+            for (k = 0; k < r; ++k) {
+                double s = 0.0;
+                for (i = 0; i < d_in; ++i) s += xt[i] * W_down[i * r + k];
+                h[k] = s;
+            }
+            sigma_token(mode, r, h, om1, ph1, M, om2, ph2, a, b, c);
+            if (h_out) memcpy(h_out + t * r, h, sizeof(double) * r);
+            if (b_out) memcpy(b_out + t * r, b, sizeof(double) * r);
+            if (c_out) memcpy(c_out + t * r, c, sizeof(double) * r);
+        }
+        /* y = x W + bias + c W_up, each term summed in ascending index order */
+        for (o = 0; o < d_out; ++o) {
+            double s = 0.0, br = 0.0;
+            for (i = 0; i < d_in; ++i) s += xt[i] * W[i * d_out + o];
+            if (bias) s = s + bias[o];
+            for (k = 0; k < r; ++k) br += c[k] * W_up[k * d_out + o];
+            y[t * d_out + o] = s + br;
+        }
+        free(h);
+    }
+}
+
+/*
+ * Backward pass for L = sum(y * dy): the chain rule through Eq. 1 and Eq. 2,
+ * recomputing the forward intermediates from the inputs.
+ *
+ * Outputs (each may be NULL to skip it):
+ *   dx [T][d_in], dW [d_in][d_out], dbias [d_out], dW_down [d_in][r],
+ *   dM [r][r], dom1/dph1/dom2/dph2 [r], dW_up [r][d_out].
+ * Optional intermediates for sampled checks (each may be NULL), all [T][r]:
+ *   c_out (= sigma(h)), a_out, db_out, dh_out.
+ * In the identity and single-cosine modes the gradients of parameters that the
+ * mode does not use are written as zero.
+ */
+void oracle_bwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
+                const double *x, const double *W, const double *W_down,
+                const double *om1, const double *ph1, const double *M,
+                const double *om2, const double *ph2, const double *W_up,
+                const double *dy, double *dx, double *dW, double *dbias,
+                double *dW_down, double *dM, double *dom1, double *dph1,
+                double *dom2, double *dph2, double *dW_up, double *c_out,
+                double *a_out, double *db_out, double *dh_out)
+{
+    /* per-token intermediates, [T][r] each */
+    size_t n = (size_t)T * (size_t)(r > 0 ? r : 1);
+    double *H = (double *)calloc(n, sizeof(double));
+    double *U1 = (double *)calloc(n, sizeof(double));
+    double *A = (double *)calloc(n, sizeof(double));
+    double *B = (double *)calloc(n, sizeof(double));
+    double *C = (double *)calloc(n, sizeof(double));
+    double *DU1 = (double *)calloc(n, sizeof(double));
+    double *DU2 = (double *)calloc(n, sizeof(double));
+    double *DB = (double *)calloc(n, sizeof(double));
+    double *DH = (double *)calloc(n, sizeof(double));
+    int64_t t, i, j, k, o;
+
+    if (r > 0) {
+#pragma omp parallel for schedule(static) private(i, j, k, o)
+        for (t = 0; t < T; ++t) {
+            const double *xt = x + t * d_in;
+            const double *dyt = dy + t * d_out;
+            double *h = H + t * r, *u1 = U1 + t * r, *a = A + t * r;
+            double *b = B + t * r, *c = C + t * r;
+            double *du1 = DU1 + t * r, *du2 = DU2 + t * r;
+            double *db = DB + t * r, *dh = DH + t * r;
+            double *dc = (double *)malloc(sizeof(double) * 2 * r);
+            double *da = dc + r;
+            /* forward intermediates */
+            for (k = 0; k < r; ++k) {
+                double s = 0.0;
+                for (i = 0; i < d_in; ++i) s += xt[i] * W_down[i * r + k];
+                h[k] = s;
+            }
+            sigma_token(mode, r, h, om1, ph1, M, om2, ph2, a, b, c);
+            for (k = 0; k < r; ++k) u1[k] = om1 ? om1[k] * h[k] + ph1[k] : 0.0;
+            /* dc = dy W_up^T */
+            for (k = 0; k < r; ++k) {
+                double s = 0.0;
+                for (o = 0; o < d_out; ++o) s += dyt[o] * W_up[k * d_out + o];
+                dc[k] = s;
+            }
+            if (mode == ORACLE_IDENTITY) {
+                /* sigma(h) = h: dh = dc */
+                for (k = 0; k < r; ++k) dh[k] = dc[k];
+            } else if (mode == ORACLE_COS1) {
+                /* c = cos(u1): du1 = -sin(u1) dc, dh = omega1 du1 */
+                for (k = 0; k < r; ++k) {
+                    du1[k] = -sin(u1[k]) * dc[k];
+                    dh[k] = om1[k] * du1[k];
+                }
+            } else {
+                for (j = 0; j < r; ++j) {
+                    double u2 = om2[j] * b[j] + ph2[j];
+                    du2[j] = -sin(u2) * dc[j];
+                    db[j] = om2[j] * du2[j];
+                }
+                for (i = 0; i < r; ++i) {
+                    double s = 0.0;
+                    for (j = 0; j < r; ++j) s += db[j] * M[i * r + j];
+                    da[i] = s;
+                }
+                for (i = 0; i < r; ++i) {
+                    du1[i] = -sin(u1[i]) * da[i];
+                    dh[i] = om1[i] * du1[i];
+                }
+            }
+            free(dc);
+        }
+    }
+
+    /* dx = dy W^T + dh W_down^T */
+    if (dx) {
+#pragma omp parallel for schedule(static) private(i, k, o)
+        for (t = 0; t < T; ++t) {
+            for (i = 0; i < d_in; ++i) {
+                double s = 0.0, sb = 0.0;
+                for (o = 0; o < d_out; ++o) s += dy[t * d_out + o] * W[i * d_out + o];
+                for (k = 0; k < r; ++k) sb += DH[t * r + k] * W_down[i * r + k];
+                dx[t * d_in + i] = s + sb;
+            }
+        }
+    }
+    /* dW = x^T dy: dW[i][o] = sum_t x[t][i] dy[t][o] */
+    if (dW) {
+#pragma omp parallel for schedule(static) private(t, o)
+        for (i = 0; i < d_in; ++i) {
+            double *row = dW + i * d_out;
+            for (o = 0; o < d_out; ++o) row[o] = 0.0;
+            for (t = 0; t < T; ++t) {
+                double xv = x[t * d_in + i];
+                const double *dyt = dy + t * d_out;
+                for (o = 0; o < d_out; ++o) row[o] += xv * dyt[o];
+            }
+        }
+    }
+    if (dbias) {
+        for (o = 0; o < d_out; ++o) dbias[o] = 0.0;
+        for (t = 0; t < T; ++t)
+            for (o = 0; o < d_out; ++o) dbias[o] += dy[t * d_out + o];
+    }
+    /* dW_up = c^T dy */
+    if (dW_up && r > 0) {
+#pragma omp parallel for schedule(static) private(t, o)
+        for (k = 0; k < r; ++k) {
+            double *row = dW_up + k * d_out;
+            for (o = 0; o < d_out; ++o) row[o] = 0.0;
+            for (t = 0; t < T; ++t) {
+                double cv = C[t * r + k];
+                const double *dyt = dy + t * d_out;
+                for (o = 0; o < d_out; ++o) row[o] += cv * dyt[o];
+            }
+        }
+    }
+    /* dW_down = x^T dh */
+    if (dW_down && r > 0) {
+#pragma omp parallel for schedule(static) private(t, k)
+        for (i = 0; i < d_in; ++i) {
+            double *row = dW_down + i * r;
+            for (k = 0; k < r; ++k) row[k] = 0.0;
+            for (t = 0; t < T; ++t) {
+                double xv = x[t * d_in + i];
+                for (k = 0; k < r; ++k) row[k] += xv * DH[t * r + k];
+            }
+        }
+    }
+    /* dM = a^T db (zero when the mode has no M) */
+    if (dM && r > 0) {
+        for (i = 0; i < r * r; ++i) dM[i] = 0.0;
+        if (mode == ORACLE_COSNET)
+            for (t = 0; t < T; ++t)
+                for (i = 0; i < r; ++i)
+                    for (j = 0; j < r; ++j)
+                        dM[i * r + j] += A[t * r + i] * DB[t * r + j];
+    }
+    /* frequency and phase gradients: sums over tokens */
+    if (r > 0) {
+        for (k = 0; k < r; ++k) {
+            double so1 = 0.0, sp1 = 0.0, so2 = 0.0, sp2 = 0.0;
+            if (mode != ORACLE_IDENTITY) {
+                for (t = 0; t < T; ++t) {
+                    so1 += DU1[t * r + k] * H[t * r + k];
+                    sp1 += DU1[t * r + k];
+                }
+            }
+            if (mode == ORACLE_COSNET) {
+                for (t = 0; t < T; ++t) {
+                    so2 += DU2[t * r + k] * B[t * r + k];
+                    sp2 += DU2[t * r + k];
+                }
+            }
+            if (dom1) dom1[k] = so1;
+            if (dph1) dph1[k] = sp1;
+            if (dom2) dom2[k] = so2;
+            if (dph2) dph2[k] = sp2;
+        }
+        if (c_out) memcpy(c_out, C, sizeof(double) * n);
+        if (a_out) memcpy(a_out, A, sizeof(double) * n);
+        if (db_out) memcpy(db_out, DB, sizeof(double) * n);
+        if (dh_out) memcpy(dh_out, DH, sizeof(double) * n);
+    }
+    free(H); free(U1); free(A); free(B); free(C);
+    free(DU1); free(DU2); free(DB); free(DH);
+}
+
+/*
+ * Selected elements of a token-summed outer product:
+ *     out[p] = sum_t P[t][rows[p]] * Q[t][cols[p]]     (ascending t)
+ * P is [T][p_ld], Q is [T][q_ld].  This is the definition of one element of a
+ * weight gradient (x^T dy, c^T dy, x^T dh, a^T db), used to check sampled
+ * elements of large gradients without forming all of them.
+ */
+void oracle_outer_elems(int64_t T, const double *P, int64_t p_ld,
+                        const double *Q, int64_t q_ld, int64_t n,
+                        const int64_t *rows, const int64_t *cols, double *out)
+{
+    int64_t p;
+#pragma omp parallel for schedule(static)
+    for (p = 0; p < n; ++p) {
+        double s = 0.0;
+        int64_t t;
+        for (t = 0; t < T; ++t) s += P[t * p_ld + rows[p]] * Q[t * q_ld + cols[p]];
+        out[p] = s;
+    }
+}
