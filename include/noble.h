@@ -1,0 +1,188 @@
+/*
+ * noble.h -- C ABI of the NOBLE linear layer with the CosNet branch on GB300.
+ *
+ * The layer (NOBLE, arXiv 2603.06492, Eq. 1 in Section 3.1) is
+ *
+ *     y = x W^T + bias + sigma(x W_down^T) W_up^T
+ *
+ * written here with nn.Linear-style "out x in" weight storage, where the paper
+ * writes the same thing with row vectors as x W + b + sigma(x W_down) W_up.
+ * sigma is CosNet (Eq. 2 in Section 3.2; Eqs. 5-7 in Appendix A), applied per
+ * token to h = x W_down^T in R^r:
+ *
+ *     a = cos(omega1 * h + phi1)           elementwise, learnable omega1, phi1
+ *     b = a M          b_j = sum_i a_i M[i][j]
+ *     c = cos(omega2 * b + phi2)           elementwise, learnable omega2, phi2
+ *     sigma(h) = c
+ *
+ * Eq. 2 writes M . cos(...) for a column vector; this library reads it with
+ * row vectors as b = a M, i.e. M[i][j] couples input channel i to output
+ * channel j.  The backward pass is the chain rule through these definitions
+ * (the paper trains with autograd and does not write it out).
+ *
+ * Conventions shared by every entry point
+ * ---------------------------------------
+ *  - Every pointer argument is a DEVICE pointer on the current CUDA device,
+ *    except `desc`, which is a host pointer read during the call only.
+ *  - The caller owns and allocates every buffer; no entry point allocates or
+ *    frees device memory.  Cached TMA descriptors live in host memory.
+ *  - All tensors are dense, row-major and contiguous:
+ *        x [T][d_in]      y, dy [T][d_out]      dx [T][d_in]
+ *        W [d_out][d_in]  W_down [r][d_in]      W_up [d_out][r]
+ *        M [r][r]         omega1, phi1, omega2, phi2 [r]   bias [d_out]
+ *  - Operand dtype (x, W, W_down, W_up, y, dy, dx) is desc->dtype: bf16 or
+ *    fp32.  omega, phi, M, bias and every parameter gradient are always fp32.
+ *    bf16 operands use tensor cores with fp32 accumulation; fp32 operands use
+ *    exact fp32 FMA (no TF32), a validation mode.
+ *  - Calls are asynchronous on `stream` (a cudaStream_t; NULL = legacy
+ *    default stream).  Outputs are overwritten, never accumulated into.
+ *  - Arguments are checked on the host before anything is enqueued.  On an
+ *    argument error the call returns a status other than NOBLE_OK, enqueues
+ *    nothing and leaves every output untouched; noble_last_error() then
+ *    describes it.  NOBLE_ERR_CUDA from a failed launch part-way leaves the
+ *    outputs undefined.
+ *  - Requirements: T >= 0; d_in, d_out >= 8 and multiples of 8;
+ *    r in {0, 16, 32, 64, 128, 256} (r = 0 is the plain layer, and the branch
+ *    pointers may then be NULL); every pointer 16-byte aligned.
+ *  - Kernels never wait without a bound.  A wait that runs out records
+ *    NOBLE_ERR_TIMEOUT in a device status word, which
+ *    noble_get_device_status() reports.
+ */
+#ifndef NOBLE_H
+#define NOBLE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct CUstream_st *noble_stream; /* same type as cudaStream_t */
+
+typedef enum {
+    NOBLE_OK = 0,
+    NOBLE_ERR_INVALID_ARG = 1,     /* NULL pointer, negative or bad size      */
+    NOBLE_ERR_MISALIGNED = 2,      /* a pointer is not 16-byte aligned         */
+    NOBLE_ERR_UNSUPPORTED = 3,     /* r, d_in, d_out or dtype not supported    */
+    NOBLE_ERR_BUFFER_TOO_SMALL = 4,/* saved / workspace size below the query   */
+    NOBLE_ERR_CUDA = 5,            /* a CUDA runtime or driver call failed     */
+    NOBLE_ERR_TIMEOUT = 6,         /* a device-side bounded wait expired       */
+    NOBLE_ERR_NO_DEVICE = 7        /* no usable sm_103 device is current       */
+} noble_status;
+
+typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
+
+typedef struct {
+    int64_t T;      /* tokens (rows of x)                          */
+    int64_t d_in;   /* input features                              */
+    int64_t d_out;  /* output features                             */
+    int64_t r;      /* bottleneck rank; 0 = plain linear layer     */
+    int32_t dtype;  /* noble_dtype of the operands                 */
+    uint32_t flags; /* reserved, must be 0                         */
+} noble_linear_desc;
+
+/*
+ * Bytes of the saved-activation buffer that noble_linear_fwd writes and
+ * noble_linear_bwd reads (per token: h and b in fp32, c in the operand dtype,
+ * plus a copy of the mixing matrix).  0 when r == 0.  Returns 0 for an
+ * invalid descriptor as well; the entry points then report why.
+ */
+size_t noble_linear_saved_bytes(const noble_linear_desc *desc);
+
+/*
+ * Bytes of scratch memory noble_linear_bwd needs (dh in the operand dtype,
+ * dc and db in fp32, and fixed-size per-block partial sums for dM, domega
+ * and dphi).  Nonzero for every valid descriptor.
+ */
+size_t noble_linear_bwd_workspace_bytes(const noble_linear_desc *desc);
+
+/*
+ * Forward pass, Eq. 1 with sigma = CosNet (Eq. 2; Eqs. 5-7).
+ *   In : x, W, bias (NULL = no bias), W_down, omega1, phi1, M, omega2,
+ *        phi2, W_up.
+ *   Out: y [T][d_out] (operand dtype);
+ *        saved: `saved_bytes` >= noble_linear_saved_bytes(desc) bytes,
+ *        opaque, to be passed unchanged to noble_linear_bwd (may be NULL
+ *        when r == 0).  A smaller size returns NOBLE_ERR_BUFFER_TOO_SMALL.
+ */
+noble_status noble_linear_fwd(const noble_linear_desc *desc,
+                              const void *x, const void *W, const float *bias,
+                              const void *W_down, const float *omega1,
+                              const float *phi1, const float *M,
+                              const float *omega2, const float *phi2,
+                              const void *W_up, void *y, void *saved,
+                              size_t saved_bytes, noble_stream stream);
+
+/*
+ * Backward pass: gradients of L = sum(y * dy) by the chain rule through Eq. 1
+ * and Eq. 2.
+ *   In : dy [T][d_out] (operand dtype), the forward inputs, and `saved` as
+ *        written by noble_linear_fwd with the same desc and parameters.
+ *   Out: dx [T][d_in] (operand dtype);
+ *        dW [d_out][d_in], dbias [d_out] (NULL = skip), dW_down [r][d_in],
+ *        dM [r][r], domega1, dphi1, domega2, dphi2 [r], dW_up [d_out][r],
+ *        all fp32 (branch gradients may be NULL when r == 0).
+ *   workspace: `workspace_bytes` >= noble_linear_bwd_workspace_bytes(desc)
+ *        bytes of device scratch, contents undefined on entry and exit.
+ *        Smaller saved or workspace sizes return NOBLE_ERR_BUFFER_TOO_SMALL.
+ * The fp32 reductions over tokens (dM, domega, dphi, dbias) run in a fixed
+ * order, so repeated calls give bit-identical results.
+ */
+noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy,
+                              const void *x, const void *W,
+                              const void *W_down, const float *omega1,
+                              const float *phi1, const float *M,
+                              const float *omega2, const float *phi2,
+                              const void *W_up, const void *saved,
+                              size_t saved_bytes, void *dx,
+                              float *dW, float *dbias, float *dW_down,
+                              float *dM, float *domega1, float *dphi1,
+                              float *domega2, float *dphi2, float *dW_up,
+                              void *workspace, size_t workspace_bytes,
+                              noble_stream stream);
+
+/*
+ * Synchronises `stream`, then reads and clears the device status word of the
+ * current device.  NOBLE_ERR_TIMEOUT if any kernel gave up a bounded wait
+ * since the last call, NOBLE_ERR_CUDA if the stream reported an error,
+ * NOBLE_OK otherwise.
+ */
+noble_status noble_get_device_status(noble_stream stream);
+
+/* Static description of a status code. */
+const char *noble_status_string(noble_status s);
+
+/* Description of the last error returned on the calling thread ("" if none). */
+const char *noble_last_error(void);
+
+/* Number of kernels this library has launched in the process so far. */
+uint64_t noble_kernel_launch_count(void);
+
+/*
+ * Test hook: ORs `bits` into the current device's status word (synchronous),
+ * so that the reporting path of a device-side timeout can be exercised
+ * without making any kernel wait.
+ */
+noble_status noble_debug_raise_device_status(uint32_t bits);
+
+/*
+ * Instrumentation (no paper counterpart).  When enabled, every kernel the
+ * library launches is bracketed by two CUDA events on its own stream and
+ * attributed to a kernel class together with its algorithmic FLOPs and DRAM
+ * bytes.  noble_profile_count() waits for the recorded events, aggregates
+ * them and returns the number of classes; noble_profile_entry() reads class
+ * i of that snapshot (bound: 0 tensor pipe, 1 HBM, 2 CUDA-core ALU).
+ */
+void noble_profile_enable(int on);
+void noble_profile_reset(void);
+int noble_profile_count(void);
+noble_status noble_profile_entry(int i, char *name, size_t name_len,
+                                 uint64_t *launches, double *ms,
+                                 double *flops, double *bytes, int *bound);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* NOBLE_H */

@@ -1,0 +1,239 @@
+"""ctypes binding of ``libnoble.so`` (include/noble.h), plus thin torch helpers.
+
+Argument marshalling only: every step of the layer runs in the library's
+kernels.  There is no fallback: if the library is missing or cannot run on the
+current device the call raises.
+
+Functions with the C names take device pointers given as ints, torch tensors
+or None.  ``NobleLinearBuffers`` / ``forward`` / ``backward`` allocate the
+caller-owned buffers with torch and call the same entry points.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import re
+import threading
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libnoble.so")
+HEADER = os.path.join(os.path.dirname(HERE), "include", "noble.h")
+
+NOBLE_BF16, NOBLE_FP32 = 0, 1
+STATUS = {0: "NOBLE_OK", 1: "NOBLE_ERR_INVALID_ARG", 2: "NOBLE_ERR_MISALIGNED",
+          3: "NOBLE_ERR_UNSUPPORTED", 4: "NOBLE_ERR_BUFFER_TOO_SMALL", 5: "NOBLE_ERR_CUDA",
+          6: "NOBLE_ERR_TIMEOUT", 7: "NOBLE_ERR_NO_DEVICE"}
+
+
+class NobleError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{STATUS.get(status, status)}: {msg}")
+        self.status = status
+
+
+class Desc(ctypes.Structure):
+    _fields_ = [("T", ctypes.c_int64), ("d_in", ctypes.c_int64), ("d_out", ctypes.c_int64),
+                ("r", ctypes.c_int64), ("dtype", ctypes.c_int32), ("flags", ctypes.c_uint32)]
+
+
+def make_desc(T, d_in, d_out, r, dtype) -> Desc:
+    if isinstance(dtype, str):
+        dtype = {"bf16": NOBLE_BF16, "fp32": NOBLE_FP32}[dtype]
+    return Desc(T, d_in, d_out, r, dtype, 0)
+
+
+_lib = None
+_lock = threading.Lock()
+
+
+def declared_functions() -> list[str]:
+    """Names of the functions include/noble.h declares."""
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(noble_[a-z_0-9]+)\s*\(", src)))
+
+
+def load(path: str | None = None) -> ctypes.CDLL:
+    """Load the library (once).  Raises if it has not been built."""
+    global _lib
+    with _lock:
+        if _lib is not None:
+            return _lib
+        path = path or LIB_PATH
+        if not os.path.exists(path):
+            raise RuntimeError(f"{path} is missing: build it with paper_2603_06492_gb300.build.build()")
+        lib = ctypes.CDLL(path)
+        P, S, D = ctypes.c_void_p, ctypes.c_size_t, ctypes.POINTER(Desc)
+        lib.noble_linear_saved_bytes.argtypes = [D]
+        lib.noble_linear_saved_bytes.restype = S
+        lib.noble_linear_bwd_workspace_bytes.argtypes = [D]
+        lib.noble_linear_bwd_workspace_bytes.restype = S
+        lib.noble_linear_fwd.argtypes = [D] + [P] * 12 + [S, P]
+        lib.noble_linear_fwd.restype = ctypes.c_int
+        lib.noble_linear_bwd.argtypes = [D] + [P] * 11 + [S] + [P] * 11 + [S, P]
+        lib.noble_linear_bwd.restype = ctypes.c_int
+        lib.noble_get_device_status.argtypes = [P]
+        lib.noble_get_device_status.restype = ctypes.c_int
+        lib.noble_status_string.argtypes = [ctypes.c_int]
+        lib.noble_status_string.restype = ctypes.c_char_p
+        lib.noble_last_error.argtypes = []
+        lib.noble_last_error.restype = ctypes.c_char_p
+        lib.noble_kernel_launch_count.argtypes = []
+        lib.noble_kernel_launch_count.restype = ctypes.c_uint64
+        lib.noble_debug_raise_device_status.argtypes = [ctypes.c_uint32]
+        lib.noble_debug_raise_device_status.restype = ctypes.c_int
+        lib.noble_profile_enable.argtypes = [ctypes.c_int]
+        lib.noble_profile_enable.restype = None
+        lib.noble_profile_reset.argtypes = []
+        lib.noble_profile_reset.restype = None
+        lib.noble_profile_count.argtypes = []
+        lib.noble_profile_count.restype = ctypes.c_int
+        lib.noble_profile_entry.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_size_t] + [P] * 5
+        lib.noble_profile_entry.restype = ctypes.c_int
+        _lib = lib
+        return lib
+
+
+def _p(a):
+    """Pointer value of a torch tensor, an int or None."""
+    if a is None:
+        return None
+    if isinstance(a, int):
+        return a
+    return a.data_ptr()
+
+
+def _check(status: int):
+    if status != 0:
+        lib = load()
+        raise NobleError(status, lib.noble_last_error().decode() or
+                         lib.noble_status_string(status).decode())
+
+
+def noble_linear_saved_bytes(desc: Desc) -> int:
+    return load().noble_linear_saved_bytes(ctypes.byref(desc))
+
+
+def noble_linear_bwd_workspace_bytes(desc: Desc) -> int:
+    return load().noble_linear_bwd_workspace_bytes(ctypes.byref(desc))
+
+
+def noble_linear_fwd(desc, x, W, bias, W_down, omega1, phi1, M, omega2, phi2, W_up, y, saved,
+                     saved_bytes, stream):
+    _check(load().noble_linear_fwd(ctypes.byref(desc), _p(x), _p(W), _p(bias), _p(W_down),
+                                   _p(omega1), _p(phi1), _p(M), _p(omega2), _p(phi2), _p(W_up),
+                                   _p(y), _p(saved), saved_bytes, stream))
+
+
+def noble_linear_bwd(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up, saved,
+                     saved_bytes, dx, dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2,
+                     dW_up, workspace, workspace_bytes, stream):
+    _check(load().noble_linear_bwd(ctypes.byref(desc), _p(dy), _p(x), _p(W), _p(W_down),
+                                   _p(omega1), _p(phi1), _p(M), _p(omega2), _p(phi2), _p(W_up),
+                                   _p(saved), saved_bytes, _p(dx), _p(dW), _p(dbias), _p(dW_down),
+                                   _p(dM), _p(domega1), _p(dphi1), _p(domega2), _p(dphi2),
+                                   _p(dW_up), _p(workspace), workspace_bytes, stream))
+
+
+def noble_get_device_status(stream=None):
+    _check(load().noble_get_device_status(stream))
+
+
+def noble_kernel_launch_count() -> int:
+    return load().noble_kernel_launch_count()
+
+
+def noble_debug_raise_device_status(bits: int):
+    _check(load().noble_debug_raise_device_status(bits))
+
+
+def profile_read() -> dict:
+    """Per-kernel-class totals recorded since the last reset (see noble.h)."""
+    lib = load()
+    n = lib.noble_profile_count()
+    out = {}
+    for i in range(n):
+        name = ctypes.create_string_buffer(128)
+        launches, bound = ctypes.c_uint64(), ctypes.c_int()
+        ms, flops, nbytes = ctypes.c_double(), ctypes.c_double(), ctypes.c_double()
+        _check(lib.noble_profile_entry(i, name, 128, ctypes.byref(launches), ctypes.byref(ms),
+                                       ctypes.byref(flops), ctypes.byref(nbytes), ctypes.byref(bound)))
+        out[name.value.decode()] = {"name": name.value.decode(), "launches": launches.value,
+                                    "ms": ms.value, "flops": flops.value, "bytes": nbytes.value,
+                                    "bound": {0: "tensor", 1: "hbm", 2: "alu"}[bound.value]}
+    return out
+
+
+# ---------------------------------------------------------------- torch side
+PARAM_NAMES = ("W", "bias", "W_down", "omega1", "phi1", "M", "omega2", "phi2", "W_up")
+GRAD_NAMES = ("dW", "dbias", "dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2", "dW_up")
+
+
+def _stream_handle(stream):
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+class NobleLinearBuffers:
+    """Caller-owned device buffers for one layer shape (allocated with torch)."""
+
+    def __init__(self, T, d_in, d_out, r, dtype, device="cuda", with_grads=True):
+        import torch
+        self.desc = make_desc(T, d_in, d_out, r, dtype)
+        tdt = torch.bfloat16 if self.desc.dtype == NOBLE_BF16 else torch.float32
+        self.saved_bytes = noble_linear_saved_bytes(self.desc)
+        self.workspace_bytes = noble_linear_bwd_workspace_bytes(self.desc)
+        self.y = torch.empty((T, d_out), dtype=tdt, device=device)
+        self.saved = (torch.empty(self.saved_bytes, dtype=torch.uint8, device=device)
+                      if self.saved_bytes else None)
+        if with_grads:
+            f32 = dict(dtype=torch.float32, device=device)
+            self.dx = torch.empty((T, d_in), dtype=tdt, device=device)
+            self.workspace = torch.empty(self.workspace_bytes, dtype=torch.uint8, device=device)
+            self.grads = {"dW": torch.empty((d_out, d_in), **f32),
+                          "dbias": torch.empty(d_out, **f32)}
+            if r > 0:
+                self.grads.update({"dW_down": torch.empty((r, d_in), **f32),
+                                   "dM": torch.empty((r, r), **f32),
+                                   "domega1": torch.empty(r, **f32),
+                                   "dphi1": torch.empty(r, **f32),
+                                   "domega2": torch.empty(r, **f32),
+                                   "dphi2": torch.empty(r, **f32),
+                                   "dW_up": torch.empty((d_out, r), **f32)})
+
+
+def forward(buf: NobleLinearBuffers, x, params: dict, stream=None):
+    """y = NOBLE(x) into ``buf.y``; saves activations in ``buf.saved``."""
+    p = params
+    noble_linear_fwd(buf.desc, x, p["W"], p.get("bias"), p.get("W_down"), p.get("omega1"),
+                     p.get("phi1"), p.get("M"), p.get("omega2"), p.get("phi2"), p.get("W_up"),
+                     buf.y, buf.saved, buf.saved_bytes, _stream_handle(stream))
+    return buf.y
+
+
+def backward(buf: NobleLinearBuffers, x, dy, params: dict, stream=None, with_dbias=True):
+    """dx into ``buf.dx`` and parameter gradients into ``buf.grads``."""
+    p, g = params, buf.grads
+    noble_linear_bwd(buf.desc, dy, x, p["W"], p.get("W_down"), p.get("omega1"), p.get("phi1"),
+                     p.get("M"), p.get("omega2"), p.get("phi2"), p.get("W_up"), buf.saved,
+                     buf.saved_bytes, buf.dx, g["dW"], g["dbias"] if with_dbias else None,
+                     g.get("dW_down"), g.get("dM"), g.get("domega1"), g.get("dphi1"),
+                     g.get("domega2"), g.get("dphi2"), g.get("dW_up"), buf.workspace,
+                     buf.workspace_bytes, _stream_handle(stream))
+    return buf.dx, g
+
+
+def params_to_device(inp: dict, dtype: str, device="cuda") -> dict:
+    """Move numpy inputs (library layout, see inputs.py) to device tensors:
+    operands in ``dtype``, omega/phi/M/bias in fp32."""
+    import numpy as np
+    import torch
+    tdt = torch.bfloat16 if dtype == "bf16" else torch.float32
+    out = {}
+    for k, v in inp.items():
+        t = torch.from_numpy(np.ascontiguousarray(v, dtype=np.float32))
+        if k in ("x", "W", "W_down", "W_up", "dy"):
+            t = t.to(tdt)
+        out[k] = t.to(device)
+    return out

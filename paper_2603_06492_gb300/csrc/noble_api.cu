@@ -1,0 +1,460 @@
+// C-ABI entry points of the NOBLE linear layer (declared in include/noble.h).
+//
+// Host side only: argument validation, buffer carving and kernel dispatch.
+// Forward = Eq. 1 (Section 3.1) with CosNet (Eq. 2, Section 3.2; Eqs. 5-7,
+// Appendix A); backward = the chain rule through the same definitions.
+#include <atomic>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+
+#include "../../include/noble.h"
+#include "common.cuh"
+#include "profile.cuh"
+#include "simt.cuh"
+#include "tc_path.cuh"
+
+namespace noble {
+
+__device__ uint32_t g_device_status = 0;
+
+namespace {
+
+thread_local char g_last_error[512] = "";
+std::atomic<uint64_t> g_launches{0};
+
+noble_status fail(noble_status s, const char *fmt, ...)
+{
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_last_error, sizeof(g_last_error), fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+noble_status check_launch(const char *what)
+{
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(NOBLE_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+    return NOBLE_OK;
+}
+
+// Launch through `f`, bracketed by profiling events when profiling is on.
+template <class F>
+noble_status run(cudaStream_t st, const KernelInfo &ki, F &&f)
+{
+    const int slot = Profiler::get().begin(st);
+    f();
+    Profiler::get().end(slot, st, ki);
+    return check_launch(ki.name);
+}
+
+#define NOBLE_TRY(expr)                              \
+    do {                                             \
+        noble_status _s = (expr);                    \
+        if (_s != NOBLE_OK) return _s;               \
+    } while (0)
+
+bool rank_supported(int64_t r) { return r == 0 || r == 16 || r == 32 || r == 64 || r == 128 || r == 256; }
+
+noble_status validate_desc(const noble_linear_desc *d)
+{
+    if (!d) return fail(NOBLE_ERR_INVALID_ARG, "desc is NULL");
+    if (d->T < 0 || d->d_in <= 0 || d->d_out <= 0 || d->r < 0)
+        return fail(NOBLE_ERR_INVALID_ARG, "negative or zero size (T=%lld d_in=%lld d_out=%lld r=%lld)",
+                    (long long)d->T, (long long)d->d_in, (long long)d->d_out, (long long)d->r);
+    if (d->T > (int64_t)INT32_MAX || d->d_in > (1 << 20) || d->d_out > (1 << 20))
+        return fail(NOBLE_ERR_UNSUPPORTED, "size too large (T <= 2^31-1, d_in/d_out <= 2^20)");
+    if (d->d_in < 8 || d->d_out < 8 || d->d_in % 8 || d->d_out % 8)
+        return fail(NOBLE_ERR_UNSUPPORTED, "d_in=%lld and d_out=%lld must be multiples of 8 and >= 8",
+                    (long long)d->d_in, (long long)d->d_out);
+    if (!rank_supported(d->r))
+        return fail(NOBLE_ERR_UNSUPPORTED, "r=%lld not in {0,16,32,64,128,256}", (long long)d->r);
+    if (d->dtype != NOBLE_BF16 && d->dtype != NOBLE_FP32)
+        return fail(NOBLE_ERR_UNSUPPORTED, "dtype %d not supported", (int)d->dtype);
+    if (d->flags != 0) return fail(NOBLE_ERR_UNSUPPORTED, "flags must be 0");
+    return NOBLE_OK;
+}
+
+noble_status check_ptr(const void *p, const char *name, bool nullable)
+{
+    if (!p) return nullable ? NOBLE_OK : fail(NOBLE_ERR_INVALID_ARG, "%s is NULL", name);
+    if (reinterpret_cast<uintptr_t>(p) % 16) return fail(NOBLE_ERR_MISALIGNED, "%s is not 16-byte aligned", name);
+    return NOBLE_OK;
+}
+
+noble_status check_device()
+{
+    static int cached[64];  // 0 unknown, 1 ok, 2 bad
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) {
+        cudaGetLastError();
+        return fail(NOBLE_ERR_NO_DEVICE, "no current CUDA device");
+    }
+    if (dev < 64 && cached[dev] == 1) return NOBLE_OK;
+    int major = 0, minor = 0;
+    cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev);
+    cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev);
+    cudaGetLastError();
+    if (major != 10 || minor != 3) {
+        if (dev < 64) cached[dev] = 2;
+        return fail(NOBLE_ERR_NO_DEVICE, "device %d is sm_%d%d; this library is built for sm_103a", dev, major, minor);
+    }
+    if (dev < 64) cached[dev] = 1;
+    return NOBLE_OK;
+}
+
+size_t esize(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 ? 2 : 4; }
+
+// Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r].
+struct SavedLayout {
+    size_t h, b, c, total;
+};
+SavedLayout saved_layout(const noble_linear_desc *d)
+{
+    SavedLayout L{};
+    if (d->r == 0) return L;
+    const size_t tr = (size_t)d->T * (size_t)d->r;
+    L.h = 0;
+    L.b = align_up(L.h + tr * 4, 256);
+    L.c = align_up(L.b + tr * 4, 256);
+    L.total = align_up(L.c + tr * esize(d), 256);
+    return L;
+}
+
+constexpr int64_t kDmChunk = 1024;     // tokens per dM partial
+constexpr int64_t kBiasChunk = 512;    // tokens per dbias partial
+int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
+
+// Backward scratch: dh (dtype), dc, a, db (fp32) [T][r]; Mt fp32 [r][r];
+// per-block partials of the CosNet sums, of dM and of dbias.
+struct WorkLayout {
+    size_t dh, dc, a, db, mt, cos_part, dm_part, bias_part, total;
+    int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
+};
+WorkLayout work_layout(const noble_linear_desc *d)
+{
+    WorkLayout L{};
+    const int64_t T = d->T, r = d->r;
+    const size_t tr = (size_t)T * (size_t)r;
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
+    L.dh = take(tr * esize(d));
+    L.dc = take(tr * 4);
+    L.a = take(tr * 4);
+    L.db = take(tr * 4);
+    L.mt = take((size_t)r * r * 4);
+    L.n_cos_blocks = r ? ceil_div(T, cosnet_tokens_per_block(r)) : 0;
+    L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
+    L.n_dm_chunks = r ? ceil_div(T, kDmChunk) : 0;
+    L.dm_part = take((size_t)L.n_dm_chunks * r * r * 4);
+    L.n_bias_chunks = ceil_div(T, kBiasChunk);
+    L.bias_part = take((size_t)L.n_bias_chunks * d->d_out * 4);
+    L.total = off < 256 ? 256 : off;
+    return L;
+}
+
+// ------------------------------------------------------------ SIMT dispatch
+template <typename TIn, typename TOut>
+noble_status simt_gemm(cudaStream_t st, int64_t M, int64_t N, simt::Seg s0, const simt::Seg *s1,
+                       const float *bias, TOut *C, int64_t ldc, int64_t k_chunk = 0,
+                       int64_t n_chunks = 1, int64_t c_chunk_stride = 0)
+{
+    if (M == 0 || N == 0) return NOBLE_OK;
+    dim3 grid((unsigned)ceil_div(N, simt::kBN), (unsigned)ceil_div(M, simt::kBM), (unsigned)n_chunks);
+    simt::Seg empty{};
+    const double K = (double)s0.K + (s1 ? (double)s1->K : 0.0);
+    const KernelInfo ki{"simt_gemm", kBoundAlu, 2.0 * M * N * K, 0.0};
+    return run(st, ki, [&] {
+        simt::gemm_kernel<TIn, TOut><<<grid, simt::kThreads, 0, st>>>(
+            M, N, s0, s1 ? *s1 : empty, s1 ? 2 : 1, bias, C, ldc, k_chunk, c_chunk_stride);
+    });
+}
+
+noble_status reduce(cudaStream_t st, int64_t nparts, int64_t n, int64_t seg_len, const float *part,
+                    float *o0, float *o1 = nullptr, float *o2 = nullptr, float *o3 = nullptr)
+{
+    simt::Outs4 outs{{o0, o1, o2, o3}};
+    const KernelInfo ki{"reduce_partials", kBoundHbm, (double)nparts * n, 4.0 * (nparts + 1) * n};
+    return run(st, ki, [&] {
+        simt::reduce_partials<<<(unsigned)ceil_div(n, 256), 256, 0, st>>>(nparts, n, seg_len, part, outs);
+    });
+}
+
+template <typename TIn>
+noble_status fwd_simt(const noble_linear_desc *d, const TIn *x, const TIn *W, const float *bias,
+                      const TIn *W_down, const float *om1, const float *ph1, const float *M,
+                      const float *om2, const float *ph2, const TIn *W_up, TIn *y, char *saved,
+                      cudaStream_t st)
+{
+    const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
+    const SavedLayout SL = saved_layout(d);
+    float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
+    TIn *c = (TIn *)(saved + SL.c);
+    simt::Seg main{{x, di, 1}, {W, di, 1}, di};
+    if (r > 0) {
+        simt::Seg down{{x, di, 1}, {W_down, di, 1}, di};
+        NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, down, nullptr, nullptr, h, r)));
+        const int tpb = cosnet_tokens_per_block(r);
+        const KernelInfo ki{"simt_cosnet_fwd", kBoundAlu, 2.0 * T * r * r, 0.0};
+        NOBLE_TRY(run(st, ki, [&] {
+            simt::cosnet_fwd_rows<TIn><<<(unsigned)ceil_div(T, tpb), 256, tpb * r * sizeof(float), st>>>(
+                T, (int)r, tpb, h, om1, ph1, M, om2, ph2, b, c);
+        }));
+        simt::Seg up{{c, r, 1}, {W_up, r, 1}, r};
+        return simt_gemm<TIn, TIn>(st, T, dout, main, &up, bias, y, dout);
+    }
+    return simt_gemm<TIn, TIn>(st, T, dout, main, nullptr, bias, y, dout);
+}
+
+template <typename TIn>
+noble_status bwd_simt(const noble_linear_desc *d, const TIn *dy, const TIn *x, const TIn *W,
+                      const TIn *W_down, const float *om1, const float *ph1, const float *M,
+                      const float *om2, const float *ph2, const TIn *W_up, const char *saved,
+                      TIn *dx, float *dW, float *dbias, float *dW_down, float *dM, float *dom1,
+                      float *dph1, float *dom2, float *dph2, float *dW_up, char *ws, cudaStream_t st)
+{
+    const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
+    const SavedLayout SL = saved_layout(d);
+    const WorkLayout WL = work_layout(d);
+    const float *h = (const float *)(saved + SL.h), *b = (const float *)(saved + SL.b);
+    const TIn *c = (const TIn *)(saved + SL.c);
+    TIn *dh = (TIn *)(ws + WL.dh);
+    if (r > 0) {
+        float *dc = (float *)(ws + WL.dc), *a = (float *)(ws + WL.a), *db = (float *)(ws + WL.db);
+        float *Mt = (float *)(ws + WL.mt), *cpart = (float *)(ws + WL.cos_part);
+        float *dmpart = (float *)(ws + WL.dm_part);
+        const KernelInfo kt{"transpose_M", kBoundHbm, 0.0, 8.0 * r * r};
+        NOBLE_TRY(run(st, kt, [&] {
+            simt::transpose_square<<<(unsigned)ceil_div(r * r, 256), 256, 0, st>>>((int)r, M, Mt);
+        }));
+        // dc = dy W_up
+        simt::Seg sdc{{dy, dout, 1}, {W_up, 1, r}, dout};
+        NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, sdc, nullptr, nullptr, dc, r)));
+        const int tpb = cosnet_tokens_per_block(r);
+        const KernelInfo kc{"simt_cosnet_bwd", kBoundAlu, 2.0 * T * r * r, 0.0};
+        NOBLE_TRY(run(st, kc, [&] {
+            simt::cosnet_bwd_rows<TIn><<<(unsigned)WL.n_cos_blocks, 256, 5 * tpb * r * sizeof(float), st>>>(
+                T, (int)r, tpb, h, b, dc, om1, ph1, Mt, om2, ph2, dh, a, db, cpart);
+        }));
+        NOBLE_TRY(reduce(st, WL.n_cos_blocks, 4 * r, r, cpart, dom1, dph1, dom2, dph2));
+        // dM = a^T db, fixed token chunks
+        simt::Seg sdm{{a, 1, r}, {db, 1, r}, T};
+        NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
+                                           WL.n_dm_chunks, r * r)));
+        NOBLE_TRY(reduce(st, WL.n_dm_chunks, r * r, r * r, dmpart, dM));
+        // dW_up = dy^T c ; dW_down = dh^T x
+        simt::Seg sup{{dy, 1, dout}, {c, 1, r}, T};
+        NOBLE_TRY((simt_gemm<TIn, float>(st, dout, r, sup, nullptr, nullptr, dW_up, r)));
+        simt::Seg sdn{{dh, 1, r}, {x, 1, di}, T};
+        NOBLE_TRY((simt_gemm<TIn, float>(st, r, di, sdn, nullptr, nullptr, dW_down, di)));
+    }
+    // dx = dy W + dh W_down
+    simt::Seg sdx{{dy, dout, 1}, {W, 1, di}, dout};
+    simt::Seg sdx2{{dh, r, 1}, {W_down, 1, di}, r};
+    NOBLE_TRY((simt_gemm<TIn, TIn>(st, T, di, sdx, r > 0 ? &sdx2 : nullptr, nullptr, dx, di)));
+    // dW = dy^T x
+    simt::Seg sdw{{dy, 1, dout}, {x, 1, di}, T};
+    NOBLE_TRY((simt_gemm<TIn, float>(st, dout, di, sdw, nullptr, nullptr, dW, di)));
+    if (dbias) {
+        float *bpart = (float *)(ws + WL.bias_part);
+        dim3 grid((unsigned)ceil_div(dout, 256), (unsigned)WL.n_bias_chunks);
+        const KernelInfo kb{"colsum_dbias", kBoundHbm, (double)T * dout, (double)T * dout * sizeof(TIn)};
+        NOBLE_TRY(run(st, kb, [&] {
+            simt::colsum_partial<TIn><<<grid, 256, 0, st>>>(T, dout, kBiasChunk, dy, bpart);
+        }));
+        NOBLE_TRY(reduce(st, WL.n_bias_chunks, dout, dout, bpart, dbias));
+    }
+    return NOBLE_OK;
+}
+
+noble_status zero_grads(const noble_linear_desc *d, float *dW, float *dbias, float *dW_down, float *dM,
+                        float *dom1, float *dph1, float *dom2, float *dph2, float *dW_up,
+                        cudaStream_t st)
+{
+    const size_t di = d->d_in, dout = d->d_out, r = d->r;
+    struct { void *p; size_t n; } z[] = {{dW, di * dout}, {dbias, dout}, {dW_down, r * di}, {dM, r * r},
+                                        {dom1, r}, {dph1, r}, {dom2, r}, {dph2, r}, {dW_up, dout * r}};
+    for (auto &e : z)
+        if (e.p && e.n && cudaMemsetAsync(e.p, 0, e.n * 4, st) != cudaSuccess)
+            return fail(NOBLE_ERR_CUDA, "cudaMemsetAsync: %s", cudaGetErrorString(cudaGetLastError()));
+    return NOBLE_OK;
+}
+
+}  // namespace
+}  // namespace noble
+
+using namespace noble;
+
+extern "C" {
+
+size_t noble_linear_saved_bytes(const noble_linear_desc *desc)
+{
+    if (validate_desc(desc) != NOBLE_OK) return 0;
+    return saved_layout(desc).total;
+}
+
+size_t noble_linear_bwd_workspace_bytes(const noble_linear_desc *desc)
+{
+    if (validate_desc(desc) != NOBLE_OK) return 0;
+    return work_layout(desc).total;
+}
+
+noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, const void *W,
+                              const float *bias, const void *W_down, const float *omega1,
+                              const float *phi1, const float *M, const float *omega2,
+                              const float *phi2, const void *W_up, void *y, void *saved,
+                              size_t saved_bytes, noble_stream stream)
+{
+    g_last_error[0] = 0;
+    NOBLE_TRY(validate_desc(desc));
+    const bool br = desc->r > 0;
+    NOBLE_TRY(check_ptr(x, "x", false));
+    NOBLE_TRY(check_ptr(W, "W", false));
+    NOBLE_TRY(check_ptr(bias, "bias", true));
+    NOBLE_TRY(check_ptr(y, "y", false));
+    NOBLE_TRY(check_ptr(W_down, "W_down", !br));
+    NOBLE_TRY(check_ptr(omega1, "omega1", !br));
+    NOBLE_TRY(check_ptr(phi1, "phi1", !br));
+    NOBLE_TRY(check_ptr(M, "M", !br));
+    NOBLE_TRY(check_ptr(omega2, "omega2", !br));
+    NOBLE_TRY(check_ptr(phi2, "phi2", !br));
+    NOBLE_TRY(check_ptr(W_up, "W_up", !br));
+    NOBLE_TRY(check_ptr(saved, "saved", !br));
+    if (saved_bytes < saved_layout(desc).total)
+        return fail(NOBLE_ERR_BUFFER_TOO_SMALL, "saved_bytes=%zu < %zu", saved_bytes, saved_layout(desc).total);
+    NOBLE_TRY(check_device());
+    if (desc->T == 0) return NOBLE_OK;
+    cudaStream_t st = (cudaStream_t)stream;
+    if (desc->dtype == NOBLE_BF16) {
+        using bf = __nv_bfloat16;
+        if (tc::fwd_supported(desc))
+            return tc::fwd(desc, (const bf *)x, (const bf *)W, bias, (const bf *)W_down, omega1, phi1, M,
+                           omega2, phi2, (const bf *)W_up, (bf *)y, (char *)saved, st, g_launches);
+        return fwd_simt<bf>(desc, (const bf *)x, (const bf *)W, bias, (const bf *)W_down, omega1, phi1, M,
+                            omega2, phi2, (const bf *)W_up, (bf *)y, (char *)saved, st);
+    }
+    return fwd_simt<float>(desc, (const float *)x, (const float *)W, bias, (const float *)W_down, omega1,
+                           phi1, M, omega2, phi2, (const float *)W_up, (float *)y, (char *)saved, st);
+}
+
+noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, const void *x,
+                              const void *W, const void *W_down, const float *omega1,
+                              const float *phi1, const float *M, const float *omega2,
+                              const float *phi2, const void *W_up, const void *saved,
+                              size_t saved_bytes, void *dx,
+                              float *dW, float *dbias, float *dW_down, float *dM, float *domega1,
+                              float *dphi1, float *domega2, float *dphi2, float *dW_up,
+                              void *workspace, size_t workspace_bytes, noble_stream stream)
+{
+    g_last_error[0] = 0;
+    NOBLE_TRY(validate_desc(desc));
+    const bool br = desc->r > 0;
+    const char *names[] = {"dy", "x", "W", "dx", "dW", "workspace"};
+    const void *req[] = {dy, x, W, dx, dW, workspace};
+    for (int i = 0; i < 6; ++i) NOBLE_TRY(check_ptr(req[i], names[i], false));
+    NOBLE_TRY(check_ptr(dbias, "dbias", true));
+    const char *bnames[] = {"W_down", "omega1", "phi1", "M", "omega2", "phi2", "W_up", "saved",
+                            "dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2", "dW_up"};
+    const void *bptr[] = {W_down, omega1, phi1, M, omega2, phi2, W_up, saved,
+                          dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up};
+    for (int i = 0; i < 15; ++i) NOBLE_TRY(check_ptr(bptr[i], bnames[i], !br));
+    if (saved_bytes < saved_layout(desc).total)
+        return fail(NOBLE_ERR_BUFFER_TOO_SMALL, "saved_bytes=%zu < %zu", saved_bytes, saved_layout(desc).total);
+    if (workspace_bytes < work_layout(desc).total)
+        return fail(NOBLE_ERR_BUFFER_TOO_SMALL, "workspace_bytes=%zu < %zu", workspace_bytes,
+                    work_layout(desc).total);
+    NOBLE_TRY(check_device());
+    cudaStream_t st = (cudaStream_t)stream;
+    if (desc->T == 0)
+        return zero_grads(desc, dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, st);
+    if (desc->dtype == NOBLE_BF16) {
+        using bf = __nv_bfloat16;
+        if (tc::bwd_supported(desc))
+            return tc::bwd(desc, (const bf *)dy, (const bf *)x, (const bf *)W, (const bf *)W_down, omega1, phi1,
+                           M, omega2, phi2, (const bf *)W_up, (const char *)saved, (bf *)dx, dW, dbias,
+                           dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace, st,
+                           g_launches);
+        return bwd_simt<bf>(desc, (const bf *)dy, (const bf *)x, (const bf *)W, (const bf *)W_down, omega1,
+                            phi1, M, omega2, phi2, (const bf *)W_up, (const char *)saved, (bf *)dx, dW,
+                            dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace,
+                            st);
+    }
+    return bwd_simt<float>(desc, (const float *)dy, (const float *)x, (const float *)W, (const float *)W_down,
+                           omega1, phi1, M, omega2, phi2, (const float *)W_up, (const char *)saved,
+                           (float *)dx, dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up,
+                           (char *)workspace, st);
+}
+
+noble_status noble_get_device_status(noble_stream stream)
+{
+    g_last_error[0] = 0;
+    cudaError_t e = cudaStreamSynchronize((cudaStream_t)stream);
+    if (e != cudaSuccess) return fail(NOBLE_ERR_CUDA, "stream: %s", cudaGetErrorString(e));
+    uint32_t v = 0, zero = 0;
+    e = cudaMemcpyFromSymbol(&v, g_device_status, sizeof(v));
+    if (e == cudaSuccess && v) e = cudaMemcpyToSymbol(g_device_status, &zero, sizeof(zero));
+    if (e != cudaSuccess) return fail(NOBLE_ERR_CUDA, "status word: %s", cudaGetErrorString(e));
+    if (v & kStatusTimeout) return fail(NOBLE_ERR_TIMEOUT, "a kernel gave up a bounded wait (status 0x%x)", v);
+    if (v) return fail(NOBLE_ERR_CUDA, "device status 0x%x", v);
+    return NOBLE_OK;
+}
+
+noble_status noble_debug_raise_device_status(uint32_t bits)
+{
+    uint32_t v = 0;
+    cudaError_t e = cudaMemcpyFromSymbol(&v, g_device_status, sizeof(v));
+    v |= bits;
+    if (e == cudaSuccess) e = cudaMemcpyToSymbol(g_device_status, &v, sizeof(v));
+    if (e != cudaSuccess) return fail(NOBLE_ERR_CUDA, "status word: %s", cudaGetErrorString(e));
+    return NOBLE_OK;
+}
+
+const char *noble_status_string(noble_status s)
+{
+    switch (s) {
+    case NOBLE_OK: return "ok";
+    case NOBLE_ERR_INVALID_ARG: return "invalid argument";
+    case NOBLE_ERR_MISALIGNED: return "pointer not 16-byte aligned";
+    case NOBLE_ERR_UNSUPPORTED: return "unsupported shape, rank, dtype or flag";
+    case NOBLE_ERR_BUFFER_TOO_SMALL: return "buffer too small";
+    case NOBLE_ERR_CUDA: return "CUDA error";
+    case NOBLE_ERR_TIMEOUT: return "device-side wait timed out";
+    case NOBLE_ERR_NO_DEVICE: return "no usable sm_103 device";
+    }
+    return "unknown status";
+}
+
+const char *noble_last_error(void) { return g_last_error; }
+
+void noble_profile_enable(int on) { Profiler::get().enable(on != 0); }
+
+void noble_profile_reset(void) { Profiler::get().reset(); }
+
+static std::vector<Profiler::Entry> g_profile_snapshot;
+
+int noble_profile_count(void)
+{
+    g_profile_snapshot = Profiler::get().read();
+    return (int)g_profile_snapshot.size();
+}
+
+noble_status noble_profile_entry(int i, char *name, size_t name_len, uint64_t *launches, double *ms,
+                                 double *flops, double *bytes, int *bound)
+{
+    if (i < 0 || i >= (int)g_profile_snapshot.size() || !name || name_len == 0)
+        return fail(NOBLE_ERR_INVALID_ARG, "profile entry %d out of range", i);
+    const Profiler::Entry &e = g_profile_snapshot[i];
+    snprintf(name, name_len, "%s", e.name.c_str());
+    if (launches) *launches = e.launches;
+    if (ms) *ms = e.ms;
+    if (flops) *flops = e.flops;
+    if (bytes) *bytes = e.bytes;
+    if (bound) *bound = e.bound;
+    return NOBLE_OK;
+}
+
+uint64_t noble_kernel_launch_count(void) { return g_launches.load(); }
+
+}  // extern "C"

@@ -1,0 +1,240 @@
+// CUDA-core (SIMT) kernels: exact fp32 FMA, no tensor cores.
+//
+// These carry the fp32 validation mode end to end and every piece of the bf16
+// path that has no tensor-core kernel yet.  Every reduction over tokens is
+// split into fixed chunks whose partial results are summed in chunk order,
+// so results are deterministic.
+#pragma once
+
+#include "common.cuh"
+
+namespace noble {
+namespace simt {
+
+// Element (row, k) of an operand lives at p[row * ld_row + k * ld_k].
+struct Operand {
+    const void *p;
+    int64_t ld_row, ld_k;
+};
+struct Seg {
+    Operand A, B;
+    int64_t K;
+};
+
+constexpr int kBM = 64, kBN = 64, kBK = 16, kThreads = 256;
+
+// C[m][n] = sum_seg sum_k A(m,k) B(n,k) (+ bias[n]), fp32 accumulation.
+// With k_chunk > 0 (single segment only) block z sums k in
+// [z*k_chunk, (z+1)*k_chunk) and writes to C + z*c_chunk_stride.
+template <typename TIn, typename TOut>
+__global__ void __launch_bounds__(kThreads)
+gemm_kernel(int64_t M, int64_t N, Seg s0, Seg s1, int nseg, const float *bias, TOut *C,
+            int64_t ldc, int64_t k_chunk, int64_t c_chunk_stride)
+{
+    __shared__ float As[kBK][kBM + 1];
+    __shared__ float Bs[kBK][kBN + 1];
+    const int tid = threadIdx.x, tx = tid % 16, ty = tid / 16;
+    const int64_t m0 = (int64_t)blockIdx.y * kBM, n0 = (int64_t)blockIdx.x * kBN;
+    const int64_t z = blockIdx.z;
+    float acc[4][4];
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) acc[i][j] = 0.f;
+
+    for (int s = 0; s < nseg; ++s) {
+        const Seg &sg = s ? s1 : s0;
+        int64_t kb = 0, ke = sg.K;
+        if (k_chunk > 0) {
+            kb = z * k_chunk;
+            ke = min(sg.K, kb + k_chunk);
+        }
+        const TIn *A = (const TIn *)sg.A.p;
+        const TIn *B = (const TIn *)sg.B.p;
+        const bool a_kc = sg.A.ld_k == 1, b_kc = sg.B.ld_k == 1;
+        for (int64_t k0 = kb; k0 < ke; k0 += kBK) {
+#pragma unroll
+            for (int i = 0; i < (kBM * kBK) / kThreads; ++i) {
+                const int l = tid + i * kThreads;
+                int mm, kk;
+                if (a_kc) { mm = l / kBK; kk = l % kBK; } else { mm = l % kBM; kk = l / kBM; }
+                const int64_t gm = m0 + mm, gk = k0 + kk;
+                float v = 0.f;
+                if (gm < M && gk < ke) v = Elem<TIn>::load(A + gm * sg.A.ld_row + gk * sg.A.ld_k);
+                As[kk][mm] = v;
+                int nn;
+                if (b_kc) { nn = l / kBK; kk = l % kBK; } else { nn = l % kBN; kk = l / kBN; }
+                const int64_t gn = n0 + nn, gk2 = k0 + kk;
+                float w = 0.f;
+                if (gn < N && gk2 < ke) w = Elem<TIn>::load(B + gn * sg.B.ld_row + gk2 * sg.B.ld_k);
+                Bs[kk][nn] = w;
+            }
+            __syncthreads();
+#pragma unroll
+            for (int kk = 0; kk < kBK; ++kk) {
+                float a[4], b[4];
+#pragma unroll
+                for (int i = 0; i < 4; ++i) a[i] = As[kk][ty * 4 + i];
+#pragma unroll
+                for (int j = 0; j < 4; ++j) b[j] = Bs[kk][tx * 4 + j];
+#pragma unroll
+                for (int i = 0; i < 4; ++i)
+#pragma unroll
+                    for (int j = 0; j < 4; ++j) acc[i][j] = fmaf(a[i], b[j], acc[i][j]);
+            }
+            __syncthreads();
+        }
+    }
+    TOut *Cz = C + z * c_chunk_stride;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const int64_t gm = m0 + ty * 4 + i;
+        if (gm >= M) continue;
+#pragma unroll
+        for (int j = 0; j < 4; ++j) {
+            const int64_t gn = n0 + tx * 4 + j;
+            if (gn >= N) continue;
+            float v = acc[i][j];
+            if (bias) v += bias[gn];
+            Elem<TOut>::store(Cz + gm * ldc + gn, v);
+        }
+    }
+}
+
+// CosNet forward on rows (Eq. 2): from h [T][r] (fp32) computes
+//   a = cos(omega1 h + phi1), b = a M, c = cos(omega2 b + phi2)
+// and writes b (fp32) and c (TOut), each [T][r].  Block: tokens_per_block rows.
+template <typename TOut>
+__global__ void __launch_bounds__(256)
+cosnet_fwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const float *om1,
+                const float *ph1, const float *M, const float *om2, const float *ph2,
+                float *b_out, TOut *c_out)
+{
+    extern __shared__ float a_s[];  // [tokens_per_block][r]
+    const int64_t t0 = (int64_t)blockIdx.x * tokens_per_block;
+    const int n = tokens_per_block * r;
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, i = idx % r;
+        const int64_t t = t0 + tt;
+        a_s[idx] = t < T ? cosf(fmaf(om1[i], h[t * r + i], ph1[i])) : 0.f;
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, j = idx % r;
+        const int64_t t = t0 + tt;
+        if (t >= T) continue;
+        float s = 0.f;
+        for (int i = 0; i < r; ++i) s = fmaf(a_s[tt * r + i], M[i * r + j], s);
+        b_out[t * r + j] = s;
+        Elem<TOut>::store(c_out + t * r + j, cosf(fmaf(om2[j], s, ph2[j])));
+    }
+}
+
+// CosNet backward on rows (chain rule through Eq. 2).  From saved h, b (fp32),
+// dc = dy W_up (fp32) and Mt = M^T computes per token
+//   du2 = -sin(u2) dc, db = omega2 du2, da = db M^T, du1 = -sin(u1) da,
+//   dh = omega1 du1, a = cos(u1)
+// writing dh (TOut), a and db (fp32) [T][r], and per-block column sums
+//   part[blk][0:r] = sum du1*h, [r:2r] = sum du1, [2r:3r] = sum du2*b,
+//   [3r:4r] = sum du2      (tokens of the block in ascending order).
+template <typename TOut>
+__global__ void __launch_bounds__(256)
+cosnet_bwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const float *b,
+                const float *dc, const float *om1, const float *ph1, const float *Mt,
+                const float *om2, const float *ph2, TOut *dh_out, float *a_out, float *db_out,
+                float *part)
+{
+    extern __shared__ float sm[];
+    const int n = tokens_per_block * r;
+    float *db_s = sm, *du2_s = sm + n, *p2_s = sm + 2 * n, *du1_s = sm + 3 * n, *p1_s = sm + 4 * n;
+    const int64_t t0 = (int64_t)blockIdx.x * tokens_per_block;
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, j = idx % r;
+        const int64_t t = t0 + tt;
+        float du2 = 0.f, bv = 0.f;
+        if (t < T) {
+            bv = b[t * r + j];
+            du2 = -sinf(fmaf(om2[j], bv, ph2[j])) * dc[t * r + j];
+        }
+        const float dbv = om2[j] * du2;
+        db_s[idx] = dbv;
+        du2_s[idx] = du2;
+        p2_s[idx] = du2 * bv;
+        if (t < T) db_out[t * r + j] = dbv;
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, i = idx % r;
+        const int64_t t = t0 + tt;
+        float du1 = 0.f, hv = 0.f;
+        if (t < T) {
+            float da = 0.f;
+            for (int j = 0; j < r; ++j) da = fmaf(db_s[tt * r + j], Mt[j * r + i], da);
+            hv = h[t * r + i];
+            const float u1 = fmaf(om1[i], hv, ph1[i]);
+            float s1, c1;
+            sincosf(u1, &s1, &c1);
+            du1 = -s1 * da;
+            a_out[t * r + i] = c1;
+            Elem<TOut>::store(dh_out + t * r + i, om1[i] * du1);
+        }
+        du1_s[idx] = du1;
+        p1_s[idx] = du1 * hv;
+    }
+    __syncthreads();
+    float *pb = part + (int64_t)blockIdx.x * 4 * r;
+    for (int j = threadIdx.x; j < r; j += blockDim.x) {
+        float so1 = 0.f, sp1 = 0.f, so2 = 0.f, sp2 = 0.f;
+        for (int tt = 0; tt < tokens_per_block; ++tt) {
+            so1 += p1_s[tt * r + j];
+            sp1 += du1_s[tt * r + j];
+            so2 += p2_s[tt * r + j];
+            sp2 += du2_s[tt * r + j];
+        }
+        pb[j] = so1;
+        pb[r + j] = sp1;
+        pb[2 * r + j] = so2;
+        pb[3 * r + j] = sp2;
+    }
+}
+
+// part[c][o] = sum over rows t in chunk c (ascending) of X[t][o].
+template <typename TIn>
+__global__ void colsum_partial(int64_t T, int64_t n, int64_t rows_per_chunk, const TIn *X,
+                               float *part)
+{
+    const int64_t o = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (o >= n) return;
+    const int64_t tb = (int64_t)blockIdx.y * rows_per_chunk;
+    const int64_t te = min(T, tb + rows_per_chunk);
+    float s = 0.f;
+    for (int64_t t = tb; t < te; ++t) s += Elem<TIn>::load(X + t * n + o);
+    part[(int64_t)blockIdx.y * n + o] = s;
+}
+
+// out[k / seg_len][k % seg_len] = sum_p part[p * n + k], p ascending.
+struct Outs4 {
+    float *p[4];
+};
+__global__ void reduce_partials(int64_t nparts, int64_t n, int64_t seg_len, const float *part,
+                                Outs4 outs)
+{
+    const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (k >= n) return;
+    float s = 0.f;
+    for (int64_t p = 0; p < nparts; ++p) s += part[p * n + k];
+    float *dst = outs.p[k / seg_len];
+    if (dst) dst[k % seg_len] = s;
+}
+
+// Mt[j][i] = M[i][j]
+__global__ void transpose_square(int r, const float *M, float *Mt)
+{
+    const int idx = blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= r * r) return;
+    const int i = idx / r, j = idx % r;
+    Mt[j * r + i] = M[i * r + j];
+}
+
+}  // namespace simt
+}  // namespace noble

@@ -1,0 +1,116 @@
+"""C-ABI checks that need no GPU: the library builds, loads, exports every
+function include/noble.h declares, and rejects bad arguments on the host
+before it touches a device."""
+import ctypes
+
+import pytest
+
+from paper_2603_06492_gb300 import binding
+from paper_2603_06492_gb300.build import build
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build()
+    return binding.load()
+
+
+def test_exports_every_declared_function(lib):
+    names = binding.declared_functions()
+    assert "noble_linear_fwd" in names and "noble_linear_bwd" in names
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+def test_status_strings(lib):
+    for code in range(8):
+        assert lib.noble_status_string(code)
+
+
+def test_buffer_size_queries(lib):
+    d = binding.make_desc(256, 128, 128, 16, "fp32")
+    sb, wb = binding.noble_linear_saved_bytes(d), binding.noble_linear_bwd_workspace_bytes(d)
+    assert sb >= 256 * 16 * (4 + 4 + 4)
+    assert wb >= 256 * 16 * 4
+    assert binding.noble_linear_saved_bytes(binding.make_desc(256, 128, 128, 0, "bf16")) == 0
+    assert binding.noble_linear_bwd_workspace_bytes(binding.make_desc(0, 128, 128, 0, "bf16")) > 0
+    # invalid descriptors report 0
+    assert binding.noble_linear_saved_bytes(binding.make_desc(256, 128, 128, 24, "bf16")) == 0
+    assert binding.noble_linear_bwd_workspace_bytes(binding.make_desc(256, 100, 128, 16, "bf16")) == 0
+
+
+FAKE = 0x100000  # 16-byte aligned and never dereferenced: validation fails first
+
+
+def _fwd(desc, **over):
+    args = dict(x=FAKE, W=FAKE, bias=None, W_down=FAKE, omega1=FAKE, phi1=FAKE, M=FAKE,
+                omega2=FAKE, phi2=FAKE, W_up=FAKE, y=FAKE, saved=FAKE,
+                saved_bytes=1 << 40, stream=None)
+    args.update(over)
+    return binding.noble_linear_fwd(desc, **args)
+
+
+@pytest.mark.parametrize("shape,code", [
+    ((256, 128, 128, 24), 3),   # rank not supported
+    ((256, 100, 128, 16), 3),   # d_in not a multiple of 8
+    ((256, 128, 4, 16), 3),     # d_out below 8
+    ((-1, 128, 128, 16), 1),    # negative T
+])
+def test_bad_shapes_rejected(lib, shape, code):
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(binding.make_desc(*shape, "bf16"))
+    assert e.value.status == code
+
+
+def test_bad_pointers_rejected(lib):
+    d = binding.make_desc(256, 128, 128, 16, "bf16")
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(d, x=None)
+    assert e.value.status == 1 and "x" in str(e.value)
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(d, W_up=FAKE + 8)
+    assert e.value.status == 2
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(d, M=None)
+    assert e.value.status == 1
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(d, saved_bytes=16)
+    assert e.value.status == 4
+    bad = binding.make_desc(256, 128, 128, 16, "bf16")
+    bad.flags = 1
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(bad)
+    assert e.value.status == 3
+    with pytest.raises(binding.NobleError) as e:
+        binding._check(binding.load().noble_linear_fwd(None, *([None] * 12), 0, None))
+    assert e.value.status == 1
+
+
+def test_branch_pointers_optional_without_rank(lib):
+    d = binding.make_desc(256, 128, 128, 0, "bf16")
+    # valid arguments reach the device check; on a machine without a GPU that
+    # is the first failure, on a GPU machine it is not reached here.
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("device present")
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(d, W_down=None, omega1=None, phi1=None, M=None, omega2=None, phi2=None,
+             W_up=None, saved=None, saved_bytes=0)
+    assert e.value.status == 7
+
+
+def test_bwd_workspace_size_checked(lib):
+    d = binding.make_desc(64, 128, 128, 16, "bf16")
+    sb = binding.noble_linear_saved_bytes(d)
+    wb = binding.noble_linear_bwd_workspace_bytes(d)
+    kw = dict(dy=FAKE, x=FAKE, W=FAKE, W_down=FAKE, omega1=FAKE, phi1=FAKE, M=FAKE, omega2=FAKE,
+              phi2=FAKE, W_up=FAKE, saved=FAKE, saved_bytes=sb, dx=FAKE, dW=FAKE, dbias=None,
+              dW_down=FAKE, dM=FAKE, domega1=FAKE, dphi1=FAKE, domega2=FAKE, dphi2=FAKE,
+              dW_up=FAKE, workspace=FAKE, workspace_bytes=wb - 1, stream=None)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_linear_bwd(d, **kw)
+    assert e.value.status == 4
+    kw.update(workspace_bytes=wb, dM=None)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_linear_bwd(d, **kw)
+    assert e.value.status == 1 and "dM" in str(e.value)

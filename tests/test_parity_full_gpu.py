@@ -1,0 +1,69 @@
+"""Parity at the measured layer shapes (configs 1-4), in the same launch
+configuration bench.py times, on outputs the oracle can compute one by one:
+
+  * y and dx on sampled tokens (tokens are independent, so the oracle runs on
+    just those rows);
+  * sampled elements of dW and all of dbias (each is one sum over tokens);
+  * every branch gradient (dW_down, dW_up, dM, domega, dphi) in full, from one
+    full-batch oracle pass of the r-wide branch.
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2603_06492_gb300.inputs import CONFIGS, layer_seed, make_layer_inputs, to_paper_orientation
+from tests.gpu_helpers import TOL, rel_err, run_gpu
+
+pytestmark = pytest.mark.gpu
+
+CASES = [(1, 0), (1, 1), (2, 0), (2, 1), (3, 0), (3, 1), (3, 2),
+         (4, 0), (4, 7), (4, 14), (4, 11)]  # config 4: r16 qkv, r64 ffn_up, r256 ffn_down, r128 ffn_down
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2603_06492_gb300.build import build
+    build()
+
+
+@pytest.mark.parametrize("cfg,li", CASES, ids=lambda v: str(v))
+def test_full_size_sampled(cfg, li):
+    layer = CONFIGS[cfg][li]
+    inp = make_layer_inputs(layer, layer_seed(cfg, li))
+    got = run_gpu(layer, inp)
+    p = to_paper_orientation(inp)
+    rng = np.random.default_rng(100 + cfg * 31 + li)
+    tol = TOL[layer.dtype]
+
+    rows = np.sort(rng.choice(layer.T, 48, replace=False))
+    rows[-1] = layer.T - 1  # the ragged tail tile
+    sub = {k: (v[rows] if k in ("x", "dy") else v) for k, v in p.items()}
+    y_ref = oracle.fwd(sub["x"], sub["W"], sub["bias"], sub["W_down"], sub["omega1"], sub["phi1"],
+                       sub["M"], sub["omega2"], sub["phi2"], sub["W_up"])
+    g_sub = oracle.bwd(sub["x"], sub["W"], sub["W_down"], sub["omega1"], sub["phi1"], sub["M"],
+                       sub["omega2"], sub["phi2"], sub["W_up"], sub["dy"],
+                       skip=("dW", "dbias", "dW_down", "dM", "domega1", "dphi1", "domega2",
+                             "dphi2", "dW_up"))
+    errs = {"y": rel_err(got["y"][rows], y_ref), "dx": rel_err(got["dx"][rows], g_sub["dx"])}
+
+    n = 512
+    o_idx = rng.integers(0, layer.d_out, n)
+    i_idx = rng.integers(0, layer.d_in, n)
+    o_idx[0], i_idx[0] = layer.d_out - 1, layer.d_in - 1
+    dW_ref = oracle.outer_elems(p["dy"], p["x"], o_idx, i_idx)
+    errs["dW"] = rel_err(got["dW"][o_idx, i_idx], dW_ref)
+    ones = np.ones((layer.T, 1))
+    dbias_ref = oracle.outer_elems(p["dy"], ones, np.arange(layer.d_out), np.zeros(layer.d_out, np.int64))
+    errs["dbias"] = rel_err(got["dbias"], dbias_ref)
+
+    g = oracle.bwd(p["x"], p["W"], p["W_down"], p["omega1"], p["phi1"], p["M"], p["omega2"],
+                   p["phi2"], p["W_up"], p["dy"], skip=("dx", "dW", "dbias"))
+    errs["dW_down"] = rel_err(got["dW_down"], g["dW_down"].T)
+    errs["dW_up"] = rel_err(got["dW_up"], g["dW_up"].T)
+    for k in ("dM", "domega1", "dphi1", "domega2", "dphi2"):
+        errs[k] = rel_err(got[k], g[k])
+    bad = {k: e for k, e in errs.items() if not e <= tol}
+    assert not bad, f"config {cfg} {layer.name}: {bad} (all {errs})"

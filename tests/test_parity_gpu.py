@@ -1,0 +1,171 @@
+"""GPU parity: the CUDA path (through the C ABI) against the fp64 oracle on the
+same seeded inputs, element by element, at sizes the oracle finishes in
+seconds (several tiles and a ragged tail), plus the special cases of the
+method and the edge cases of the interface."""
+import math
+
+import numpy as np
+import pytest
+
+from paper_2603_06492_gb300 import binding
+from paper_2603_06492_gb300.inputs import CONFIGS, Layer, layer_seed, make_layer_inputs
+from tests.gpu_helpers import assert_close, rel_err, run_gpu, run_oracle
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("needs a GPU")
+    from paper_2603_06492_gb300.build import build
+    build()
+    binding.load()
+
+
+def test_config0_fp32_full():
+    layer = CONFIGS[0][0]
+    inp = make_layer_inputs(layer, layer_seed(0, 0))
+    assert_close(run_gpu(layer, inp), run_oracle(layer, inp), "fp32", ctx="config 0")
+
+
+SMALL = [
+    # (T, d_in, d_out, r): multiple tiles in every dimension plus ragged tails
+    (300, 200, 264, 16),
+    (129, 136, 72, 32),
+    (257, 192, 328, 64),
+    (200, 256, 136, 128),
+    (130, 264, 256, 256),
+    (1, 128, 128, 64),
+    (127, 72, 40, 16),
+    (333, 200, 264, 0),
+]
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+@pytest.mark.parametrize("shape", SMALL, ids=lambda s: "x".join(map(str, s)))
+@pytest.mark.parametrize("init", ["config", "strong_branch"])
+def test_small_shapes(dtype, shape, init):
+    layer = Layer("small", *shape, dtype)
+    inp = make_layer_inputs(layer, 1234 + sum(shape), init=init)
+    got, ref = run_gpu(layer, inp), run_oracle(layer, inp)
+    assert_close(got, ref, dtype, ctx=f"{shape} {dtype} {init}")
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_paper_init(dtype):
+    layer = Layer("paper_init", 257, 192, 264, 64, dtype)
+    inp = make_layer_inputs(layer, 77, init="paper")
+    assert_close(run_gpu(layer, inp), run_oracle(layer, inp), dtype, ctx="paper init")
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_branch_delta(dtype):
+    """The branch term alone, y - (x W^T + bias), so branch errors cannot hide
+    under the main path's magnitude."""
+    layer = Layer("delta", 256, 128, 192, 32, dtype)
+    inp = make_layer_inputs(layer, 5)
+    plain = {k: v for k, v in inp.items() if k in ("x", "W", "bias", "dy")}
+    lp = layer.plain()
+    got = run_gpu(layer, inp)["y"] - run_gpu(lp, plain)["y"]
+    ref = run_oracle(layer, inp)["y"] - run_oracle(lp, plain)["y"]
+    # y itself is rounded to the operand type; compare against that rounding
+    scale = np.max(np.abs(run_oracle(layer, inp)["y"]))
+    ulp = scale * (2.0**-8 if dtype == "bf16" else 2.0**-23)
+    err = np.max(np.abs(got - ref))
+    assert err <= 2 * ulp + 1e-2 * np.max(np.abs(ref)), (err, ulp, np.max(np.abs(ref)))
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_zero_up_equals_plain_path(dtype):
+    """W_up = 0: y and dx equal the r = 0 path bit for bit; branch gradients
+    other than dW_up vanish."""
+    layer = Layer("s1", 200, 136, 264, 32, dtype)
+    inp = make_layer_inputs(layer, 11)
+    inp["W_up"] = np.zeros_like(inp["W_up"])
+    got = run_gpu(layer, inp)
+    plain = run_gpu(layer.plain(), {k: inp[k] for k in ("x", "W", "bias", "dy")})
+    assert np.array_equal(got["y"], plain["y"])
+    assert np.array_equal(got["dx"], plain["dx"])
+    assert np.array_equal(got["dW"], plain["dW"])
+    for k in ("dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2"):
+        assert np.all(got[k] == 0), k
+    assert_close(got, run_oracle(layer, inp), dtype, ctx="W_up = 0")
+
+
+def test_linear_limit_fp32():
+    """phi = -pi/2, small omega: CosNet is nearly linear; checked against the
+    oracle in fp32 (fixes the orientation of M on the device too)."""
+    layer = Layer("lin", 192, 128, 136, 16, "fp32")
+    inp = make_layer_inputs(layer, 21, init="strong_branch")
+    rng = np.random.default_rng(0)
+    for k in ("phi1", "phi2"):
+        inp[k] = np.full(16, np.float32(-math.pi / 2), dtype=np.float64)
+    inp["omega1"] = np.float32(1e-2) * rng.uniform(0.5, 2, 16).astype(np.float32).astype(np.float64)
+    inp["omega2"] = rng.uniform(0.5, 2, 16).astype(np.float32).astype(np.float64)
+    assert_close(run_gpu(layer, inp), run_oracle(layer, inp), "fp32", ctx="linear limit")
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_phase_periodicity(dtype):
+    layer = Layer("per", 256, 128, 128, 16, dtype)
+    inp = make_layer_inputs(layer, 9)
+    base = run_gpu(layer, inp)
+    shifted = dict(inp, phi1=(inp["phi1"] + 2 * math.pi).astype(np.float32).astype(np.float64))
+    got = run_gpu(layer, shifted)
+    ref = run_oracle(layer, shifted)
+    assert_close(got, ref, dtype, ctx="phase + 2 pi")
+    for k in base:
+        assert rel_err(got[k], base[k]) < (1e-4 if dtype == "fp32" else 2e-2), k
+
+
+@pytest.mark.parametrize("dtype", ["fp32", "bf16"])
+def test_deterministic(dtype):
+    layer = Layer("det", 300, 200, 264, 64, dtype)
+    inp = make_layer_inputs(layer, 3)
+    a, b = run_gpu(layer, inp), run_gpu(layer, inp, repeat=2)
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k
+
+
+def test_token_permutation_bf16():
+    layer = Layer("perm", 256, 128, 136, 32, "bf16")
+    inp = make_layer_inputs(layer, 8)
+    perm = np.random.default_rng(1).permutation(256)
+    q = dict(inp, x=inp["x"][perm], dy=inp["dy"][perm])
+    a, b = run_gpu(layer, inp), run_gpu(layer, q)
+    assert np.array_equal(b["y"], a["y"][perm])
+    assert np.array_equal(b["dx"], a["dx"][perm])
+
+
+def test_empty_batch():
+    import torch
+    layer = Layer("empty", 0, 128, 64, 16, "bf16")
+    inp = make_layer_inputs(layer, 0)
+    dev = binding.params_to_device(inp, "bf16")
+    buf = binding.NobleLinearBuffers(0, 128, 64, 16, "bf16")
+    for g in buf.grads.values():
+        g.fill_(7.0)
+    binding.forward(buf, dev["x"], dev)
+    binding.backward(buf, dev["x"], dev["dy"], dev)
+    torch.cuda.synchronize()
+    for k, g in buf.grads.items():
+        assert torch.all(g == 0), k
+
+
+def test_device_status_reporting():
+    binding.noble_get_device_status(None)
+    binding.noble_debug_raise_device_status(1)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_get_device_status(None)
+    assert e.value.status == 6
+    binding.noble_get_device_status(None)  # cleared
+
+
+def test_launch_counter_advances():
+    layer = Layer("cnt", 128, 128, 128, 16, "bf16")
+    inp = make_layer_inputs(layer, 2)
+    n0 = binding.noble_kernel_launch_count()
+    run_gpu(layer, inp)
+    assert binding.noble_kernel_launch_count() > n0
