@@ -43,7 +43,9 @@
  *    outputs undefined.
  *  - Requirements: T >= 0; d_in, d_out >= 8 and multiples of 8;
  *    r in {0, 16, 32, 64, 128, 256} (r = 0 is the plain layer, and the branch
- *    pointers may then be NULL); every pointer 16-byte aligned.
+ *    pointers may then be NULL); every pointer 16-byte aligned.  With T == 0
+ *    the per-token pointers (x, y, dy, dx) may be NULL; the forward pass then
+ *    does nothing and the backward pass writes zero gradients.
  *  - Kernels never wait without a bound.  A wait that runs out records
  *    NOBLE_ERR_TIMEOUT in a device status word, which
  *    noble_get_device_status() reports.

@@ -309,11 +309,11 @@ noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, cons
 {
     g_last_error[0] = 0;
     NOBLE_TRY(validate_desc(desc));
-    const bool br = desc->r > 0;
-    NOBLE_TRY(check_ptr(x, "x", false));
+    const bool br = desc->r > 0, empty = desc->T == 0;
+    NOBLE_TRY(check_ptr(x, "x", empty));
     NOBLE_TRY(check_ptr(W, "W", false));
     NOBLE_TRY(check_ptr(bias, "bias", true));
-    NOBLE_TRY(check_ptr(y, "y", false));
+    NOBLE_TRY(check_ptr(y, "y", empty));
     NOBLE_TRY(check_ptr(W_down, "W_down", !br));
     NOBLE_TRY(check_ptr(omega1, "omega1", !br));
     NOBLE_TRY(check_ptr(phi1, "phi1", !br));
@@ -350,10 +350,10 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, con
 {
     g_last_error[0] = 0;
     NOBLE_TRY(validate_desc(desc));
-    const bool br = desc->r > 0;
-    const char *names[] = {"dy", "x", "W", "dx", "dW", "workspace"};
-    const void *req[] = {dy, x, W, dx, dW, workspace};
-    for (int i = 0; i < 6; ++i) NOBLE_TRY(check_ptr(req[i], names[i], false));
+    const bool br = desc->r > 0, empty = desc->T == 0;
+    const char *names[] = {"dy", "x", "dx", "W", "dW", "workspace"};
+    const void *req[] = {dy, x, dx, W, dW, workspace};
+    for (int i = 0; i < 6; ++i) NOBLE_TRY(check_ptr(req[i], names[i], empty && i < 3));
     NOBLE_TRY(check_ptr(dbias, "dbias", true));
     const char *bnames[] = {"W_down", "omega1", "phi1", "M", "omega2", "phi2", "W_up", "saved",
                             "dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2", "dW_up"};
