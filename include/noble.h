@@ -44,8 +44,9 @@
  *  - Requirements: T >= 0; d_in, d_out >= 8 and multiples of 8;
  *    r in {0, 16, 32, 64, 128, 256} (r = 0 is the plain layer, and the branch
  *    pointers may then be NULL); every pointer 16-byte aligned.  With T == 0
- *    the per-token pointers (x, y, dy, dx) may be NULL; the forward pass then
- *    does nothing and the backward pass writes zero gradients.
+ *    the per-token pointers (x, y, dy, dx) and `saved` may be NULL; the
+ *    forward pass then does nothing and the backward pass writes zero
+ *    gradients.
  *  - Kernels never wait without a bound.  A wait that runs out records
  *    NOBLE_ERR_TIMEOUT in a device status word, which
  *    noble_get_device_status() reports.
@@ -75,13 +76,18 @@ typedef enum {
 
 typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
 
+/* desc->flags bits */
+#define NOBLE_FLAG_SIMT_ONLY 1u /* bf16: run every step on CUDA cores (fp32
+                                   FMA), not tensor cores; a second path for
+                                   cross-checking the tensor-core kernels */
+
 typedef struct {
     int64_t T;      /* tokens (rows of x)                          */
     int64_t d_in;   /* input features                              */
     int64_t d_out;  /* output features                             */
     int64_t r;      /* bottleneck rank; 0 = plain linear layer     */
     int32_t dtype;  /* noble_dtype of the operands                 */
-    uint32_t flags; /* reserved, must be 0                         */
+    uint32_t flags; /* NOBLE_FLAG_* bits; 0 = default              */
 } noble_linear_desc;
 
 /*
@@ -167,6 +173,23 @@ uint64_t noble_kernel_launch_count(void);
  * without making any kernel wait.
  */
 noble_status noble_debug_raise_device_status(uint32_t bits);
+
+/*
+ * Testing hook (no paper counterpart): the library's tensor-core GEMM alone,
+ *     C[z][m][n] = sum_k A0(m,k) B0(n,k) + sum_k A1(m,k) B1(n,k) (+ bias[n])
+ * with bf16 operands and fp32 accumulation.  A_s is row-major [M][K_s]
+ * (a_mn = 0) or [K_s][M] (a_mn = 1); B_s is [N][K_s] (b_mn = 0) or [K_s][N]
+ * (b_mn = 1).  bn selects the N tile (16..256; only the combinations the
+ * layer uses exist).  C is fp32 (c_fp32 = 1) or bf16, row-major [M][N] per
+ * split; with nsplit > 1 split z sums k-blocks [z*kb_per_split,
+ * (z+1)*kb_per_split) of 64 and writes C + z*M*N.  M, N, K_s multiples of 8.
+ */
+noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1,
+                                  int a_mn, int b_mn, int bn, const void *A0,
+                                  const void *B0, const void *A1,
+                                  const void *B1, const float *bias, void *C,
+                                  int c_fp32, int kb_per_split, int nsplit,
+                                  noble_stream stream);
 
 /*
  * Instrumentation (no paper counterpart).  When enabled, every kernel the

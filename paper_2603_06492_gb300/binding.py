@@ -82,6 +82,9 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.noble_kernel_launch_count.restype = ctypes.c_uint64
         lib.noble_debug_raise_device_status.argtypes = [ctypes.c_uint32]
         lib.noble_debug_raise_device_status.restype = ctypes.c_int
+        i64, ci = ctypes.c_int64, ctypes.c_int
+        lib.noble_test_gemm_bf16.argtypes = [i64] * 4 + [ci] * 3 + [P] * 6 + [ci] * 3 + [P]
+        lib.noble_test_gemm_bf16.restype = ctypes.c_int
         lib.noble_profile_enable.argtypes = [ctypes.c_int]
         lib.noble_profile_enable.restype = None
         lib.noble_profile_reset.argtypes = []
@@ -133,6 +136,13 @@ def noble_linear_bwd(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up
                                    _p(saved), saved_bytes, _p(dx), _p(dW), _p(dbias), _p(dW_down),
                                    _p(dM), _p(domega1), _p(dphi1), _p(domega2), _p(dphi2),
                                    _p(dW_up), _p(workspace), workspace_bytes, stream))
+
+
+def noble_test_gemm_bf16(M, N, K0, K1, a_mn, b_mn, bn, A0, B0, A1, B1, bias, C, c_fp32,
+                         kb_per_split, nsplit, stream):
+    _check(load().noble_test_gemm_bf16(M, N, K0, K1, a_mn, b_mn, bn, _p(A0), _p(B0), _p(A1),
+                                       _p(B1), _p(bias), _p(C), c_fp32, kb_per_split, nsplit,
+                                       stream))
 
 
 def noble_get_device_status(stream=None):

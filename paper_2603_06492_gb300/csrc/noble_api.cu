@@ -4,6 +4,7 @@
 // Forward = Eq. 1 (Section 3.1) with CosNet (Eq. 2, Section 3.2; Eqs. 5-7,
 // Appendix A); backward = the chain rule through the same definitions.
 #include <atomic>
+#include <type_traits>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -12,7 +13,7 @@
 #include "common.cuh"
 #include "profile.cuh"
 #include "simt.cuh"
-#include "tc_path.cuh"
+#include "tc_gemm.cuh"
 
 namespace noble {
 
@@ -56,6 +57,8 @@ noble_status run(cudaStream_t st, const KernelInfo &ki, F &&f)
         if (_s != NOBLE_OK) return _s;               \
     } while (0)
 
+constexpr uint32_t kFlagSimtOnly = NOBLE_FLAG_SIMT_ONLY;
+
 bool rank_supported(int64_t r) { return r == 0 || r == 16 || r == 32 || r == 64 || r == 128 || r == 256; }
 
 noble_status validate_desc(const noble_linear_desc *d)
@@ -73,7 +76,7 @@ noble_status validate_desc(const noble_linear_desc *d)
         return fail(NOBLE_ERR_UNSUPPORTED, "r=%lld not in {0,16,32,64,128,256}", (long long)d->r);
     if (d->dtype != NOBLE_BF16 && d->dtype != NOBLE_FP32)
         return fail(NOBLE_ERR_UNSUPPORTED, "dtype %d not supported", (int)d->dtype);
-    if (d->flags != 0) return fail(NOBLE_ERR_UNSUPPORTED, "flags must be 0");
+    if (d->flags & ~kFlagSimtOnly) return fail(NOBLE_ERR_UNSUPPORTED, "unknown flags 0x%x", d->flags);
     return NOBLE_OK;
 }
 
@@ -130,7 +133,7 @@ int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
 // Backward scratch: dh (dtype), dc, a, db (fp32) [T][r]; Mt fp32 [r][r];
 // per-block partials of the CosNet sums, of dM and of dbias.
 struct WorkLayout {
-    size_t dh, dc, a, db, mt, cos_part, dm_part, bias_part, total;
+    size_t dh, dc, a, db, mt, wupt, cos_part, dm_part, bias_part, total;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
 };
 WorkLayout work_layout(const noble_linear_desc *d)
@@ -145,6 +148,7 @@ WorkLayout work_layout(const noble_linear_desc *d)
     L.a = take(tr * 4);
     L.db = take(tr * 4);
     L.mt = take((size_t)r * r * 4);
+    L.wupt = take((size_t)r * d->d_out * 2);
     L.n_cos_blocks = r ? ceil_div(T, cosnet_tokens_per_block(r)) : 0;
     L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
     L.n_dm_chunks = r ? ceil_div(T, kDmChunk) : 0;
@@ -269,6 +273,246 @@ noble_status bwd_simt(const noble_linear_desc *d, const TIn *dy, const TIn *x, c
     return NOBLE_OK;
 }
 
+
+// ------------------------------------------------------------ tensor-core path
+using bf16 = __nv_bfloat16;
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                  const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn()
+{
+    static EncodeTiledFn fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            p = nullptr;
+        }
+        return reinterpret_cast<EncodeTiledFn>(p);
+    }();
+    return fn;
+}
+
+// 2-D TMA map over a row-major bf16 matrix [rows][cols]: box of 64 columns
+// (128 bytes) by box_rows rows, 128-byte swizzle, zero fill out of bounds.
+noble_status make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t cols, uint32_t box_rows)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d): rows=%lld cols=%lld box_rows=%u", (int)r,
+                    (long long)rows, (long long)cols, box_rows);
+    return NOBLE_OK;
+}
+
+// Device address of this device's status word (looked up once per device).
+uint32_t *status_ptr()
+{
+    static uint32_t *cache[64];
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && cache[dev]) return cache[dev];
+    uint32_t *p = nullptr;
+    if (cudaGetSymbolAddress((void **)&p, g_device_status) != cudaSuccess) {
+        cudaGetLastError();
+        return nullptr;
+    }
+    if (dev >= 0 && dev < 64) cache[dev] = p;
+    return p;
+}
+
+// One K segment of a tensor-core GEMM; A and B are row-major bf16 matrices
+// ([M][K] / [N][K] when K-major, [K][M] / [K][N] when MN-major).
+struct TcSeg {
+    const void *A, *B;
+    int64_t K;
+};
+
+template <int BN> struct StagesFor { static constexpr int value = BN >= 256 ? 4 : BN >= 128 ? 6 : 8; };
+
+template <int BN, bool A_MN, bool B_MN, class Epi>
+noble_status tc_gemm(cudaStream_t st, const char *name, int64_t M, int64_t N, TcSeg s0, const TcSeg *s1,
+                     int kb_per_split, int nsplit, const typename Epi::Params &ep)
+{
+    constexpr int STAGES = StagesFor<BN>::value;
+    using SM = tc::Smem<BN, STAGES>;
+    if (M == 0 || N == 0) return NOBLE_OK;
+    CUtensorMap maps[4];
+    auto mk = [&](CUtensorMap *m, const void *p, bool mn, int64_t mnrows, int64_t K, uint32_t box_rows) {
+        return mn ? make_map(m, p, K, mnrows, 64) : make_map(m, p, mnrows, K, box_rows);
+    };
+    NOBLE_TRY(mk(&maps[0], s0.A, A_MN, M, s0.K, tc::kBM));
+    NOBLE_TRY(mk(&maps[1], s0.B, B_MN, N, s0.K, BN));
+    if (s1) {
+        NOBLE_TRY(mk(&maps[2], s1->A, A_MN, M, s1->K, tc::kBM));
+        NOBLE_TRY(mk(&maps[3], s1->B, B_MN, N, s1->K, BN));
+    } else {
+        maps[2] = maps[0];
+        maps[3] = maps[1];
+    }
+    const tc::GemmArgs args{M, N, (int)ceil_div(s0.K, tc::kBK), s1 ? (int)ceil_div(s1->K, tc::kBK) : 0,
+                            kb_per_split, status_ptr()};
+    auto kern = tc::gemm_kernel<BN, A_MN, B_MN, STAGES, Epi>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kDynamic) != cudaSuccess)
+        return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
+    const dim3 grid((unsigned)ceil_div(N, BN), (unsigned)ceil_div(M, tc::kBM), (unsigned)nsplit);
+    const double K = (double)s0.K + (s1 ? (double)s1->K : 0.0);
+    const KernelInfo ki{name, kBoundTensor, 2.0 * M * N * K, 2.0 * (M + N) * K};
+    return run(st, ki, [&] {
+        kern<<<grid, tc::kThreads, SM::kDynamic, st>>>(maps[0], maps[1], maps[2], maps[3], args, ep);
+    });
+}
+
+// Runtime r -> compile-time N tile for the r-wide products.
+template <class F>
+noble_status with_rank_tile(int64_t r, F &&f)
+{
+    switch (r) {
+    case 16: return f(std::integral_constant<int, 16>{});
+    case 32: return f(std::integral_constant<int, 32>{});
+    case 64: return f(std::integral_constant<int, 64>{});
+    case 128: return f(std::integral_constant<int, 128>{});
+    case 256: return f(std::integral_constant<int, 256>{});
+    }
+    return fail(NOBLE_ERR_UNSUPPORTED, "rank %lld", (long long)r);
+}
+
+__global__ void transpose_bf16(int64_t rows, int64_t cols, const bf16 *in, bf16 *out)
+{
+    __shared__ bf16 tile[32][33];
+    const int64_t c0 = (int64_t)blockIdx.x * 32, r0 = (int64_t)blockIdx.y * 32;
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int64_t rr = r0 + i, cc = c0 + threadIdx.x;
+        if (rr < rows && cc < cols) tile[i][threadIdx.x] = in[rr * cols + cc];
+    }
+    __syncthreads();
+    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
+        const int64_t cc = c0 + i, rr = r0 + threadIdx.x;
+        if (rr < rows && cc < cols) out[cc * rows + rr] = tile[threadIdx.x][i];
+    }
+}
+
+noble_status transpose(cudaStream_t st, int64_t rows, int64_t cols, const bf16 *in, bf16 *out)
+{
+    const KernelInfo ki{"transpose_bf16", kBoundHbm, 0.0, 4.0 * rows * cols};
+    return run(st, ki, [&] {
+        transpose_bf16<<<dim3((unsigned)ceil_div(cols, 32), (unsigned)ceil_div(rows, 32)), dim3(32, 8), 0, st>>>(
+            rows, cols, in, out);
+    });
+}
+
+noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, const float *bias,
+                    const bf16 *W_down, const float *om1, const float *ph1, const float *M, const float *om2,
+                    const float *ph2, const bf16 *W_up, bf16 *y, char *saved, cudaStream_t st)
+{
+    const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
+    const TcSeg main{x, W, di};
+    const tc::EpiStore<bf16>::Params py{y, dout, bias, 0};
+    if (r == 0)
+        return tc_gemm<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", T, dout, main, nullptr, 0, 1, py);
+    const SavedLayout SL = saved_layout(d);
+    float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
+    bf16 *c = (bf16 *)(saved + SL.c);
+    // h = x W_down^T on tensor cores (fp32 out)
+    NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
+        constexpr int BN = decltype(bn)::value;
+        const tc::EpiStore<float>::Params ph{h, r, nullptr, 0};
+        return tc_gemm<BN, false, false, tc::EpiStore<float>>(st, "tc_down_h", T, r, TcSeg{x, W_down, di}, nullptr,
+                                                               0, 1, ph);
+    }));
+    const int tpb = cosnet_tokens_per_block(r);
+    const KernelInfo ki{"simt_cosnet_fwd", kBoundAlu, 2.0 * T * r * r, 0.0};
+    NOBLE_TRY(run(st, ki, [&] {
+        simt::cosnet_fwd_rows<bf16><<<(unsigned)ceil_div(T, tpb), 256, tpb * r * sizeof(float), st>>>(
+            T, (int)r, tpb, h, om1, ph1, M, om2, ph2, b, c);
+    }));
+    const TcSeg up{c, W_up, r};
+    return tc_gemm<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", T, dout, main, &up, 0, 1, py);
+}
+
+noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, const bf16 *W, const bf16 *W_down,
+                    const float *om1, const float *ph1, const float *M, const float *om2, const float *ph2,
+                    const bf16 *W_up, const char *saved, bf16 *dx, float *dW, float *dbias, float *dW_down,
+                    float *dM, float *dom1, float *dph1, float *dom2, float *dph2, float *dW_up, char *ws,
+                    cudaStream_t st)
+{
+    const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
+    const SavedLayout SL = saved_layout(d);
+    const WorkLayout WL = work_layout(d);
+    bf16 *dh = (bf16 *)(ws + WL.dh);
+    if (r > 0) {
+        const float *h = (const float *)(saved + SL.h), *b = (const float *)(saved + SL.b);
+        const bf16 *c = (const bf16 *)(saved + SL.c);
+        float *dc = (float *)(ws + WL.dc), *a = (float *)(ws + WL.a), *db = (float *)(ws + WL.db);
+        float *Mt = (float *)(ws + WL.mt), *cpart = (float *)(ws + WL.cos_part);
+        float *dmpart = (float *)(ws + WL.dm_part);
+        bf16 *wupt = (bf16 *)(ws + WL.wupt);
+        // dc = dy W_up, with W_up transposed to K-major [r][d_out] first
+        NOBLE_TRY(transpose(st, dout, r, W_up, wupt));
+        NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
+            constexpr int BN = decltype(bn)::value;
+            const tc::EpiStore<float>::Params pc{dc, r, nullptr, 0};
+            return tc_gemm<BN, false, false, tc::EpiStore<float>>(st, "tc_dc", T, r, TcSeg{dy, wupt, dout},
+                                                                   nullptr, 0, 1, pc);
+        }));
+        const KernelInfo kt{"transpose_M", kBoundHbm, 0.0, 8.0 * r * r};
+        NOBLE_TRY(run(st, kt, [&] {
+            simt::transpose_square<<<(unsigned)ceil_div(r * r, 256), 256, 0, st>>>((int)r, M, Mt);
+        }));
+        const int tpb = cosnet_tokens_per_block(r);
+        const KernelInfo kc{"simt_cosnet_bwd", kBoundAlu, 2.0 * T * r * r, 0.0};
+        NOBLE_TRY(run(st, kc, [&] {
+            simt::cosnet_bwd_rows<bf16><<<(unsigned)WL.n_cos_blocks, 256, 5 * tpb * r * sizeof(float), st>>>(
+                T, (int)r, tpb, h, b, dc, om1, ph1, Mt, om2, ph2, dh, a, db, cpart);
+        }));
+        NOBLE_TRY(reduce(st, WL.n_cos_blocks, 4 * r, r, cpart, dom1, dph1, dom2, dph2));
+        simt::Seg sdm{{a, 1, r}, {db, 1, r}, T};
+        NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
+                                           WL.n_dm_chunks, r * r)));
+        NOBLE_TRY(reduce(st, WL.n_dm_chunks, r * r, r * r, dmpart, dM));
+        // dW_up = dy^T c  [d_out][r];  dW_down = dh^T x  [r][d_in]
+        NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
+            constexpr int BN = decltype(bn)::value < 64 ? 64 : decltype(bn)::value;
+            const tc::EpiStore<float>::Params pu{dW_up, r, nullptr, 0};
+            return tc_gemm<BN, true, true, tc::EpiStore<float>>(st, "tc_dW_up", dout, r, TcSeg{dy, c, T}, nullptr,
+                                                                 0, 1, pu);
+        }));
+        const tc::EpiStore<float>::Params pd{dW_down, di, nullptr, 0};
+        NOBLE_TRY((tc_gemm<256, true, true, tc::EpiStore<float>>(st, "tc_dW_down", r, di, TcSeg{dh, x, T}, nullptr,
+                                                                  0, 1, pd)));
+    }
+    // dx = [dy | dh] [W ; W_down]
+    const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
+    const TcSeg sdx2{dh, W_down, r};
+    NOBLE_TRY((tc_gemm<256, false, true, tc::EpiStore<bf16>>(st, "tc_dx", T, di, TcSeg{dy, W, dout},
+                                                              r > 0 ? &sdx2 : nullptr, 0, 1, px)));
+    // dW = dy^T x
+    const tc::EpiStore<float>::Params pw{dW, di, nullptr, 0};
+    NOBLE_TRY((tc_gemm<256, true, true, tc::EpiStore<float>>(st, "tc_dW", dout, di, TcSeg{dy, x, T}, nullptr, 0, 1,
+                                                              pw)));
+    if (dbias) {
+        float *bpart = (float *)(ws + WL.bias_part);
+        dim3 grid((unsigned)ceil_div(dout, 256), (unsigned)WL.n_bias_chunks);
+        const KernelInfo kb{"colsum_dbias", kBoundHbm, (double)T * dout, (double)T * dout * 2};
+        NOBLE_TRY(run(st, kb, [&] {
+            simt::colsum_partial<bf16><<<grid, 256, 0, st>>>(T, dout, kBiasChunk, dy, bpart);
+        }));
+        NOBLE_TRY(reduce(st, WL.n_bias_chunks, dout, dout, bpart, dbias));
+    }
+    return NOBLE_OK;
+}
+
 noble_status zero_grads(const noble_linear_desc *d, float *dW, float *dbias, float *dW_down, float *dM,
                         float *dom1, float *dph1, float *dom2, float *dph2, float *dW_up,
                         cudaStream_t st)
@@ -321,7 +565,7 @@ noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, cons
     NOBLE_TRY(check_ptr(omega2, "omega2", !br));
     NOBLE_TRY(check_ptr(phi2, "phi2", !br));
     NOBLE_TRY(check_ptr(W_up, "W_up", !br));
-    NOBLE_TRY(check_ptr(saved, "saved", !br));
+    NOBLE_TRY(check_ptr(saved, "saved", !br || empty));
     if (saved_bytes < saved_layout(desc).total)
         return fail(NOBLE_ERR_BUFFER_TOO_SMALL, "saved_bytes=%zu < %zu", saved_bytes, saved_layout(desc).total);
     NOBLE_TRY(check_device());
@@ -329,9 +573,9 @@ noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, cons
     cudaStream_t st = (cudaStream_t)stream;
     if (desc->dtype == NOBLE_BF16) {
         using bf = __nv_bfloat16;
-        if (tc::fwd_supported(desc))
-            return tc::fwd(desc, (const bf *)x, (const bf *)W, bias, (const bf *)W_down, omega1, phi1, M,
-                           omega2, phi2, (const bf *)W_up, (bf *)y, (char *)saved, st, g_launches);
+        if (!(desc->flags & kFlagSimtOnly))
+            return fwd_tc(desc, (const bf *)x, (const bf *)W, bias, (const bf *)W_down, omega1, phi1, M, omega2,
+                          phi2, (const bf *)W_up, (bf *)y, (char *)saved, st);
         return fwd_simt<bf>(desc, (const bf *)x, (const bf *)W, bias, (const bf *)W_down, omega1, phi1, M,
                             omega2, phi2, (const bf *)W_up, (bf *)y, (char *)saved, st);
     }
@@ -359,7 +603,7 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, con
                             "dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2", "dW_up"};
     const void *bptr[] = {W_down, omega1, phi1, M, omega2, phi2, W_up, saved,
                           dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up};
-    for (int i = 0; i < 15; ++i) NOBLE_TRY(check_ptr(bptr[i], bnames[i], !br));
+    for (int i = 0; i < 15; ++i) NOBLE_TRY(check_ptr(bptr[i], bnames[i], !br || (empty && i == 7)));
     if (saved_bytes < saved_layout(desc).total)
         return fail(NOBLE_ERR_BUFFER_TOO_SMALL, "saved_bytes=%zu < %zu", saved_bytes, saved_layout(desc).total);
     if (workspace_bytes < work_layout(desc).total)
@@ -371,11 +615,10 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, con
         return zero_grads(desc, dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, st);
     if (desc->dtype == NOBLE_BF16) {
         using bf = __nv_bfloat16;
-        if (tc::bwd_supported(desc))
-            return tc::bwd(desc, (const bf *)dy, (const bf *)x, (const bf *)W, (const bf *)W_down, omega1, phi1,
-                           M, omega2, phi2, (const bf *)W_up, (const char *)saved, (bf *)dx, dW, dbias,
-                           dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace, st,
-                           g_launches);
+        if (!(desc->flags & kFlagSimtOnly))
+            return bwd_tc(desc, (const bf *)dy, (const bf *)x, (const bf *)W, (const bf *)W_down, omega1, phi1, M,
+                          omega2, phi2, (const bf *)W_up, (const char *)saved, (bf *)dx, dW, dbias, dW_down, dM,
+                          domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace, st);
         return bwd_simt<bf>(desc, (const bf *)dy, (const bf *)x, (const bf *)W, (const bf *)W_down, omega1,
                             phi1, M, omega2, phi2, (const bf *)W_up, (const char *)saved, (bf *)dx, dW,
                             dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace,
@@ -427,6 +670,46 @@ const char *noble_status_string(noble_status s)
 }
 
 const char *noble_last_error(void) { return g_last_error; }
+
+noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, int a_mn, int b_mn, int bn,
+                                  const void *A0, const void *B0, const void *A1, const void *B1,
+                                  const float *bias, void *C, int c_fp32, int kb_per_split, int nsplit,
+                                  noble_stream stream)
+{
+    g_last_error[0] = 0;
+    if (M <= 0 || N <= 0 || K0 <= 0 || K1 < 0 || N % 8 || K0 % 8 || K1 % 8 || M % 8 || nsplit < 1)
+        return fail(NOBLE_ERR_INVALID_ARG, "bad GEMM sizes");
+    const void *ptrs[] = {A0, B0, C};
+    for (const void *p : ptrs) NOBLE_TRY(check_ptr(p, "operand", false));
+    if (K1 > 0) {
+        NOBLE_TRY(check_ptr(A1, "A1", false));
+        NOBLE_TRY(check_ptr(B1, "B1", false));
+    }
+    NOBLE_TRY(check_device());
+    cudaStream_t st = (cudaStream_t)stream;
+    const TcSeg s0{A0, B0, K0}, s1v{A1, B1, K1};
+    const TcSeg *s1 = K1 > 0 ? &s1v : nullptr;
+    const int64_t split_stride = nsplit > 1 ? M * N : 0;
+    const tc::EpiStore<float>::Params pf{(float *)C, N, bias, split_stride};
+    const tc::EpiStore<bf16>::Params pb{(bf16 *)C, N, bias, split_stride};
+#define NOBLE_TEST_CASE(BN_, AMN, BMN)                                                                      \
+    if (bn == BN_ && a_mn == AMN && b_mn == BMN)                                                            \
+        return c_fp32 ? tc_gemm<BN_, AMN, BMN, tc::EpiStore<float>>(st, "test", M, N, s0, s1, kb_per_split,  \
+                                                                     nsplit, pf)                            \
+                      : tc_gemm<BN_, AMN, BMN, tc::EpiStore<bf16>>(st, "test", M, N, s0, s1, kb_per_split,   \
+                                                                    nsplit, pb);
+    NOBLE_TEST_CASE(256, false, false)
+    NOBLE_TEST_CASE(128, false, false)
+    NOBLE_TEST_CASE(64, false, false)
+    NOBLE_TEST_CASE(32, false, false)
+    NOBLE_TEST_CASE(16, false, false)
+    NOBLE_TEST_CASE(256, false, true)
+    NOBLE_TEST_CASE(256, true, true)
+    NOBLE_TEST_CASE(128, true, true)
+    NOBLE_TEST_CASE(64, true, true)
+#undef NOBLE_TEST_CASE
+    return fail(NOBLE_ERR_UNSUPPORTED, "no GEMM instance for bn=%d a_mn=%d b_mn=%d", bn, a_mn, b_mn);
+}
 
 void noble_profile_enable(int on) { Profiler::get().enable(on != 0); }
 
