@@ -77,7 +77,7 @@ def test_bad_pointers_rejected(lib):
         _fwd(d, saved_bytes=16)
     assert e.value.status == 4
     bad = binding.make_desc(256, 128, 128, 16, "bf16")
-    bad.flags = 1
+    bad.flags = 2  # unknown flag bit
     with pytest.raises(binding.NobleError) as e:
         _fwd(bad)
     assert e.value.status == 3
