@@ -677,7 +677,9 @@ noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, 
                                   noble_stream stream)
 {
     g_last_error[0] = 0;
-    if (M <= 0 || N <= 0 || K0 <= 0 || K1 < 0 || N % 8 || K0 % 8 || K1 % 8 || M % 8 || nsplit < 1)
+    // the innermost dimension of every operand must be a multiple of 8 elements (16 bytes)
+    if (M <= 0 || N <= 0 || K0 <= 0 || K1 < 0 || nsplit < 1 || N % 8 || (a_mn && M % 8) ||
+        (!(a_mn && b_mn) && (K0 % 8 || K1 % 8)))
         return fail(NOBLE_ERR_INVALID_ARG, "bad GEMM sizes");
     const void *ptrs[] = {A0, B0, C};
     for (const void *p : ptrs) NOBLE_TRY(check_ptr(p, "operand", false));
