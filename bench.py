@@ -139,14 +139,14 @@ def run_reference(args, rank):
     import oracle
     oracle.build()
     for _ in range(args.warmup):
-        oracle_sample(layers, args.cpu_tokens)
+        oracle_sample(layers, args.ref_tokens)
     secs, flops = 0.0, 0.0
     for s in range(args.steps):
-        t, f = oracle_sample(layers, args.cpu_tokens, seed=100 + s)
+        t, f = oracle_sample(layers, args.ref_tokens, seed=100 + s)
         secs += t
         flops += f
     v = flops / secs / 1e12
-    sample = (f"first {args.cpu_tokens} of 16384 tokens of each of the 3 layers per step "
+    sample = (f"first {args.ref_tokens} of 16384 tokens of each of the 3 layers per step "
               f"(fwd+bwd, fp64)")
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
@@ -167,10 +167,15 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="own", choices=["own", "reference"])
-    ap.add_argument("--cpu-tokens", type=int, default=48,
-                    help="tokens per layer in the oracle's bounded sample")
+    ap.add_argument("--cpu-tokens", type=int, default=512,
+                    help="tokens per layer in the oracle's bounded sample (cpu_baseline)")
+    ap.add_argument("--ref-tokens", type=int, default=64,
+                    help="tokens per layer in each step of --impl reference")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--profile-run", action="store_true",
+                    help="fwd+bwd of the selected layers only, for ncu; prints no bench line")
+    ap.add_argument("--layers", default="", help="comma-separated layer names (default: all)")
     args = ap.parse_args()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -193,11 +198,15 @@ def main():
     if dist is not None:
         dist.barrier()
     binding.load()
-    assert args.warmup >= 3, "at least 3 warm-up steps"
+    assert args.profile_run or args.warmup >= 3, "at least 3 warm-up steps"
 
     layers = CONFIGS[CONFIG_INDEX]
+    if args.layers:
+        keep = set(args.layers.split(","))
+        layers = [l for l in layers if l.name in keep]
     dev_inputs, bufs, plain_bufs = [], [], []
-    for li, layer in enumerate(layers):
+    for layer in layers:
+        li = [l.name for l in CONFIGS[CONFIG_INDEX]].index(layer.name)
         inp = make_layer_inputs(layer, layer_seed(CONFIG_INDEX, li))
         dev_inputs.append(binding.params_to_device(inp, layer.dtype))
         del inp
@@ -229,6 +238,14 @@ def main():
             dist.all_reduce(t, op=dist.ReduceOp.MAX)
             ms = float(t.item())
         return ms
+
+    if args.profile_run:
+        for _ in range(args.warmup + args.steps):
+            step(bufs)
+        torch.cuda.synchronize()
+        binding.noble_get_device_status(None)
+        print("profile run done", flush=True)
+        return
 
     # warm-up (NOBLE and plain)
     for _ in range(args.warmup):
