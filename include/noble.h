@@ -151,6 +151,43 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy,
                               noble_stream stream);
 
 /*
+ * Backward pass without a caller workspace, for callers that cannot allocate
+ * device memory: code that runs inside a host framework or plugin which owns
+ * every device allocation and hands its extensions no allocator, or a
+ * real-time loop that forbids allocation once it has started.  The paper has
+ * no counterpart; this is an interface convenience.
+ *
+ * Same arguments, results and errors as noble_linear_bwd, minus `workspace`
+ * and `workspace_bytes`: the scratch is a static device array inside the
+ * library, NOBLE_NOALLOC_SCRATCH_BYTES (64 MiB) long, which every GPU that
+ * loads the library holds until the process exits.  No cudaMalloc, cudaFree
+ * or other allocating call is made.
+ *  - A shape whose noble_linear_bwd_workspace_bytes() exceeds that size is
+ *    rejected with NOBLE_ERR_BUFFER_TOO_SMALL before anything is enqueued.
+ *  - The first call on a device looks up the array's device address (once
+ *    per device, with that device current); make that first call before any
+ *    stream capture.
+ *  - Every call on a device shares the one array, and it keeps the last
+ *    call's contents.  Nothing in it needs to start at zero: each call writes
+ *    every scratch value before reading it.  Calls whose work overlaps on the
+ *    GPU (other streams, other host threads) race on the array and give wrong
+ *    results; the caller must order them, e.g. on a single stream.
+ */
+#define NOBLE_NOALLOC_SCRATCH_BYTES (64u << 20)
+noble_status noble_linear_bwd_noalloc(const noble_linear_desc *desc,
+                                      const void *dy, const void *x,
+                                      const void *W, const void *W_down,
+                                      const float *omega1, const float *phi1,
+                                      const float *M, const float *omega2,
+                                      const float *phi2, const void *W_up,
+                                      const void *saved, size_t saved_bytes,
+                                      void *dx, float *dW, float *dbias,
+                                      float *dW_down, float *dM,
+                                      float *domega1, float *dphi1,
+                                      float *domega2, float *dphi2,
+                                      float *dW_up, noble_stream stream);
+
+/*
  * Synchronises `stream`, then reads and clears the device status word of the
  * current device.  NOBLE_ERR_TIMEOUT if any kernel gave up a bounded wait
  * since the last call, NOBLE_ERR_CUDA if the stream reported an error,

@@ -72,6 +72,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.noble_linear_fwd.restype = ctypes.c_int
         lib.noble_linear_bwd.argtypes = [D] + [P] * 11 + [S] + [P] * 11 + [S, P]
         lib.noble_linear_bwd.restype = ctypes.c_int
+        lib.noble_linear_bwd_noalloc.argtypes = [D] + [P] * 11 + [S] + [P] * 10 + [P]
+        lib.noble_linear_bwd_noalloc.restype = ctypes.c_int
         lib.noble_get_device_status.argtypes = [P]
         lib.noble_get_device_status.restype = ctypes.c_int
         lib.noble_status_string.argtypes = [ctypes.c_int]
@@ -143,6 +145,20 @@ def noble_test_gemm_bf16(M, N, K0, K1, a_mn, b_mn, bn, A0, B0, A1, B1, bias, C, 
     _check(load().noble_test_gemm_bf16(M, N, K0, K1, a_mn, b_mn, bn, _p(A0), _p(B0), _p(A1),
                                        _p(B1), _p(bias), _p(C), c_fp32, kb_per_split, nsplit,
                                        stream))
+
+
+def noble_linear_bwd_noalloc(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up, saved,
+                             saved_bytes, dx, dW, dbias, dW_down, dM, domega1, dphi1, domega2,
+                             dphi2, dW_up, stream):
+    """Backward pass using the library's static scratch (no workspace argument)."""
+    _check(load().noble_linear_bwd_noalloc(ctypes.byref(desc), _p(dy), _p(x), _p(W), _p(W_down),
+                                           _p(omega1), _p(phi1), _p(M), _p(omega2), _p(phi2),
+                                           _p(W_up), _p(saved), saved_bytes, _p(dx), _p(dW),
+                                           _p(dbias), _p(dW_down), _p(dM), _p(domega1),
+                                           _p(dphi1), _p(domega2), _p(dphi2), _p(dW_up), stream))
+
+
+NOALLOC_SCRATCH_BYTES = 64 << 20
 
 
 def noble_get_device_status(stream=None):

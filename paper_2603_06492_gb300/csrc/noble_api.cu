@@ -4,6 +4,7 @@
 // Forward = Eq. 1 (Section 3.1) with CosNet (Eq. 2, Section 3.2; Eqs. 5-7,
 // Appendix A); backward = the chain rule through the same definitions.
 #include <atomic>
+#include <mutex>
 #include <type_traits>
 #include <cstdarg>
 #include <cstdio>
@@ -18,6 +19,11 @@
 namespace noble {
 
 __device__ uint32_t g_device_status = 0;
+
+// Library-owned scratch for noble_linear_bwd_noalloc (see include/noble.h).
+// Every GPU that loads this library holds it until the process exits.
+constexpr size_t kNoallocScratchBytes = (size_t)NOBLE_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_noalloc_scratch[kNoallocScratchBytes];
 
 namespace {
 
@@ -670,6 +676,56 @@ const char *noble_status_string(noble_status s)
 }
 
 const char *noble_last_error(void) { return g_last_error; }
+
+// Device address of g_noalloc_scratch for the current device.  The host-side
+// name of a __device__ array is only a stand-in, so the address is looked up
+// once per device (with that device current) and cached.
+static noble_status noalloc_scratch_ptr(void **out)
+{
+    static std::mutex mu;
+    static void *cache[64];
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+        cudaGetLastError();
+        return fail(NOBLE_ERR_NO_DEVICE, "no current CUDA device for the static scratch");
+    }
+    std::lock_guard<std::mutex> g(mu);
+    if (!cache[dev]) {
+        void *p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+        if (e != cudaSuccess || !p) {
+            cudaGetLastError();
+            return fail(NOBLE_ERR_CUDA, "cudaGetSymbolAddress(static scratch): %s", cudaGetErrorString(e));
+        }
+        cache[dev] = p;
+    }
+    *out = cache[dev];
+    return NOBLE_OK;
+}
+
+noble_status noble_linear_bwd_noalloc(const noble_linear_desc *desc, const void *dy, const void *x,
+                                      const void *W, const void *W_down, const float *omega1,
+                                      const float *phi1, const float *M, const float *omega2,
+                                      const float *phi2, const void *W_up, const void *saved,
+                                      size_t saved_bytes, void *dx, float *dW, float *dbias,
+                                      float *dW_down, float *dM, float *domega1, float *dphi1,
+                                      float *domega2, float *dphi2, float *dW_up, noble_stream stream)
+{
+    g_last_error[0] = 0;
+    NOBLE_TRY(validate_desc(desc));
+    const size_t need = work_layout(desc).total;
+    if (need > kNoallocScratchBytes)
+        return fail(NOBLE_ERR_BUFFER_TOO_SMALL,
+                    "this shape needs %zu bytes of backward scratch; the static scratch of "
+                    "noble_linear_bwd_noalloc holds %zu (use noble_linear_bwd with a workspace)",
+                    need, kNoallocScratchBytes);
+    NOBLE_TRY(check_device());
+    void *scratch = nullptr;
+    NOBLE_TRY(noalloc_scratch_ptr(&scratch));
+    return noble_linear_bwd(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up, saved, saved_bytes, dx,
+                            dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, scratch,
+                            kNoallocScratchBytes, stream);
+}
 
 noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, int a_mn, int b_mn, int bn,
                                   const void *A0, const void *B0, const void *A1, const void *B1,
