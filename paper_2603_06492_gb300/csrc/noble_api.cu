@@ -15,6 +15,7 @@
 #include "profile.cuh"
 #include "simt.cuh"
 #include "tc_gemm.cuh"
+#include "tc_persistent.cuh"
 
 namespace noble {
 
@@ -133,7 +134,7 @@ SavedLayout saved_layout(const noble_linear_desc *d)
 }
 
 constexpr int64_t kDmChunk = 1024;     // tokens per dM partial
-constexpr int64_t kBiasChunk = 512;    // tokens per dbias partial
+constexpr int64_t kBiasChunk = 128;    // tokens per dbias partial
 int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
 
 // Backward scratch: dh (dtype), dc, a, db (fp32) [T][r]; Mt fp32 [r][r];
@@ -188,7 +189,7 @@ noble_status reduce(cudaStream_t st, int64_t nparts, int64_t n, int64_t seg_len,
     simt::Outs4 outs{{o0, o1, o2, o3}};
     const KernelInfo ki{"reduce_partials", kBoundHbm, (double)nparts * n, 4.0 * (nparts + 1) * n};
     return run(st, ki, [&] {
-        simt::reduce_partials<<<(unsigned)ceil_div(n, 256), 256, 0, st>>>(nparts, n, seg_len, part, outs);
+        simt::reduce_partials<<<(unsigned)ceil_div(n, 32), 256, 0, st>>>(nparts, n, seg_len, part, outs);
     });
 }
 
@@ -380,6 +381,92 @@ noble_status tc_gemm(cudaStream_t st, const char *name, int64_t M, int64_t N, Tc
     });
 }
 
+
+int num_sms()
+{
+    static int cache[64];
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (dev >= 0 && dev < 64 && cache[dev]) return cache[dev];
+    int n = 0;
+    cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+    cudaGetLastError();
+    if (n <= 0) n = 1;
+    if (dev >= 0 && dev < 64) cache[dev] = n;
+    return n;
+}
+
+// One problem of a grouped persistent GEMM launch.
+struct ProbSpec {
+    int64_t M, N;
+    TcSeg s0;
+    const TcSeg *s1;  // nullptr = single segment
+    int bn;           // N tile (multiple of 32; of 64 when B is MN-major)
+    int nsplit = 1;
+    int kb_per_split = 0;
+};
+
+template <int BN_MAX> struct PStagesFor { static constexpr int value = BN_MAX >= 256 ? 4 : 6; };
+
+template <int BN_MAX, bool A_MN, bool B_MN, class Epi>
+noble_status tc_group(cudaStream_t st, const char *name, int n, const ProbSpec *specs,
+                      const typename Epi::Params *eps)
+{
+    constexpr int STAGES = PStagesFor<BN_MAX>::value;
+    using SM = tc::PSmem<BN_MAX, STAGES>;
+    if (n < 1 || n > tc::kMaxProblems) return fail(NOBLE_ERR_INVALID_ARG, "%s: %d problems", name, n);
+    tc::GroupMaps maps;
+    tc::GroupArgs<typename Epi::Params> g{};
+    int tiles = 0;
+    double flops = 0, bytes = 0;
+    int np = 0;
+    for (int i = 0; i < n; ++i) {
+        const ProbSpec &P = specs[i];
+        if (P.M == 0 || P.N == 0) continue;
+        if (P.bn % 32 || P.bn > BN_MAX || (B_MN && P.bn % 64))
+            return fail(NOBLE_ERR_INVALID_ARG, "%s: tile width %d", name, P.bn);
+        auto mk = [&](CUtensorMap *m, const void *p, bool mn, int64_t mnrows, int64_t K, uint32_t box_rows) {
+            return mn ? make_map(m, p, K, mnrows, 64) : make_map(m, p, mnrows, K, box_rows);
+        };
+        NOBLE_TRY(mk(&maps.m[np][0], P.s0.A, A_MN, P.M, P.s0.K, tc::kBM));
+        NOBLE_TRY(mk(&maps.m[np][1], P.s0.B, B_MN, P.N, P.s0.K, (uint32_t)P.bn));
+        if (P.s1) {
+            NOBLE_TRY(mk(&maps.m[np][2], P.s1->A, A_MN, P.M, P.s1->K, tc::kBM));
+            NOBLE_TRY(mk(&maps.m[np][3], P.s1->B, B_MN, P.N, P.s1->K, (uint32_t)P.bn));
+        } else {
+            maps.m[np][2] = maps.m[np][0];
+            maps.m[np][3] = maps.m[np][1];
+        }
+        auto &q = g.p[np];
+        q.M = P.M;
+        q.N = P.N;
+        q.kb0 = (int)ceil_div(P.s0.K, tc::kBK);
+        q.kb1 = P.s1 ? (int)ceil_div(P.s1->K, tc::kBK) : 0;
+        q.bn = P.bn;
+        q.tiles_m = (int)ceil_div(P.M, tc::kBM);
+        q.tiles_n = (int)ceil_div(P.N, P.bn);
+        q.nsplit = P.nsplit;
+        q.kb_per_split = P.kb_per_split;
+        q.tile_begin = tiles;
+        q.ep = eps[i];
+        tiles += q.tiles_m * q.tiles_n * q.nsplit;
+        const double K = (double)P.s0.K + (P.s1 ? (double)P.s1->K : 0.0);
+        flops += 2.0 * P.M * P.N * K;
+        bytes += 2.0 * (P.M + P.N) * K;
+        ++np;
+    }
+    if (np == 0) return NOBLE_OK;
+    g.nproblems = np;
+    g.total_tiles = tiles;
+    g.status = status_ptr();
+    auto kern = tc::gemm_persistent<BN_MAX, A_MN, B_MN, STAGES, Epi>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kDynamic) != cudaSuccess)
+        return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
+    const int grid = tiles < num_sms() ? tiles : num_sms();
+    const KernelInfo ki{name, kBoundTensor, flops, bytes};
+    return run(st, ki, [&] { kern<<<grid, tc::kThreads, SM::kDynamic, st>>>(maps, g); });
+}
+
 // Runtime r -> compile-time N tile for the r-wide products.
 template <class F>
 noble_status with_rank_tile(int64_t r, F &&f)
@@ -425,8 +512,10 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
     const TcSeg main{x, W, di};
     const tc::EpiStore<bf16>::Params py{y, dout, bias, 0};
-    if (r == 0)
-        return tc_gemm<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", T, dout, main, nullptr, 0, 1, py);
+    if (r == 0) {
+        const ProbSpec P{T, dout, main, nullptr, 256};
+        return tc_group<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
+    }
     const SavedLayout SL = saved_layout(d);
     float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
     bf16 *c = (bf16 *)(saved + SL.c);
@@ -444,7 +533,8 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
             T, (int)r, tpb, h, om1, ph1, M, om2, ph2, b, c);
     }));
     const TcSeg up{c, W_up, r};
-    return tc_gemm<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", T, dout, main, &up, 0, 1, py);
+    const ProbSpec P{T, dout, main, &up, 256};
+    return tc_group<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
 }
 
 noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, const bf16 *W, const bf16 *W_down,
@@ -487,32 +577,36 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
                                            WL.n_dm_chunks, r * r)));
         NOBLE_TRY(reduce(st, WL.n_dm_chunks, r * r, r * r, dmpart, dM));
-        // dW_up = dy^T c  [d_out][r];  dW_down = dh^T x  [r][d_in]
-        NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-            constexpr int BN = decltype(bn)::value < 64 ? 64 : decltype(bn)::value;
-            const tc::EpiStore<float>::Params pu{dW_up, r, nullptr, 0};
-            return tc_gemm<BN, true, true, tc::EpiStore<float>>(st, "tc_dW_up", dout, r, TcSeg{dy, c, T}, nullptr,
-                                                                 0, 1, pu);
-        }));
-        const tc::EpiStore<float>::Params pd{dW_down, di, nullptr, 0};
-        NOBLE_TRY((tc_gemm<256, true, true, tc::EpiStore<float>>(st, "tc_dW_down", r, di, TcSeg{dh, x, T}, nullptr,
-                                                                  0, 1, pd)));
     }
     // dx = [dy | dh] [W ; W_down]
-    const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
-    const TcSeg sdx2{dh, W_down, r};
-    NOBLE_TRY((tc_gemm<256, false, true, tc::EpiStore<bf16>>(st, "tc_dx", T, di, TcSeg{dy, W, dout},
-                                                              r > 0 ? &sdx2 : nullptr, 0, 1, px)));
-    // dW = dy^T x
-    const tc::EpiStore<float>::Params pw{dW, di, nullptr, 0};
-    NOBLE_TRY((tc_gemm<256, true, true, tc::EpiStore<float>>(st, "tc_dW", dout, di, TcSeg{dy, x, T}, nullptr, 0, 1,
-                                                              pw)));
+    {
+        const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
+        const TcSeg sdx2{dh, W_down, r};
+        const ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
+        NOBLE_TRY((tc_group<256, false, true, tc::EpiStore<bf16>>(st, "tc_dx", 1, &P, &px)));
+    }
+    // weight gradients in one launch: dW_down = dh^T x, dW_up = dy^T c, dW = dy^T x
+    {
+        const bf16 *c = r > 0 ? (const bf16 *)(saved + SL.c) : nullptr;
+        ProbSpec P[3];
+        tc::EpiStore<float>::Params E[3];
+        int n = 0;
+        if (r > 0) {
+            P[n] = ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256};
+            E[n++] = {dW_down, di, nullptr, 0};
+            P[n] = ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 64 ? 64 : (int)r};
+            E[n++] = {dW_up, r, nullptr, 0};
+        }
+        P[n] = ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256};
+        E[n++] = {dW, di, nullptr, 0};
+        NOBLE_TRY((tc_group<256, true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
+    }
     if (dbias) {
         float *bpart = (float *)(ws + WL.bias_part);
-        dim3 grid((unsigned)ceil_div(dout, 256), (unsigned)WL.n_bias_chunks);
+        dim3 grid((unsigned)ceil_div(dout, 256 * 8), (unsigned)WL.n_bias_chunks);
         const KernelInfo kb{"colsum_dbias", kBoundHbm, (double)T * dout, (double)T * dout * 2};
         NOBLE_TRY(run(st, kb, [&] {
-            simt::colsum_partial<bf16><<<grid, 256, 0, st>>>(T, dout, kBiasChunk, dy, bpart);
+            simt::colsum_partial_bf16x8<<<grid, 256, 0, st>>>(T, dout, kBiasChunk, dy, bpart);
         }));
         NOBLE_TRY(reduce(st, WL.n_bias_chunks, dout, dout, bpart, dbias));
     }

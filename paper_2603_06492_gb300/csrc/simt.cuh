@@ -212,19 +212,59 @@ __global__ void colsum_partial(int64_t T, int64_t n, int64_t rows_per_chunk, con
     part[(int64_t)blockIdx.y * n + o] = s;
 }
 
-// out[k / seg_len][k % seg_len] = sum_p part[p * n + k], p ascending.
+// bf16 column sums, 8 columns (16 bytes) per thread and row: part[c][o] =
+// sum over rows t in chunk c (ascending) of X[t][o].  n must be a multiple of 8.
+__global__ void __launch_bounds__(256) colsum_partial_bf16x8(int64_t T, int64_t n, int64_t rows_per_chunk,
+                                                             const __nv_bfloat16 *X, float *part)
+{
+    const int64_t o = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) * 8;
+    if (o >= n) return;
+    const int64_t tb = (int64_t)blockIdx.y * rows_per_chunk;
+    const int64_t te = min(T, tb + rows_per_chunk);
+    float s[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+    for (int64_t t = tb; t < te; ++t) {
+        const uint4 q = __ldg(reinterpret_cast<const uint4 *>(X + t * n + o));
+        const __nv_bfloat162 *h = reinterpret_cast<const __nv_bfloat162 *>(&q);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(h[i]);
+            s[2 * i] += f.x;
+            s[2 * i + 1] += f.y;
+        }
+    }
+    float4 *dst = reinterpret_cast<float4 *>(part + (int64_t)blockIdx.y * n + o);
+    dst[0] = make_float4(s[0], s[1], s[2], s[3]);
+    dst[1] = make_float4(s[4], s[5], s[6], s[7]);
+}
+
+// out[k / seg_len][k % seg_len] = sum_p part[p * n + k].
+// Block = 8 warps over 32 columns; warp w sums parts [w*P/8, (w+1)*P/8) in
+// ascending order, then the 8 warp sums are added in warp order, so the
+// result does not depend on scheduling.
 struct Outs4 {
     float *p[4];
 };
-__global__ void reduce_partials(int64_t nparts, int64_t n, int64_t seg_len, const float *part,
-                                Outs4 outs)
+__global__ void __launch_bounds__(256) reduce_partials(int64_t nparts, int64_t n, int64_t seg_len,
+                                                       const float *part, Outs4 outs)
 {
-    const int64_t k = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (k >= n) return;
+    __shared__ float sm[8][33];
+    const int lane = threadIdx.x % 32, w = threadIdx.x / 32;
+    const int64_t k = (int64_t)blockIdx.x * 32 + lane;
+    const int64_t per = (nparts + 7) / 8;
+    const int64_t pb = w * per, pe = min(nparts, pb + per);
     float s = 0.f;
-    for (int64_t p = 0; p < nparts; ++p) s += part[p * n + k];
-    float *dst = outs.p[k / seg_len];
-    if (dst) dst[k % seg_len] = s;
+    if (k < n)
+        for (int64_t p = pb; p < pe; ++p) s += part[p * n + k];
+    sm[w][lane] = s;
+    __syncthreads();
+    if (w == 0 && k < n) {
+        float t = 0.f;
+#pragma unroll
+        for (int i = 0; i < 8; ++i) t += sm[i][lane];
+        float *dst = outs.p[k / seg_len];
+        if (dst) dst[k % seg_len] = t;
+    }
 }
 
 // Mt[j][i] = M[i][j]

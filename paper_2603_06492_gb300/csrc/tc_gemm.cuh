@@ -58,6 +58,47 @@ struct EpiStore {
         int64_t split_stride;  // elements between blockIdx.z partial outputs
     };
 
+    // 32 accumulator columns [c, c+32) of this thread's row -> C (+ bias)
+    __device__ static __forceinline__ void store32(const Params &p, OutT *out, const float (&v)[32], int64_t n_base,
+                                                   int64_t N)
+    {
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+            const int64_t n = n_base + g * 8;
+            if (n >= N) break;
+            float f[8];
+#pragma unroll
+            for (int i = 0; i < 8; ++i) f[i] = v[g * 8 + i] + (p.bias ? __ldg(p.bias + n + i) : 0.f);
+            if constexpr (sizeof(OutT) == 2) {
+                uint4 q;
+                q.x = ptx::pack_bf16x2(f[0], f[1]);
+                q.y = ptx::pack_bf16x2(f[2], f[3]);
+                q.z = ptx::pack_bf16x2(f[4], f[5]);
+                q.w = ptx::pack_bf16x2(f[6], f[7]);
+                *reinterpret_cast<uint4 *>(out + n) = q;
+            } else {
+                *reinterpret_cast<float4 *>(out + n) = make_float4(f[0], f[1], f[2], f[3]);
+                *reinterpret_cast<float4 *>(out + n + 4) = make_float4(f[4], f[5], f[6], f[7]);
+            }
+        }
+    }
+
+    // Runtime tile width bn (a multiple of 32), for the persistent kernel.
+    __device__ static void run_dyn(const Params &p, uint32_t tmem, int bn, int quarter, int lane, int64_t m0,
+                                   int64_t n0, int64_t M, int64_t N, int z)
+    {
+        const int64_t row = m0 + quarter * 32 + lane;
+        OutT *out = p.C + (int64_t)z * p.split_stride + row * p.ldc;
+        const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+#pragma unroll 1
+        for (int c = 0; c < bn; c += 32) {
+            if (n0 + c >= N) break;  // warp-uniform: whole chunk past the edge
+            float v[32];
+            ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
+            if (row < M) store32(p, out, v, n0 + c, N);
+        }
+    }
+
     template <int BN>
     __device__ static void run(const Params &p, uint32_t tmem, int quarter, int lane, int64_t m0,
                                int64_t n0, int64_t M, int64_t N, int z)
