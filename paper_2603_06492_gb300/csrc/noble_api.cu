@@ -16,6 +16,7 @@
 #include "simt.cuh"
 #include "tc_gemm.cuh"
 #include "tc_persistent.cuh"
+#include "tc_cosnet.cuh"
 
 namespace noble {
 
@@ -117,30 +118,39 @@ noble_status check_device()
 
 size_t esize(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 ? 2 : 4; }
 
-// Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r].
+// True when the bf16 tensor-core path runs (the default for bf16 operands).
+bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->flags & kFlagSimtOnly); }
+
+// Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r],
+// then (tensor-core path) the bf16 mixing matrix transposed, Mt[j][i] = M[i][j].
 struct SavedLayout {
-    size_t h, b, c, total;
+    size_t h, b, c, mt, total;
 };
 SavedLayout saved_layout(const noble_linear_desc *d)
 {
     SavedLayout L{};
-    if (d->r == 0) return L;
+    if (d->r == 0 || d->T == 0) return L;
     const size_t tr = (size_t)d->T * (size_t)d->r;
     L.h = 0;
     L.b = align_up(L.h + tr * 4, 256);
     L.c = align_up(L.b + tr * 4, 256);
-    L.total = align_up(L.c + tr * esize(d), 256);
+    L.mt = align_up(L.c + tr * esize(d), 256);
+    L.total = align_up(L.mt + (use_tc(d) ? (size_t)d->r * d->r * 2 : 0), 256);
     return L;
 }
 
-constexpr int64_t kDmChunk = 1024;     // tokens per dM partial
-constexpr int64_t kBiasChunk = 128;    // tokens per dbias partial
+constexpr int64_t kDmChunk = 1024;     // tokens per dM partial (CUDA-core path)
+constexpr int64_t kBiasChunk = 128;    // tokens per dbias partial (CUDA-core path)
+constexpr int64_t kOnesCols = 8;       // width of the all-ones operand that yields dbias
 int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
 
-// Backward scratch: dh (dtype), dc, a, db (fp32) [T][r]; Mt fp32 [r][r];
-// per-block partials of the CosNet sums, of dM and of dbias.
+// Backward scratch.
+//   CUDA-core path: dh (dtype), dc, a, db (fp32) [T][r]; M^T fp32; per-block
+//     partials of the CosNet sums, of dM and of dbias.
+//   tensor-core path: dh, a, db (bf16) [T][r]; W_up^T (bf16 [r][d_out]);
+//     M (bf16); an all-ones [T][8] bf16 operand; per-tile CosNet partials.
 struct WorkLayout {
-    size_t dh, dc, a, db, mt, wupt, cos_part, dm_part, bias_part, total;
+    size_t dh, dc, a, db, mt, wupt, mb, ones, cos_part, dm_part, bias_part, total;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
 };
 WorkLayout work_layout(const noble_linear_desc *d)
@@ -151,17 +161,26 @@ WorkLayout work_layout(const noble_linear_desc *d)
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     L.dh = take(tr * esize(d));
-    L.dc = take(tr * 4);
-    L.a = take(tr * 4);
-    L.db = take(tr * 4);
-    L.mt = take((size_t)r * r * 4);
-    L.wupt = take((size_t)r * d->d_out * 2);
-    L.n_cos_blocks = r ? ceil_div(T, cosnet_tokens_per_block(r)) : 0;
-    L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
-    L.n_dm_chunks = r ? ceil_div(T, kDmChunk) : 0;
-    L.dm_part = take((size_t)L.n_dm_chunks * r * r * 4);
-    L.n_bias_chunks = ceil_div(T, kBiasChunk);
-    L.bias_part = take((size_t)L.n_bias_chunks * d->d_out * 4);
+    if (use_tc(d)) {
+        L.a = take(tr * 2);
+        L.db = take(tr * 2);
+        L.wupt = take((size_t)r * d->d_out * 2);
+        L.mb = take((size_t)r * r * 2);
+        L.ones = take((size_t)T * kOnesCols * 2);
+        L.n_cos_blocks = r ? ceil_div(T, 128) : 0;
+        L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
+    } else {
+        L.dc = take(tr * 4);
+        L.a = take(tr * 4);
+        L.db = take(tr * 4);
+        L.mt = take((size_t)r * r * 4);
+        L.n_cos_blocks = r ? ceil_div(T, cosnet_tokens_per_block(r)) : 0;
+        L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
+        L.n_dm_chunks = r ? ceil_div(T, kDmChunk) : 0;
+        L.dm_part = take((size_t)L.n_dm_chunks * r * r * 4);
+        L.n_bias_chunks = ceil_div(T, kBiasChunk);
+        L.bias_part = take((size_t)L.n_bias_chunks * d->d_out * 4);
+    }
     L.total = off < 256 ? 256 : off;
     return L;
 }
@@ -481,27 +500,79 @@ noble_status with_rank_tile(int64_t r, F &&f)
     return fail(NOBLE_ERR_UNSUPPORTED, "rank %lld", (long long)r);
 }
 
-__global__ void transpose_bf16(int64_t rows, int64_t cols, const bf16 *in, bf16 *out)
+// Preparation of the small bf16 operands of the tensor-core path, in one
+// launch: blocks [0, nt) transpose W_up [d_out][r] into wupt [r][d_out] in
+// 32 x 32 tiles; the following blocks convert M (fp32) to bf16, transposed
+// (mt, forward) and/or as is (mb, backward); the rest fill the all-ones
+// [T][kOnesCols] operand.
+__global__ void prep_bf16_kernel(int64_t d_out, int r, const bf16 *W_up, bf16 *wupt, int nt, const float *M,
+                                 bf16 *mt, bf16 *mb, int nm, int64_t ones_n, bf16 *ones)
 {
     __shared__ bf16 tile[32][33];
-    const int64_t c0 = (int64_t)blockIdx.x * 32, r0 = (int64_t)blockIdx.y * 32;
-    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
-        const int64_t rr = r0 + i, cc = c0 + threadIdx.x;
-        if (rr < rows && cc < cols) tile[i][threadIdx.x] = in[rr * cols + cc];
+    const int b = blockIdx.x;
+    if (b < nt) {
+        const int tiles_c = (r + 31) / 32;
+        const int64_t r0 = (int64_t)(b / tiles_c) * 32, c0 = (int64_t)(b % tiles_c) * 32;
+        for (int i = threadIdx.x / 32; i < 32; i += blockDim.x / 32) {
+            const int64_t rr = r0 + i, cc = c0 + threadIdx.x % 32;
+            if (rr < d_out && cc < r) tile[i][threadIdx.x % 32] = W_up[rr * r + cc];
+        }
+        __syncthreads();
+        for (int i = threadIdx.x / 32; i < 32; i += blockDim.x / 32) {
+            const int64_t cc = c0 + i, rr = r0 + threadIdx.x % 32;
+            if (rr < d_out && cc < r) wupt[cc * d_out + rr] = tile[threadIdx.x % 32][i];
+        }
+        return;
     }
-    __syncthreads();
-    for (int i = threadIdx.y; i < 32; i += blockDim.y) {
-        const int64_t cc = c0 + i, rr = r0 + threadIdx.x;
-        if (rr < rows && cc < cols) out[cc * rows + rr] = tile[threadIdx.x][i];
+    if (b < nt + nm) {
+        const int64_t idx = (int64_t)(b - nt) * blockDim.x + threadIdx.x;
+        if (idx < (int64_t)r * r) {
+            const int i = (int)(idx / r), j = (int)(idx % r);
+            const bf16 v = __float2bfloat16_rn(M[idx]);
+            if (mb) mb[idx] = v;
+            if (mt) mt[(int64_t)j * r + i] = v;
+        }
+        return;
     }
+    const int64_t idx = (int64_t)(b - nt - nm) * blockDim.x + threadIdx.x;
+    if (idx < ones_n) ones[idx] = __float2bfloat16_rn(1.f);
 }
 
-noble_status transpose(cudaStream_t st, int64_t rows, int64_t cols, const bf16 *in, bf16 *out)
+noble_status prep_bf16(cudaStream_t st, int64_t d_out, int64_t r, const bf16 *W_up, bf16 *wupt, const float *M,
+                       bf16 *mt, bf16 *mb, int64_t ones_n, bf16 *ones)
 {
-    const KernelInfo ki{"transpose_bf16", kBoundHbm, 0.0, 4.0 * rows * cols};
+    const int nt = wupt ? (int)(ceil_div(d_out, 32) * ceil_div(r, 32)) : 0;
+    const int nm = (mt || mb) ? (int)ceil_div(r * r, 256) : 0;
+    const int no = ones ? (int)ceil_div(ones_n, 256) : 0;
+    if (nt + nm + no == 0) return NOBLE_OK;
+    const KernelInfo ki{"prep_bf16", kBoundHbm, 0.0,
+                        4.0 * (wupt ? d_out * r : 0) + 6.0 * (nm ? r * r : 0) + 2.0 * (ones ? ones_n : 0)};
     return run(st, ki, [&] {
-        transpose_bf16<<<dim3((unsigned)ceil_div(cols, 32), (unsigned)ceil_div(rows, 32)), dim3(32, 8), 0, st>>>(
-            rows, cols, in, out);
+        prep_bf16_kernel<<<nt + nm + no, 256, 0, st>>>(d_out, (int)r, W_up, wupt, nt, M, mt, mb, nm,
+                                                       ones ? ones_n : 0, ones);
+    });
+}
+
+// Fused r-wide GEMM + CosNet launch (forward or backward), one tile per CTA.
+template <int R, bool BWD>
+noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const bf16 *A, int64_t K, const bf16 *B,
+                           const bf16 *Mx, const tc::CosnetArgs &args_in)
+{
+    using Cfg = tc::CosnetCfg<R>;
+    CUtensorMap mA, mB, mM;
+    NOBLE_TRY(make_map(&mA, A, T, K, tc::kBM));
+    NOBLE_TRY(make_map(&mB, B, R, K, R));
+    NOBLE_TRY(make_map(&mM, Mx, R, R, R));
+    tc::CosnetArgs args = args_in;
+    args.T = T;
+    args.kb = (int)ceil_div(K, tc::kBK);
+    args.status = status_ptr();
+    auto kern = tc::cosnet_gemm_kernel<R, BWD>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kDynamic) != cudaSuccess)
+        return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
+    const KernelInfo ki{name, kBoundHbm, 2.0 * T * R * (K + R), 2.0 * T * K + 2.0 * R * K + (BWD ? 14.0 : 10.0) * T * R};
+    return run(st, ki, [&] {
+        kern<<<(unsigned)ceil_div(T, tc::kBM), tc::kThreads, Cfg::kDynamic, st>>>(mA, mB, mM, args);
     });
 }
 
@@ -518,19 +589,13 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     }
     const SavedLayout SL = saved_layout(d);
     float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
-    bf16 *c = (bf16 *)(saved + SL.c);
-    // h = x W_down^T on tensor cores (fp32 out)
+    bf16 *c = (bf16 *)(saved + SL.c), *mt = (bf16 *)(saved + SL.mt);
+    NOBLE_TRY(prep_bf16(st, dout, r, nullptr, nullptr, M, mt, nullptr, 0, nullptr));
+    tc::CosnetArgs a{};
+    a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2;
+    a.h_out = h, a.b_out = b, a.c_out = c;
     NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-        constexpr int BN = decltype(bn)::value;
-        const tc::EpiStore<float>::Params ph{h, r, nullptr, 0};
-        return tc_gemm<BN, false, false, tc::EpiStore<float>>(st, "tc_down_h", T, r, TcSeg{x, W_down, di}, nullptr,
-                                                               0, 1, ph);
-    }));
-    const int tpb = cosnet_tokens_per_block(r);
-    const KernelInfo ki{"simt_cosnet_fwd", kBoundAlu, 2.0 * T * r * r, 0.0};
-    NOBLE_TRY(run(st, ki, [&] {
-        simt::cosnet_fwd_rows<bf16><<<(unsigned)ceil_div(T, tpb), 256, tpb * r * sizeof(float), st>>>(
-            T, (int)r, tpb, h, om1, ph1, M, om2, ph2, b, c);
+        return cosnet_launch<decltype(bn)::value, false>(st, "tc_down_cosnet_fwd", T, x, di, W_down, mt, a);
     }));
     const TcSeg up{c, W_up, r};
     const ProbSpec P{T, dout, main, &up, 256};
@@ -546,37 +611,20 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
     const SavedLayout SL = saved_layout(d);
     const WorkLayout WL = work_layout(d);
-    bf16 *dh = (bf16 *)(ws + WL.dh);
+    bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
+    bf16 *wupt = (bf16 *)(ws + WL.wupt), *mb = (bf16 *)(ws + WL.mb), *ones = (bf16 *)(ws + WL.ones);
+    NOBLE_TRY(prep_bf16(st, dout, r, r ? W_up : nullptr, r ? wupt : nullptr, M, nullptr, r ? mb : nullptr,
+                        dbias ? T * kOnesCols : 0, dbias ? ones : nullptr));
     if (r > 0) {
-        const float *h = (const float *)(saved + SL.h), *b = (const float *)(saved + SL.b);
-        const bf16 *c = (const bf16 *)(saved + SL.c);
-        float *dc = (float *)(ws + WL.dc), *a = (float *)(ws + WL.a), *db = (float *)(ws + WL.db);
-        float *Mt = (float *)(ws + WL.mt), *cpart = (float *)(ws + WL.cos_part);
-        float *dmpart = (float *)(ws + WL.dm_part);
-        bf16 *wupt = (bf16 *)(ws + WL.wupt);
-        // dc = dy W_up, with W_up transposed to K-major [r][d_out] first
-        NOBLE_TRY(transpose(st, dout, r, W_up, wupt));
+        float *cpart = (float *)(ws + WL.cos_part);
+        tc::CosnetArgs ca{};
+        ca.om1 = om1, ca.ph1 = ph1, ca.om2 = om2, ca.ph2 = ph2;
+        ca.h_in = (const float *)(saved + SL.h), ca.b_in = (const float *)(saved + SL.b);
+        ca.dh_out = dh, ca.a_out = a, ca.db_out = db, ca.part = cpart;
         NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-            constexpr int BN = decltype(bn)::value;
-            const tc::EpiStore<float>::Params pc{dc, r, nullptr, 0};
-            return tc_gemm<BN, false, false, tc::EpiStore<float>>(st, "tc_dc", T, r, TcSeg{dy, wupt, dout},
-                                                                   nullptr, 0, 1, pc);
-        }));
-        const KernelInfo kt{"transpose_M", kBoundHbm, 0.0, 8.0 * r * r};
-        NOBLE_TRY(run(st, kt, [&] {
-            simt::transpose_square<<<(unsigned)ceil_div(r * r, 256), 256, 0, st>>>((int)r, M, Mt);
-        }));
-        const int tpb = cosnet_tokens_per_block(r);
-        const KernelInfo kc{"simt_cosnet_bwd", kBoundAlu, 2.0 * T * r * r, 0.0};
-        NOBLE_TRY(run(st, kc, [&] {
-            simt::cosnet_bwd_rows<bf16><<<(unsigned)WL.n_cos_blocks, 256, 5 * tpb * r * sizeof(float), st>>>(
-                T, (int)r, tpb, h, b, dc, om1, ph1, Mt, om2, ph2, dh, a, db, cpart);
+            return cosnet_launch<decltype(bn)::value, true>(st, "tc_dc_cosnet_bwd", T, dy, dout, wupt, mb, ca);
         }));
         NOBLE_TRY(reduce(st, WL.n_cos_blocks, 4 * r, r, cpart, dom1, dph1, dom2, dph2));
-        simt::Seg sdm{{a, 1, r}, {db, 1, r}, T};
-        NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
-                                           WL.n_dm_chunks, r * r)));
-        NOBLE_TRY(reduce(st, WL.n_dm_chunks, r * r, r * r, dmpart, dM));
     }
     // dx = [dy | dh] [W ; W_down]
     {
@@ -585,30 +633,29 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         const ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
         NOBLE_TRY((tc_group<256, false, true, tc::EpiStore<bf16>>(st, "tc_dx", 1, &P, &px)));
     }
-    // weight gradients in one launch: dW_down = dh^T x, dW_up = dy^T c, dW = dy^T x
+    // every token-summed product in one launch: dW_down = dh^T x, dW_up = dy^T c,
+    // dM = a^T db, dbias = dy^T 1, dW = dy^T x
     {
         const bf16 *c = r > 0 ? (const bf16 *)(saved + SL.c) : nullptr;
-        ProbSpec P[3];
-        tc::EpiStore<float>::Params E[3];
+        ProbSpec P[5];
+        tc::EpiStore<float>::Params E[5];
         int n = 0;
         if (r > 0) {
             P[n] = ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256};
             E[n++] = {dW_down, di, nullptr, 0};
             P[n] = ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 64 ? 64 : (int)r};
             E[n++] = {dW_up, r, nullptr, 0};
+            P[n] = ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 64 ? 64 : (int)r};
+            E[n++] = {dM, r, nullptr, 0};
+        }
+        if (dbias) {
+            P[n] = ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 64};
+            E[n] = {dbias, 1, nullptr, 0};
+            E[n++].col0 = 1;
         }
         P[n] = ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256};
         E[n++] = {dW, di, nullptr, 0};
         NOBLE_TRY((tc_group<256, true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
-    }
-    if (dbias) {
-        float *bpart = (float *)(ws + WL.bias_part);
-        dim3 grid((unsigned)ceil_div(dout, 256 * 8), (unsigned)WL.n_bias_chunks);
-        const KernelInfo kb{"colsum_dbias", kBoundHbm, (double)T * dout, (double)T * dout * 2};
-        NOBLE_TRY(run(st, kb, [&] {
-            simt::colsum_partial_bf16x8<<<grid, 256, 0, st>>>(T, dout, kBiasChunk, dy, bpart);
-        }));
-        NOBLE_TRY(reduce(st, WL.n_bias_chunks, dout, dout, bpart, dbias));
     }
     return NOBLE_OK;
 }

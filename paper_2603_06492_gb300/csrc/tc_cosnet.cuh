@@ -1,0 +1,409 @@
+// Fused r-wide GEMM + CosNet kernels (one 128-token tile per CTA, N = r).
+//
+// Forward (Eq. 2; Eqs. 5-7):   h = x W_down^T             (tcgen05, TMEM cols [0, r))
+//   epilogue: a = cos(omega1 h + phi1) -> bf16 tile in shared memory
+//             b = a M                    (second tcgen05 MMA, TMEM cols [R_OFF, R_OFF + r))
+//             c = cos(omega2 b + phi2)
+//   writes h, b (fp32) and c (bf16), each [T][r].
+//
+// Backward (chain rule through Eq. 2):   dc = dy W_up         (tcgen05)
+//   epilogue: du2 = -sin(omega2 b + phi2) dc,  db = omega2 du2 -> bf16 tile
+//             da  = db M^T               (second tcgen05 MMA)
+//             du1 = -sin(omega1 h + phi1) da,  dh = omega1 du1,  a = cos(omega1 h + phi1)
+//   writes dh, a, db (bf16, [T][r]) and per-CTA column sums
+//             part[cta][0] = sum du1*h, [1] = sum du1, [2] = sum du2*b, [3] = sum du2
+//   (each [r]), reduced over the 128 tokens of the tile in a fixed order.
+//
+// The mixing matrix enters as a bf16 K-major operand loaded once per CTA by
+// TMA: Mt[j][i] = M[i][j] for the forward (b_j = sum_i a_i M[i][j]) and M
+// itself for the backward (da_i = sum_j db_j M[i][j]).
+#pragma once
+
+#include "tc_gemm.cuh"
+
+namespace noble {
+namespace tc {
+
+struct CosnetArgs {
+    int64_t T;
+    int kb;              // k-blocks of the main operand (d_in or d_out)
+    const float *om1, *ph1, *om2, *ph2;
+    // forward outputs
+    float *h_out, *b_out;
+    __nv_bfloat16 *c_out;
+    // backward inputs / outputs
+    const float *h_in, *b_in;
+    __nv_bfloat16 *dh_out, *a_out, *db_out;
+    float *part;         // [gridDim.x][4][r]
+    uint32_t *status;
+};
+
+template <int R>
+struct CosnetCfg {
+    static constexpr int kRCols = R < 32 ? 32 : R;         // TMEM columns per accumulator
+    static constexpr uint32_t kTmemCols = 2 * kRCols;     // h|dc and b|da
+    static constexpr uint32_t kA = kBM * kBK * 2;
+    static constexpr uint32_t kB = R * kBK * 2;
+    static constexpr uint32_t kStage = kA + kB;
+    static constexpr int kMkb = (R + 63) / 64;            // k-blocks of the r x r operand
+    static constexpr uint32_t kMBytes = kMkb * R * 128;
+    static constexpr uint32_t kTileBytes = kMkb * kBM * 128;  // epilogue A tile (a or db), bf16
+    static constexpr uint32_t kExtra = 4 * R * 4 + 4 * 4 * R * 4 + 256;  // params, column sums, barriers
+    static constexpr uint32_t kFit = (227u * 1024u - 1024u - kExtra) / kStage;
+    static constexpr int kStages = kFit > 8 ? 8 : (int)kFit;
+    static_assert(kStages >= 2, "pipeline depth");
+    // after the main loop the ring holds the epilogue operand tile and, behind
+    // it, the r x r mixing matrix (loaded by TMA once the ring is free)
+    static constexpr uint32_t kMOff = kTileBytes;  // 1024-aligned
+    static_assert(kTileBytes + kMBytes <= kStages * kStage, "epilogue operands fit in the ring");
+    static constexpr uint32_t kParamOff = kStages * kStage;  // omega/phi copies, 4 x R floats
+    static constexpr uint32_t kPartOff = kParamOff + 4 * R * 4;  // [4 warps][4][R] floats
+    static constexpr uint32_t kBarOff = kPartOff + 4 * 4 * R * 4;
+    static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 3) + 16;
+    static constexpr uint32_t kDynamic = kBytes + 1024;
+};
+
+// Sum over the warp's 32 lanes of each of 32 columns: on return lane l holds
+// the sum of column l.  Fixed butterfly (recursive halving), deterministic.
+__device__ __forceinline__ float warp_colsum32(float (&v)[32])
+{
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int w = 16; w >= 1; w >>= 1) {
+        const bool upper = (lane & w) != 0;
+#pragma unroll
+        for (int i = 0; i < w; ++i) {
+            const float send = upper ? v[i] : v[i + w];
+            const float keep = upper ? v[i + w] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, w);
+        }
+    }
+    return v[0];
+}
+
+// Byte offset of element (row, col) in a 128-row bf16 K-major tile stored as
+// 64-column blocks with the 128-byte swizzle (what TMA writes and UMMA reads).
+__device__ __forceinline__ uint32_t sw128_offset(int row, int col)
+{
+    return (uint32_t)(col >> 6) * (kBM * 128) + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4) + (col & 7) * 2;
+}
+
+template <int R, bool BWD>
+__global__ void __launch_bounds__(kThreads, 1)
+cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
+                   const __grid_constant__ CUtensorMap mM, const CosnetArgs args)
+{
+    using C = CosnetCfg<R>;
+    constexpr int STAGES = C::kStages;
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t raw = ptx::smem_u32(smem_raw);
+    const uint32_t sbase = (raw + 1023u) & ~1023u;
+    uint8_t *smem = smem_raw + (sbase - raw);
+    const uint32_t bar0 = sbase + C::kBarOff;
+    auto full_bar = [&](int s) { return bar0 + 8u * s; };
+    auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
+    const uint32_t tmem_full = bar0 + 8u * (2 * STAGES);
+    const uint32_t m_full = bar0 + 8u * (2 * STAGES + 1);
+    const uint32_t mma2_done = bar0 + 8u * (2 * STAGES + 2);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kBarOff + 8 * (2 * STAGES + 3));
+    float *prm = reinterpret_cast<float *>(smem + C::kParamOff);  // om1 | ph1 | om2 | ph2
+    float *cpart = reinterpret_cast<float *>(smem + C::kPartOff);  // [4][4][R]
+
+    const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
+    const int64_t m0 = (int64_t)blockIdx.x * kBM;
+
+    if (warp == 0 && lane == 0) {
+        ptx::tma_prefetch_desc(&mA);
+        ptx::tma_prefetch_desc(&mB);
+        for (int s = 0; s < STAGES; ++s) {
+            ptx::mbar_init(full_bar(s), 1);
+            ptx::mbar_init(empty_bar(s), 1);
+        }
+        ptx::mbar_init(tmem_full, 1);
+        ptx::mbar_init(m_full, 1);
+        ptx::mbar_init(mma2_done, 1);
+        ptx::fence_barrier_init();
+    }
+    if (warp == 1) {
+        ptx::tmem_alloc(ptx::smem_u32(tmem_slot), C::kTmemCols);
+        ptx::tmem_relinquish();
+    }
+    for (int i = threadIdx.x; i < R; i += blockDim.x) {
+        prm[i] = args.om1[i];
+        prm[R + i] = args.ph1[i];
+        prm[2 * R + i] = args.om2[i];
+        prm[3 * R + i] = args.ph2[i];
+    }
+    ptx::tc_fence_before();
+    __syncthreads();
+    ptx::tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int issued = 0;
+            for (int i = 0; i < args.kb; ++i) {
+                const int s = i % STAGES;
+                const uint32_t ph = (i / STAGES) & 1;
+                if (!ptx::mbar_wait(empty_bar(s), ph ^ 1, args.status)) break;
+                const uint32_t fb = full_bar(s);
+                ptx::mbar_arrive_expect_tx(fb, C::kStage);
+                const uint32_t sA = sbase + s * C::kStage;
+                ptx::tma_load_2d(sA, &mA, fb, i * kBK, (int)m0);
+                ptx::tma_load_2d(sA + C::kA, &mB, fb, i * kBK, 0);
+                ++issued;
+            }
+            for (int i = issued > STAGES ? issued - STAGES : 0; i < issued; ++i)
+                ptx::mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1, nullptr);
+            // mixing matrix into the ring once every main-loop MMA is done
+            if (issued == args.kb && ptx::mbar_wait(tmem_full, 0, args.status)) {
+                ptx::mbar_arrive_expect_tx(m_full, C::kMBytes);
+#pragma unroll
+                for (int kb = 0; kb < C::kMkb; ++kb)
+                    ptx::tma_load_2d(sbase + C::kMOff + kb * R * 128, &mM, m_full, kb * 64, 0);
+                ptx::mbar_wait(m_full, 0, nullptr);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
+            for (int i = 0; i < args.kb; ++i) {
+                const int s = i % STAGES;
+                const uint32_t ph = (i / STAGES) & 1;
+                if (!ptx::mbar_wait(full_bar(s), ph, args.status)) break;
+                ptx::tc_fence_after();
+                const uint32_t sA = sbase + s * C::kStage, sB = sA + C::kA;
+#pragma unroll
+                for (int kk = 0; kk < kBK / 16; ++kk)
+                    ptx::mma_bf16(tmem, ptx::smem_desc_sw128(sA + kk * 32, 16, 1024),
+                                  ptx::smem_desc_sw128(sB + kk * 32, 16, 1024), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                ptx::mma_commit(empty_bar(s));
+            }
+            ptx::mma_commit(tmem_full);
+            ptx::mbar_wait(tmem_full, 0, nullptr);
+        }
+    } else {
+        // ---------------- epilogue: 4 warps, one token row per thread
+        const int quarter = warp % 4;
+        const int row = quarter * 32 + lane;
+        const int64_t t = m0 + row;
+        const bool live = t < args.T;
+        const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+        const uint32_t acc2 = lane_addr + C::kRCols;
+        const float *om1 = prm, *ph1 = prm + R, *om2 = prm + 2 * R, *ph2 = prm + 3 * R;
+        uint8_t *tile = smem;  // the ring is free once the main accumulator is complete
+        bool ok = ptx::mbar_wait(tmem_full, 0, args.status);
+        ok = __all_sync(0xffffffffu, ok);
+        if (ok) {
+            ptx::tc_fence_after();
+            // ---- phase 1: first accumulator -> bf16 operand tile (+ outputs)
+#pragma unroll 1
+            for (int c = 0; c < R; c += 32) {
+                float v[32];
+                if constexpr (R >= 32) {
+                    ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
+                } else {
+                    float w[16];
+                    ptx::tmem_ld_32x32b_x16(lane_addr + c, w);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) v[i] = w[i], v[i + 16] = 0.f;
+                }
+                constexpr int W = R < 32 ? R : 32;
+                if constexpr (!BWD) {
+                    // v = h: store h, operand a = cos(omega1 h + phi1)
+                    if (live) {
+                        float4 *dst = reinterpret_cast<float4 *>(args.h_out + t * R + c);
+#pragma unroll
+                        for (int i = 0; i < W / 4; ++i)
+                            dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                    }
+#pragma unroll
+                    for (int g = 0; g < W / 8; ++g) {
+                        float o[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const int k = c + 8 * g + i;
+                            o[i] = cosf(fmaf(om1[k], v[8 * g + i], ph1[k]));
+                        }
+                        uint4 q;
+                        q.x = ptx::pack_bf16x2(o[0], o[1]);
+                        q.y = ptx::pack_bf16x2(o[2], o[3]);
+                        q.z = ptx::pack_bf16x2(o[4], o[5]);
+                        q.w = ptx::pack_bf16x2(o[6], o[7]);
+                        *reinterpret_cast<uint4 *>(tile + sw128_offset(row, c + 8 * g)) = q;
+                    }
+                } else {
+                    // v = dc; with b of this row: du2, operand db = omega2 du2
+                    float bv[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) bv[i] = 0.f;
+                    if (live) {
+                        const float4 *src = reinterpret_cast<const float4 *>(args.b_in + t * R + c);
+#pragma unroll
+                        for (int i = 0; i < W / 4; ++i) {
+                            const float4 q = __ldg(src + i);
+                            bv[4 * i] = q.x, bv[4 * i + 1] = q.y, bv[4 * i + 2] = q.z, bv[4 * i + 3] = q.w;
+                        }
+                    }
+                    float q2[32], q3[32];
+#pragma unroll
+                    for (int i = W; i < 32; ++i) q2[i] = 0.f, q3[i] = 0.f;
+#pragma unroll
+                    for (int g = 0; g < W / 8; ++g) {
+                        float o[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const int k = c + 8 * g + i, j = 8 * g + i;
+                            const float du2 = live ? -sinf(fmaf(om2[k], bv[j], ph2[k])) * v[j] : 0.f;
+                            o[i] = om2[k] * du2;
+                            q2[j] = du2 * bv[j];
+                            q3[j] = du2;
+                        }
+                        uint4 q;
+                        q.x = ptx::pack_bf16x2(o[0], o[1]);
+                        q.y = ptx::pack_bf16x2(o[2], o[3]);
+                        q.z = ptx::pack_bf16x2(o[4], o[5]);
+                        q.w = ptx::pack_bf16x2(o[6], o[7]);
+                        *reinterpret_cast<uint4 *>(tile + sw128_offset(row, c + 8 * g)) = q;
+                        if (live) *reinterpret_cast<uint4 *>(args.db_out + t * R + c + 8 * g) = q;
+                    }
+                    const float s2 = warp_colsum32(q2);
+                    const float s3 = warp_colsum32(q3);
+                    if (c + lane < R) {
+                        cpart[(quarter * 4 + 2) * R + c + lane] = s2;
+                        cpart[(quarter * 4 + 3) * R + c + lane] = s3;
+                    }
+                }
+            }
+            // ---- second MMA: (128 x r operand tile) x (r x r mixing matrix)
+            ptx::fence_proxy_async_smem();
+            ptx::named_barrier_sync(1, 128);
+            if (threadIdx.x == 64) {
+                bool mok = ptx::mbar_wait(m_full, 0, args.status);
+                ptx::tc_fence_after();
+                if (mok) {
+                    constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
+#pragma unroll
+                    for (int kk = 0; kk < R / 16; ++kk) {
+                        const uint32_t aoff = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
+                        const uint32_t boff = (kk >> 2) * (R * 128) + (kk & 3) * 32;
+                        ptx::mma_bf16(tmem + C::kRCols, ptx::smem_desc_sw128(sbase + aoff, 16, 1024),
+                                      ptx::smem_desc_sw128(sbase + C::kMOff + boff, 16, 1024), idesc,
+                                      kk > 0 ? 1u : 0u);
+                    }
+                }
+                ptx::mma_commit(mma2_done);
+            }
+            ok = ptx::mbar_wait(mma2_done, 0, args.status);
+            ok = __all_sync(0xffffffffu, ok);
+        }
+        if (ok) {
+            ptx::tc_fence_after();
+            // ---- phase 2: second accumulator
+#pragma unroll 1
+            for (int c = 0; c < R; c += 32) {
+                float v[32];
+                if constexpr (R >= 32) {
+                    ptx::tmem_ld_32x32b_x32(acc2 + c, v);
+                } else {
+                    float w[16];
+                    ptx::tmem_ld_32x32b_x16(acc2 + c, w);
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) v[i] = w[i], v[i + 16] = 0.f;
+                }
+                constexpr int W = R < 32 ? R : 32;
+                if constexpr (!BWD) {
+                    // v = b
+                    if (live) {
+                        float4 *dst = reinterpret_cast<float4 *>(args.b_out + t * R + c);
+#pragma unroll
+                        for (int i = 0; i < W / 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+#pragma unroll
+                        for (int g = 0; g < W / 8; ++g) {
+                            float cc[8];
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) cc[i] = cosf(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
+                            uint4 q;
+                            q.x = ptx::pack_bf16x2(cc[0], cc[1]);
+                            q.y = ptx::pack_bf16x2(cc[2], cc[3]);
+                            q.z = ptx::pack_bf16x2(cc[4], cc[5]);
+                            q.w = ptx::pack_bf16x2(cc[6], cc[7]);
+                            *reinterpret_cast<uint4 *>(args.c_out + t * R + c + 8 * g) = q;
+                        }
+                    }
+                } else {
+                    // v = da; with h of this row: du1, dh = omega1 du1, a = cos(u1)
+                    float hv[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) hv[i] = 0.f;
+                    if (live) {
+                        const float4 *src = reinterpret_cast<const float4 *>(args.h_in + t * R + c);
+#pragma unroll
+                        for (int i = 0; i < W / 4; ++i) {
+                            const float4 q = __ldg(src + i);
+                            hv[4 * i] = q.x, hv[4 * i + 1] = q.y, hv[4 * i + 2] = q.z, hv[4 * i + 3] = q.w;
+                        }
+                    }
+                    float q0[32], q1[32];
+#pragma unroll
+                    for (int i = W; i < 32; ++i) q0[i] = 0.f, q1[i] = 0.f;
+#pragma unroll
+                    for (int g = 0; g < W / 8; ++g) {
+                        float dh[8], av[8];
+#pragma unroll
+                        for (int i = 0; i < 8; ++i) {
+                            const int k = c + 8 * g + i, j = 8 * g + i;
+                            float s1, c1;
+                            sincosf(fmaf(om1[k], hv[j], ph1[k]), &s1, &c1);
+                            const float du1 = live ? -s1 * v[j] : 0.f;
+                            dh[i] = om1[k] * du1;
+                            av[i] = c1;
+                            q0[j] = du1 * hv[j];
+                            q1[j] = du1;
+                        }
+                        if (live) {
+                            uint4 q;
+                            q.x = ptx::pack_bf16x2(dh[0], dh[1]);
+                            q.y = ptx::pack_bf16x2(dh[2], dh[3]);
+                            q.z = ptx::pack_bf16x2(dh[4], dh[5]);
+                            q.w = ptx::pack_bf16x2(dh[6], dh[7]);
+                            *reinterpret_cast<uint4 *>(args.dh_out + t * R + c + 8 * g) = q;
+                            q.x = ptx::pack_bf16x2(av[0], av[1]);
+                            q.y = ptx::pack_bf16x2(av[2], av[3]);
+                            q.z = ptx::pack_bf16x2(av[4], av[5]);
+                            q.w = ptx::pack_bf16x2(av[6], av[7]);
+                            *reinterpret_cast<uint4 *>(args.a_out + t * R + c + 8 * g) = q;
+                        }
+                    }
+                    const float s0 = warp_colsum32(q0);
+                    const float s1 = warp_colsum32(q1);
+                    if (c + lane < R) {
+                        cpart[(quarter * 4 + 0) * R + c + lane] = s0;
+                        cpart[(quarter * 4 + 1) * R + c + lane] = s1;
+                    }
+                }
+            }
+            if constexpr (BWD) {
+                // per-CTA column sums: the four warps added in warp order
+                ptx::named_barrier_sync(1, 128);
+                for (int k = threadIdx.x - 64; k < 4 * R; k += 128) {
+                    const int q = k / R, col = k % R;
+                    float s = 0.f;
+#pragma unroll
+                    for (int w = 0; w < 4; ++w) s += cpart[(w * 4 + q) * R + col];
+                    args.part[(int64_t)blockIdx.x * 4 * R + k] = s;
+                }
+            }
+        }
+    }
+
+    ptx::tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        ptx::tc_fence_after();
+        ptx::tmem_dealloc(tmem, C::kTmemCols);
+    }
+}
+
+}  // namespace tc
+}  // namespace noble

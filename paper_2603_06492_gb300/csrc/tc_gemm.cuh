@@ -56,6 +56,7 @@ struct EpiStore {
         int64_t ldc;
         const float *bias;
         int64_t split_stride;  // elements between blockIdx.z partial outputs
+        int col0 = 0;          // store only column 0 of each row, to C[row * ldc]
     };
 
     // 32 accumulator columns [c, c+32) of this thread's row -> C (+ bias)
@@ -90,6 +91,12 @@ struct EpiStore {
         const int64_t row = m0 + quarter * 32 + lane;
         OutT *out = p.C + (int64_t)z * p.split_stride + row * p.ldc;
         const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+        if (p.col0) {
+            float v[32];
+            ptx::tmem_ld_32x32b_x32(lane_addr, v);
+            if (row < M && n0 == 0) *out = (OutT)v[0];
+            return;
+        }
 #pragma unroll 1
         for (int c = 0; c < bn; c += 32) {
             if (n0 + c >= N) break;  // warp-uniform: whole chunk past the edge

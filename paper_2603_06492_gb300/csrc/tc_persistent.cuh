@@ -17,7 +17,7 @@
 namespace noble {
 namespace tc {
 
-constexpr int kMaxProblems = 4;
+constexpr int kMaxProblems = 6;
 
 template <class EpiParams>
 struct Problem {
