@@ -122,7 +122,8 @@ size_t esize(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 ? 2 : 4
 bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->flags & kFlagSimtOnly); }
 
 // Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r],
-// then (tensor-core path) the bf16 mixing matrix transposed, Mt[j][i] = M[i][j].
+// then (tensor-core path) the mixing matrix transposed, Mt[j][i] = M[i][j],
+// as bf16 high and low parts [2][r][r].
 struct SavedLayout {
     size_t h, b, c, mt, total;
 };
@@ -135,7 +136,7 @@ SavedLayout saved_layout(const noble_linear_desc *d)
     L.b = align_up(L.h + tr * 4, 256);
     L.c = align_up(L.b + tr * 4, 256);
     L.mt = align_up(L.c + tr * esize(d), 256);
-    L.total = align_up(L.mt + (use_tc(d) ? (size_t)d->r * d->r * 2 : 0), 256);
+    L.total = align_up(L.mt + (use_tc(d) ? 2 * (size_t)d->r * d->r * 2 : 0), 256);
     return L;
 }
 
@@ -148,7 +149,8 @@ int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
 //   CUDA-core path: dh (dtype), dc, a, db (fp32) [T][r]; M^T fp32; per-block
 //     partials of the CosNet sums, of dM and of dbias.
 //   tensor-core path: dh, a, db (bf16) [T][r]; W_up^T (bf16 [r][d_out]);
-//     M (bf16); an all-ones [T][8] bf16 operand; per-tile CosNet partials.
+//     M as bf16 high and low parts [2][r][r]; an all-ones [T][8] bf16
+//     operand; per-tile CosNet partials.
 struct WorkLayout {
     size_t dh, dc, a, db, mt, wupt, mb, ones, cos_part, dm_part, bias_part, total;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
@@ -165,7 +167,7 @@ WorkLayout work_layout(const noble_linear_desc *d)
         L.a = take(tr * 2);
         L.db = take(tr * 2);
         L.wupt = take((size_t)r * d->d_out * 2);
-        L.mb = take((size_t)r * r * 2);
+        L.mb = take(2 * (size_t)r * r * 2);
         L.ones = take((size_t)T * kOnesCols * 2);
         L.n_cos_blocks = r ? ceil_div(T, 128) : 0;
         L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
@@ -502,9 +504,9 @@ noble_status with_rank_tile(int64_t r, F &&f)
 
 // Preparation of the small bf16 operands of the tensor-core path, in one
 // launch: blocks [0, nt) transpose W_up [d_out][r] into wupt [r][d_out] in
-// 32 x 32 tiles; the following blocks convert M (fp32) to bf16, transposed
-// (mt, forward) and/or as is (mb, backward); the rest fill the all-ones
-// [T][kOnesCols] operand.
+// 32 x 32 tiles; the following blocks split M (fp32) into bf16 high and low
+// parts, transposed (mt, forward) and/or as is (mb, backward); the rest fill
+// the all-ones [T][kOnesCols] operand.
 __global__ void prep_bf16_kernel(int64_t d_out, int r, const bf16 *W_up, bf16 *wupt, int nt, const float *M,
                                  bf16 *mt, bf16 *mb, int nm, int64_t ones_n, bf16 *ones)
 {
@@ -527,10 +529,14 @@ __global__ void prep_bf16_kernel(int64_t d_out, int r, const bf16 *W_up, bf16 *w
     if (b < nt + nm) {
         const int64_t idx = (int64_t)(b - nt) * blockDim.x + threadIdx.x;
         if (idx < (int64_t)r * r) {
+            // high and low bf16 parts, stored as [2][r][r] (rows [0,r) hi, [r,2r) lo)
             const int i = (int)(idx / r), j = (int)(idx % r);
-            const bf16 v = __float2bfloat16_rn(M[idx]);
-            if (mb) mb[idx] = v;
-            if (mt) mt[(int64_t)j * r + i] = v;
+            const float m = M[idx];
+            const bf16 hi = __float2bfloat16_rn(m);
+            const bf16 lo = __float2bfloat16_rn(m - __bfloat162float(hi));
+            const int64_t rr = (int64_t)r * r;
+            if (mb) mb[idx] = hi, mb[rr + idx] = lo;
+            if (mt) mt[(int64_t)j * r + i] = hi, mt[rr + (int64_t)j * r + i] = lo;
         }
         return;
     }
@@ -562,7 +568,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     CUtensorMap mA, mB, mM;
     NOBLE_TRY(make_map(&mA, A, T, K, tc::kBM));
     NOBLE_TRY(make_map(&mB, B, R, K, R));
-    NOBLE_TRY(make_map(&mM, Mx, R, R, R));
+    NOBLE_TRY(make_map(&mM, Mx, 2 * R, R, R));  // [2][R][R]: high then low part
     tc::CosnetArgs args = args_in;
     args.T = T;
     args.kb = (int)ceil_div(K, tc::kBK);

@@ -14,9 +14,16 @@
 //             part[cta][0] = sum du1*h, [1] = sum du1, [2] = sum du2*b, [3] = sum du2
 //   (each [r]), reduced over the 128 tokens of the tile in a fixed order.
 //
-// The mixing matrix enters as a bf16 K-major operand loaded once per CTA by
-// TMA: Mt[j][i] = M[i][j] for the forward (b_j = sum_i a_i M[i][j]) and M
-// itself for the backward (da_i = sum_j db_j M[i][j]).
+// The mixing matrix enters as a bf16 K-major operand loaded by TMA once the
+// main loop is done: Mt[j][i] = M[i][j] for the forward (b_j = sum_i a_i
+// M[i][j]) and M itself for the backward (da_i = sum_j db_j M[i][j]).  Both
+// the row operand (a or db) and the matrix are split into bf16 high and low
+// parts, x = x_hi + x_lo, and the product is formed as
+//     x_hi M_hi + x_lo M_hi + x_hi M_lo
+// with fp32 accumulation, which keeps it close to fp32 accuracy (the dropped
+// x_lo M_lo term is about 2^-16 relative).  A single bf16 product would carry
+// the rounding of M as an error shared by every token, which the sums over
+// tokens of the frequency and phase gradients do not average away.
 #pragma once
 
 #include "tc_gemm.cuh"
@@ -46,20 +53,25 @@ struct CosnetCfg {
     static constexpr uint32_t kB = R * kBK * 2;
     static constexpr uint32_t kStage = kA + kB;
     static constexpr int kMkb = (R + 63) / 64;            // k-blocks of the r x r operand
-    static constexpr uint32_t kMBytes = kMkb * R * 128;
-    static constexpr uint32_t kTileBytes = kMkb * kBM * 128;  // epilogue A tile (a or db), bf16
+    static constexpr int kKSteps = R < 64 ? R / 16 : 4;   // MMA K-steps per k-block
+    static constexpr uint32_t kMkbBytes = 2 * R * 128;    // one k-block of M_hi and M_lo
+    static constexpr uint32_t kTileBytes = kMkb * kBM * 128;  // epilogue row-operand tile, bf16
     static constexpr uint32_t kExtra = 4 * R * 4 + 4 * 4 * R * 4 + 256;  // params, column sums, barriers
     static constexpr uint32_t kFit = (227u * 1024u - 1024u - kExtra) / kStage;
     static constexpr int kStages = kFit > 8 ? 8 : (int)kFit;
     static_assert(kStages >= 2, "pipeline depth");
-    // after the main loop the ring holds the epilogue operand tile and, behind
-    // it, the r x r mixing matrix (loaded by TMA once the ring is free)
-    static constexpr uint32_t kMOff = kTileBytes;  // 1024-aligned
-    static_assert(kTileBytes + kMBytes <= kStages * kStage, "epilogue operands fit in the ring");
-    static constexpr uint32_t kParamOff = kStages * kStage;  // omega/phi copies, 4 x R floats
+    // After the main loop the ring holds the hi and lo row-operand tiles and,
+    // behind them, the mixing matrix in passes of kChunkKb k-blocks.
+    static constexpr uint32_t kRing = kStages * kStage;
+    static constexpr int kFitKb = (int)((kRing - 2 * kTileBytes) / kMkbBytes);
+    static constexpr int kChunkKb = kFitKb >= kMkb ? kMkb : kFitKb;
+    static_assert(kChunkKb >= 1 && kMkb % kChunkKb == 0, "mixing matrix passes");
+    static constexpr int kPasses = kMkb / kChunkKb;
+    static constexpr uint32_t kMOff = 2 * kTileBytes;  // 1024-aligned
+    static constexpr uint32_t kParamOff = kRing;        // omega/phi copies, 4 x R floats
     static constexpr uint32_t kPartOff = kParamOff + 4 * R * 4;  // [4 warps][4][R] floats
     static constexpr uint32_t kBarOff = kPartOff + 4 * 4 * R * 4;
-    static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 3) + 16;
+    static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 4) + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
 
@@ -88,6 +100,28 @@ __device__ __forceinline__ uint32_t sw128_offset(int row, int col)
     return (uint32_t)(col >> 6) * (kBM * 128) + row * 128 + ((((col & 63) >> 3) ^ (row & 7)) << 4) + (col & 7) * 2;
 }
 
+// Row `row`, columns [col, col+8) of the row operand: the bf16 high part goes
+// to the first tile, the bf16 rounding of the remainder to the second tile
+// (kTileBytes further).  Returns the packed high part.
+template <uint32_t kTileBytes>
+__device__ __forceinline__ uint4 store_hi_lo_impl(uint8_t *tile, int row, int col, const float (&o)[8])
+{
+    uint4 hi, lo;
+    uint32_t *ph = &hi.x, *pl = &lo.x;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 h2 = __floats2bfloat162_rn(o[2 * i], o[2 * i + 1]);
+        const float2 hf = __bfloat1622float2(h2);
+        const __nv_bfloat162 l2 = __floats2bfloat162_rn(o[2 * i] - hf.x, o[2 * i + 1] - hf.y);
+        ph[i] = *reinterpret_cast<const uint32_t *>(&h2);
+        pl[i] = *reinterpret_cast<const uint32_t *>(&l2);
+    }
+    const uint32_t off = sw128_offset(row, col);
+    *reinterpret_cast<uint4 *>(tile + off) = hi;
+    *reinterpret_cast<uint4 *>(tile + kTileBytes + off) = lo;
+    return hi;
+}
+
 template <int R, bool BWD>
 __global__ void __launch_bounds__(kThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
@@ -95,6 +129,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 {
     using C = CosnetCfg<R>;
     constexpr int STAGES = C::kStages;
+    auto store_hi_lo = [](uint8_t *tile, int row, int col, const float(&o)[8]) {
+        return store_hi_lo_impl<C::kTileBytes>(tile, row, col, o);
+    };
     extern __shared__ uint8_t smem_raw[];
     const uint32_t raw = ptx::smem_u32(smem_raw);
     const uint32_t sbase = (raw + 1023u) & ~1023u;
@@ -105,7 +142,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
     const uint32_t tmem_full = bar0 + 8u * (2 * STAGES);
     const uint32_t m_full = bar0 + 8u * (2 * STAGES + 1);
     const uint32_t mma2_done = bar0 + 8u * (2 * STAGES + 2);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kBarOff + 8 * (2 * STAGES + 3));
+    const uint32_t m_empty = bar0 + 8u * (2 * STAGES + 3);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kBarOff + 8 * (2 * STAGES + 4));
     float *prm = reinterpret_cast<float *>(smem + C::kParamOff);  // om1 | ph1 | om2 | ph2
     float *cpart = reinterpret_cast<float *>(smem + C::kPartOff);  // [4][4][R]
 
@@ -122,6 +160,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ptx::mbar_init(tmem_full, 1);
         ptx::mbar_init(m_full, 1);
         ptx::mbar_init(mma2_done, 1);
+        ptx::mbar_init(m_empty, 1);
         ptx::fence_barrier_init();
     }
     if (warp == 1) {
@@ -155,13 +194,21 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
             for (int i = issued > STAGES ? issued - STAGES : 0; i < issued; ++i)
                 ptx::mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1, nullptr);
-            // mixing matrix into the ring once every main-loop MMA is done
+            // mixing matrix (rows [0, r) = hi, [r, 2r) = lo) into the ring once
+            // every main-loop MMA is done, kChunkKb k-blocks per pass
             if (issued == args.kb && ptx::mbar_wait(tmem_full, 0, args.status)) {
-                ptx::mbar_arrive_expect_tx(m_full, C::kMBytes);
-#pragma unroll
-                for (int kb = 0; kb < C::kMkb; ++kb)
-                    ptx::tma_load_2d(sbase + C::kMOff + kb * R * 128, &mM, m_full, kb * 64, 0);
-                ptx::mbar_wait(m_full, 0, nullptr);
+                for (int pass = 0; pass < C::kPasses; ++pass) {
+                    if (pass > 0 && !ptx::mbar_wait(m_empty, (pass - 1) & 1, args.status)) break;
+                    const uint32_t mf = m_full;
+                    ptx::mbar_arrive_expect_tx(mf, C::kChunkKb * C::kMkbBytes);
+                    for (int j = 0; j < C::kChunkKb; ++j) {
+                        const int kb = pass * C::kChunkKb + j;
+                        const uint32_t dst = sbase + C::kMOff + j * C::kMkbBytes;
+                        ptx::tma_load_2d(dst, &mM, mf, kb * 64, 0);
+                        ptx::tma_load_2d(dst + R * 128, &mM, mf, kb * 64, R);
+                    }
+                    ptx::mbar_wait(mf, pass & 1, nullptr);
+                }
             }
         }
     } else if (warp == 1) {
@@ -225,12 +272,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                             const int k = c + 8 * g + i;
                             o[i] = cosf(fmaf(om1[k], v[8 * g + i], ph1[k]));
                         }
-                        uint4 q;
-                        q.x = ptx::pack_bf16x2(o[0], o[1]);
-                        q.y = ptx::pack_bf16x2(o[2], o[3]);
-                        q.z = ptx::pack_bf16x2(o[4], o[5]);
-                        q.w = ptx::pack_bf16x2(o[6], o[7]);
-                        *reinterpret_cast<uint4 *>(tile + sw128_offset(row, c + 8 * g)) = q;
+                        store_hi_lo(tile, row, c + 8 * g, o);
                     }
                 } else {
                     // v = dc; with b of this row: du2, operand db = omega2 du2
@@ -259,12 +301,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                             q2[j] = du2 * bv[j];
                             q3[j] = du2;
                         }
-                        uint4 q;
-                        q.x = ptx::pack_bf16x2(o[0], o[1]);
-                        q.y = ptx::pack_bf16x2(o[2], o[3]);
-                        q.z = ptx::pack_bf16x2(o[4], o[5]);
-                        q.w = ptx::pack_bf16x2(o[6], o[7]);
-                        *reinterpret_cast<uint4 *>(tile + sw128_offset(row, c + 8 * g)) = q;
+                        const uint4 q = store_hi_lo(tile, row, c + 8 * g, o);
                         if (live) *reinterpret_cast<uint4 *>(args.db_out + t * R + c + 8 * g) = q;
                     }
                     const float s2 = warp_colsum32(q2);
@@ -279,18 +316,31 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             ptx::fence_proxy_async_smem();
             ptx::named_barrier_sync(1, 128);
             if (threadIdx.x == 64) {
-                bool mok = ptx::mbar_wait(m_full, 0, args.status);
-                ptx::tc_fence_after();
-                if (mok) {
-                    constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
+                constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
+                const uint32_t acc = tmem + C::kRCols;
+                bool mok = true;
+                for (int pass = 0; pass < C::kPasses && mok; ++pass) {
+                    mok = ptx::mbar_wait(m_full, pass & 1, args.status);
+                    ptx::tc_fence_after();
+                    if (!mok) break;
+                    for (int j = 0; j < C::kChunkKb; ++j) {
+                        const int kb = pass * C::kChunkKb + j;
 #pragma unroll
-                    for (int kk = 0; kk < R / 16; ++kk) {
-                        const uint32_t aoff = (kk >> 2) * (kBM * 128) + (kk & 3) * 32;
-                        const uint32_t boff = (kk >> 2) * (R * 128) + (kk & 3) * 32;
-                        ptx::mma_bf16(tmem + C::kRCols, ptx::smem_desc_sw128(sbase + aoff, 16, 1024),
-                                      ptx::smem_desc_sw128(sbase + C::kMOff + boff, 16, 1024), idesc,
-                                      kk > 0 ? 1u : 0u);
+                        for (int kk = 0; kk < C::kKSteps; ++kk) {
+                            const uint32_t a_hi = sbase + kb * (kBM * 128) + kk * 32;
+                            const uint32_t a_lo = a_hi + C::kTileBytes;
+                            const uint32_t m_hi = sbase + C::kMOff + j * C::kMkbBytes + kk * 32;
+                            const uint32_t m_lo = m_hi + R * 128;
+                            const uint64_t dah = ptx::smem_desc_sw128(a_hi, 16, 1024);
+                            const uint64_t dal = ptx::smem_desc_sw128(a_lo, 16, 1024);
+                            const uint64_t dmh = ptx::smem_desc_sw128(m_hi, 16, 1024);
+                            const uint64_t dml = ptx::smem_desc_sw128(m_lo, 16, 1024);
+                            ptx::mma_bf16(acc, dah, dmh, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                            ptx::mma_bf16(acc, dal, dmh, idesc, 1u);
+                            ptx::mma_bf16(acc, dah, dml, idesc, 1u);
+                        }
                     }
+                    if (pass + 1 < C::kPasses) ptx::mma_commit(m_empty);
                 }
                 ptx::mma_commit(mma2_done);
             }
