@@ -646,6 +646,10 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         ProbSpec P[5];
         tc::EpiStore<float>::Params E[5];
         int n = 0;
+        // heaviest tiles first: the round-robin tile walk then fills the
+        // CTAs that drew fewer full tiles with the small ones
+        P[n] = ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256};
+        E[n++] = {dW, di, nullptr, 0};
         if (r > 0) {
             P[n] = ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256};
             E[n++] = {dW_down, di, nullptr, 0};
@@ -659,8 +663,6 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             E[n] = {dbias, 1, nullptr, 0};
             E[n++].col0 = 1;
         }
-        P[n] = ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256};
-        E[n++] = {dW, di, nullptr, 0};
         NOBLE_TRY((tc_group<256, true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
     }
     return NOBLE_OK;

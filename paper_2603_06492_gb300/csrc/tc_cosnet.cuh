@@ -75,6 +75,23 @@ struct CosnetCfg {
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
 
+// Cosine and sine of u for the CosNet epilogues: u is reduced to
+// [-pi, pi] by the two-constant Cody-Waite method (W. J. Cody, W. Waite,
+// "Software Manual for the Elementary Functions", 1980), with 2 pi split into
+// its fp32 rounding C1 = 6.2831854820251465 and the remainder
+// C2 = 2 pi - C1 = -1.7484555e-7, then evaluated with the hardware sin/cos
+// approximation, whose absolute error on [-pi, pi] is about 2^-21.
+// The arguments here are |u| < 100 (|omega h| plus |phi|).
+__device__ __forceinline__ float reduce_two_pi(float u)
+{
+    const float k = rintf(u * 0.159154943091895336f);  // 1 / (2 pi)
+    float r = fmaf(-k, 6.28318548202514648f, u);
+    return fmaf(-k, -1.74845553e-7f, r);
+}
+__device__ __forceinline__ float cos_reduced(float u) { return __cosf(reduce_two_pi(u)); }
+__device__ __forceinline__ float sin_reduced(float u) { return __sinf(reduce_two_pi(u)); }
+__device__ __forceinline__ void sincos_reduced(float u, float *s, float *c) { __sincosf(reduce_two_pi(u), s, c); }
+
 // Sum over the warp's 32 lanes of each of 32 columns: on return lane l holds
 // the sum of column l.  Fixed butterfly (recursive halving), deterministic.
 __device__ __forceinline__ float warp_colsum32(float (&v)[32])
@@ -270,7 +287,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const int k = c + 8 * g + i;
-                            o[i] = cosf(fmaf(om1[k], v[8 * g + i], ph1[k]));
+                            o[i] = cos_reduced(fmaf(om1[k], v[8 * g + i], ph1[k]));
                         }
                         store_hi_lo(tile, row, c + 8 * g, o);
                     }
@@ -296,7 +313,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const int k = c + 8 * g + i, j = 8 * g + i;
-                            const float du2 = live ? -sinf(fmaf(om2[k], bv[j], ph2[k])) * v[j] : 0.f;
+                            const float du2 = live ? -sin_reduced(fmaf(om2[k], bv[j], ph2[k])) * v[j] : 0.f;
                             o[i] = om2[k] * du2;
                             q2[j] = du2 * bv[j];
                             q3[j] = du2;
@@ -372,7 +389,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         for (int g = 0; g < W / 8; ++g) {
                             float cc[8];
 #pragma unroll
-                            for (int i = 0; i < 8; ++i) cc[i] = cosf(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
+                            for (int i = 0; i < 8; ++i) cc[i] = cos_reduced(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
                             uint4 q;
                             q.x = ptx::pack_bf16x2(cc[0], cc[1]);
                             q.y = ptx::pack_bf16x2(cc[2], cc[3]);
@@ -404,7 +421,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         for (int i = 0; i < 8; ++i) {
                             const int k = c + 8 * g + i, j = 8 * g + i;
                             float s1, c1;
-                            sincosf(fmaf(om1[k], hv[j], ph1[k]), &s1, &c1);
+                            sincos_reduced(fmaf(om1[k], hv[j], ph1[k]), &s1, &c1);
                             const float du1 = live ? -s1 * v[j] : 0.f;
                             dh[i] = om1[k] * du1;
                             av[i] = c1;
