@@ -17,6 +17,7 @@
 #include "tc_gemm.cuh"
 #include "tc_persistent.cuh"
 #include "tc_cosnet.cuh"
+#include "tc_pair.cuh"
 
 namespace noble {
 
@@ -488,6 +489,90 @@ noble_status tc_group(cudaStream_t st, const char *name, int n, const ProbSpec *
     return run(st, ki, [&] { kern<<<grid, tc::kThreads, SM::kDynamic, st>>>(maps, g); });
 }
 
+
+// Grouped GEMM on CTA pairs (tc_pair.cuh): every problem's tile width must be
+// 128 or 256.  Tiles are 256 rows (a pair of 128-row halves).
+template <bool A_MN, bool B_MN, class Epi>
+noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbSpec *specs,
+                           const typename Epi::Params *eps)
+{
+    constexpr int STAGES = 6;
+    using SM = tc::pair::PairSmem<STAGES>;
+    if (n < 1 || n > tc::kMaxProblems) return fail(NOBLE_ERR_INVALID_ARG, "%s: %d problems", name, n);
+    tc::GroupMaps maps;
+    tc::GroupArgs<typename Epi::Params> g{};
+    int tiles = 0, np = 0;
+    double flops = 0, bytes = 0;
+    for (int i = 0; i < n; ++i) {
+        const ProbSpec &P = specs[i];
+        if (P.M == 0 || P.N == 0) continue;
+        if (P.bn != 128 && P.bn != 256) return fail(NOBLE_ERR_INVALID_ARG, "%s: pair tile width %d", name, P.bn);
+        const uint32_t bh = (uint32_t)P.bn / 2;
+        auto mk = [&](CUtensorMap *m, const void *p, bool mn, int64_t mnrows, int64_t K, uint32_t box_rows) {
+            return mn ? make_map(m, p, K, mnrows, 64) : make_map(m, p, mnrows, K, box_rows);
+        };
+        NOBLE_TRY(mk(&maps.m[np][0], P.s0.A, A_MN, P.M, P.s0.K, tc::kBM));
+        NOBLE_TRY(mk(&maps.m[np][1], P.s0.B, B_MN, P.N, P.s0.K, bh));
+        if (P.s1) {
+            NOBLE_TRY(mk(&maps.m[np][2], P.s1->A, A_MN, P.M, P.s1->K, tc::kBM));
+            NOBLE_TRY(mk(&maps.m[np][3], P.s1->B, B_MN, P.N, P.s1->K, bh));
+        } else {
+            maps.m[np][2] = maps.m[np][0];
+            maps.m[np][3] = maps.m[np][1];
+        }
+        auto &q = g.p[np];
+        q.M = P.M;
+        q.N = P.N;
+        q.kb0 = (int)ceil_div(P.s0.K, tc::kBK);
+        q.kb1 = P.s1 ? (int)ceil_div(P.s1->K, tc::kBK) : 0;
+        q.bn = P.bn;
+        q.tiles_m = (int)ceil_div(P.M, tc::kBM);
+        q.tiles_n = (int)ceil_div(P.N, P.bn);
+        q.nsplit = P.nsplit;
+        q.kb_per_split = P.kb_per_split;
+        q.tile_begin = tiles;
+        q.ep = eps[i];
+        tiles += (int)ceil_div(q.tiles_m, 2) * q.tiles_n * q.nsplit;
+        const double K = (double)P.s0.K + (P.s1 ? (double)P.s1->K : 0.0);
+        flops += 2.0 * P.M * P.N * K;
+        bytes += 2.0 * (P.M + P.N) * K;
+        ++np;
+    }
+    if (np == 0) return NOBLE_OK;
+    g.nproblems = np;
+    g.total_tiles = tiles;
+    g.status = status_ptr();
+    auto kern = tc::pair::gemm_pair<A_MN, B_MN, STAGES, Epi>;
+    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kDynamic) != cudaSuccess)
+        return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
+    // as many pairs as can be resident at once
+    static int max_clusters_cache[64];
+    int dev = 0;
+    cudaGetDevice(&dev);
+    int max_clusters = (dev >= 0 && dev < 64) ? max_clusters_cache[dev] : 0;
+    if (max_clusters <= 0) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(2 * 64, 1, 1);
+        cfg.blockDim = dim3(tc::kThreads, 1, 1);
+        cfg.dynamicSmemBytes = SM::kDynamic;
+        cudaLaunchAttribute attr;
+        attr.id = cudaLaunchAttributeClusterDimension;
+        attr.val.clusterDim.x = 2;
+        attr.val.clusterDim.y = 1;
+        attr.val.clusterDim.z = 1;
+        cfg.attrs = &attr;
+        cfg.numAttrs = 1;
+        if (cudaOccupancyMaxActiveClusters(&max_clusters, (void *)kern, &cfg) != cudaSuccess || max_clusters <= 0) {
+            cudaGetLastError();
+            max_clusters = num_sms() / 2;
+        }
+        if (dev >= 0 && dev < 64) max_clusters_cache[dev] = max_clusters;
+    }
+    const int clusters = tiles < max_clusters ? tiles : max_clusters;
+    const KernelInfo ki{name, kBoundTensor, flops, bytes};
+    return run(st, ki, [&] { kern<<<2 * clusters, tc::kThreads, SM::kDynamic, st>>>(maps, g); });
+}
+
 // Runtime r -> compile-time N tile for the r-wide products.
 template <class F>
 noble_status with_rank_tile(int64_t r, F &&f)
@@ -591,7 +676,7 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     const tc::EpiStore<bf16>::Params py{y, dout, bias, 0};
     if (r == 0) {
         const ProbSpec P{T, dout, main, nullptr, 256};
-        return tc_group<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
+        return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
     }
     const SavedLayout SL = saved_layout(d);
     float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
@@ -605,7 +690,7 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     }));
     const TcSeg up{c, W_up, r};
     const ProbSpec P{T, dout, main, &up, 256};
-    return tc_group<256, false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
+    return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
 }
 
 noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, const bf16 *W, const bf16 *W_down,
@@ -637,7 +722,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
         const TcSeg sdx2{dh, W_down, r};
         const ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
-        NOBLE_TRY((tc_group<256, false, true, tc::EpiStore<bf16>>(st, "tc_dx", 1, &P, &px)));
+        NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>>(st, "tc_dx", 1, &P, &px)));
     }
     // every token-summed product in one launch: dW_down = dh^T x, dW_up = dy^T c,
     // dM = a^T db, dbias = dy^T 1, dW = dy^T x
@@ -653,17 +738,17 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         if (r > 0) {
             P[n] = ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256};
             E[n++] = {dW_down, di, nullptr, 0};
-            P[n] = ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 64 ? 64 : (int)r};
+            P[n] = ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r};
             E[n++] = {dW_up, r, nullptr, 0};
-            P[n] = ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 64 ? 64 : (int)r};
+            P[n] = ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r};
             E[n++] = {dM, r, nullptr, 0};
         }
         if (dbias) {
-            P[n] = ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 64};
+            P[n] = ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128};
             E[n] = {dbias, 1, nullptr, 0};
             E[n++].col0 = 1;
         }
-        NOBLE_TRY((tc_group<256, true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
+        NOBLE_TRY((tc_pair_group<true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
     }
     return NOBLE_OK;
 }
@@ -899,6 +984,19 @@ noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, 
     const int64_t split_stride = nsplit > 1 ? M * N : 0;
     const tc::EpiStore<float>::Params pf{(float *)C, N, bias, split_stride};
     const tc::EpiStore<bf16>::Params pb{(bf16 *)C, N, bias, split_stride};
+    // N tiles of 128 and 256 run on CTA pairs (the product path's kernel), 64 on
+    // the single-CTA persistent kernel, narrower ones on the one-tile kernel
+    if ((bn == 128 || bn == 256) && !(a_mn && !b_mn)) {
+        const ProbSpec P{M, N, s0, s1, bn, nsplit, kb_per_split};
+#define NOBLE_PAIR_CASE(AMN, BMN)                                                                           \
+    if (a_mn == AMN && b_mn == BMN)                                                                         \
+        return c_fp32 ? tc_pair_group<AMN, BMN, tc::EpiStore<float>>(st, "test", 1, &P, &pf)                \
+                      : tc_pair_group<AMN, BMN, tc::EpiStore<bf16>>(st, "test", 1, &P, &pb);
+        NOBLE_PAIR_CASE(false, false)
+        NOBLE_PAIR_CASE(false, true)
+        NOBLE_PAIR_CASE(true, true)
+#undef NOBLE_PAIR_CASE
+    }
 #define NOBLE_TEST_CASE(BN_, AMN, BMN)                                                                      \
     if (bn == BN_ && a_mn == AMN && b_mn == BMN)                                                            \
         return c_fp32 ? tc_gemm<BN_, AMN, BMN, tc::EpiStore<float>>(st, "test", M, N, s0, s1, kb_per_split,  \
