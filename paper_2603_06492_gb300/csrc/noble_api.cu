@@ -5,6 +5,7 @@
 // Appendix A); backward = the chain rule through the same definitions.
 #include <atomic>
 #include <mutex>
+#include <initializer_list>
 #include <type_traits>
 #include <cstdarg>
 #include <cstdio>
@@ -143,7 +144,7 @@ SavedLayout saved_layout(const noble_linear_desc *d)
 
 constexpr int64_t kDmChunk = 1024;     // tokens per dM partial (CUDA-core path)
 constexpr int64_t kBiasChunk = 128;    // tokens per dbias partial (CUDA-core path)
-constexpr int64_t kOnesCols = 8;       // width of the all-ones operand that yields dbias
+constexpr int64_t kOnesCols = 64;      // width of the all-ones operand that yields dbias
 int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
 
 // Backward scratch.
@@ -345,6 +346,31 @@ noble_status make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t col
     return NOBLE_OK;
 }
 
+// 4-D TMA map over a row-major bf16 matrix [K][MN] (MN contiguous) that loads
+// MN-major tiles in the layout [8-row K group][64-wide MN chunk][8 rows][128 B]:
+// dimensions (inner first) {64 elements, 8 rows, MN/64 chunks, K/8 groups} with
+// strides {P, 128 B, 8 P} for the row pitch P, box {64, 8, nchunks, 8}.
+// Requires MN % 64 == 0 and K % 8 == 0, so that every in-range coordinate of
+// the 4-D description is an element of the matrix.
+noble_status make_map_mn4(CUtensorMap *m, const void *ptr, int64_t K, int64_t MN, uint32_t nchunks)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    if (MN % 64 || K % 8) return fail(NOBLE_ERR_INVALID_ARG, "4-D MN-major map needs MN %% 64 == 0 and K %% 8 == 0");
+    const cuuint64_t P = (cuuint64_t)MN * 2;
+    cuuint64_t dims[4] = {64, 8, (cuuint64_t)MN / 64, (cuuint64_t)K / 8};
+    cuuint64_t strides[3] = {P, 128, 8 * P};
+    cuuint32_t box[4] = {64, 8, nchunks, 8};
+    cuuint32_t estr[4] = {1, 1, 1, 1};
+    CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled (4-D) failed (%d): K=%lld MN=%lld", (int)r, (long long)K,
+                    (long long)MN);
+    return NOBLE_OK;
+}
+
 // Device address of this device's status word (looked up once per device).
 uint32_t *status_ptr()
 {
@@ -492,7 +518,7 @@ noble_status tc_group(cudaStream_t st, const char *name, int n, const ProbSpec *
 
 // Grouped GEMM on CTA pairs (tc_pair.cuh): every problem's tile width must be
 // 128 or 256.  Tiles are 256 rows (a pair of 128-row halves).
-template <bool A_MN, bool B_MN, class Epi>
+template <bool A_MN, bool B_MN, class Epi, bool MN4 = false>
 noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbSpec *specs,
                            const typename Epi::Params *eps)
 {
@@ -509,6 +535,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         if (P.bn != 128 && P.bn != 256) return fail(NOBLE_ERR_INVALID_ARG, "%s: pair tile width %d", name, P.bn);
         const uint32_t bh = (uint32_t)P.bn / 2;
         auto mk = [&](CUtensorMap *m, const void *p, bool mn, int64_t mnrows, int64_t K, uint32_t box_rows) {
+            if (mn && MN4) return make_map_mn4(m, p, K, mnrows, box_rows / 64);
             return mn ? make_map(m, p, K, mnrows, 64) : make_map(m, p, mnrows, K, box_rows);
         };
         NOBLE_TRY(mk(&maps.m[np][0], P.s0.A, A_MN, P.M, P.s0.K, tc::kBM));
@@ -542,11 +569,11 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
     g.nproblems = np;
     g.total_tiles = tiles;
     g.status = status_ptr();
-    auto kern = tc::pair::gemm_pair<A_MN, B_MN, STAGES, Epi>;
+    auto kern = tc::pair::gemm_pair<A_MN, B_MN, STAGES, Epi, MN4>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kDynamic) != cudaSuccess)
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
     // as many pairs as can be resident at once
-    static int max_clusters_cache[64];
+    static int max_clusters_cache[64];  // per instantiation
     int dev = 0;
     cudaGetDevice(&dev);
     int max_clusters = (dev >= 0 && dev < 64) ? max_clusters_cache[dev] : 0;
@@ -667,6 +694,17 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     });
 }
 
+// MN-major operands can use the 4-D layout when every MN extent tiles by 64
+// and every K extent by 8.
+bool mn4_ok(std::initializer_list<int64_t> mn_extents, std::initializer_list<int64_t> k_extents)
+{
+    for (int64_t v : mn_extents)
+        if (v % 64) return false;
+    for (int64_t v : k_extents)
+        if (v % 8) return false;
+    return true;
+}
+
 noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, const float *bias,
                     const bf16 *W_down, const float *om1, const float *ph1, const float *M, const float *om2,
                     const float *ph2, const bf16 *W_up, bf16 *y, char *saved, cudaStream_t st)
@@ -722,7 +760,10 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
         const TcSeg sdx2{dh, W_down, r};
         const ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
-        NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>>(st, "tc_dx", 1, &P, &px)));
+        if (mn4_ok({di}, {dout, r}))
+            NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>, true>(st, "tc_dx", 1, &P, &px)));
+        else
+            NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>>(st, "tc_dx", 1, &P, &px)));
     }
     // every token-summed product in one launch: dW_down = dh^T x, dW_up = dy^T c,
     // dM = a^T db, dbias = dy^T 1, dW = dy^T x
@@ -748,7 +789,10 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             E[n] = {dbias, 1, nullptr, 0};
             E[n++].col0 = 1;
         }
-        NOBLE_TRY((tc_pair_group<true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
+        if (mn4_ok({di, dout, r, kOnesCols}, {T}))
+            NOBLE_TRY((tc_pair_group<true, true, tc::EpiStore<float>, true>(st, "tc_wgrad", n, P, E)));
+        else
+            NOBLE_TRY((tc_pair_group<true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
     }
     return NOBLE_OK;
 }
@@ -988,10 +1032,16 @@ noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, 
     // the single-CTA persistent kernel, narrower ones on the one-tile kernel
     if ((bn == 128 || bn == 256) && !(a_mn && !b_mn)) {
         const ProbSpec P{M, N, s0, s1, bn, nsplit, kb_per_split};
+        // MN-major operands take the 4-D layout when their extents allow it
+        const bool mn4 = mn4_ok({a_mn ? M : 64, b_mn ? N : 64}, {K0, K1});
 #define NOBLE_PAIR_CASE(AMN, BMN)                                                                           \
-    if (a_mn == AMN && b_mn == BMN)                                                                         \
+    if (a_mn == AMN && b_mn == BMN) {                                                                       \
+        if (mn4 && (AMN || BMN))                                                                            \
+            return c_fp32 ? tc_pair_group<AMN, BMN, tc::EpiStore<float>, true>(st, "test", 1, &P, &pf)      \
+                          : tc_pair_group<AMN, BMN, tc::EpiStore<bf16>, true>(st, "test", 1, &P, &pb);      \
         return c_fp32 ? tc_pair_group<AMN, BMN, tc::EpiStore<float>>(st, "test", 1, &P, &pf)                \
-                      : tc_pair_group<AMN, BMN, tc::EpiStore<bf16>>(st, "test", 1, &P, &pb);
+                      : tc_pair_group<AMN, BMN, tc::EpiStore<bf16>>(st, "test", 1, &P, &pb);                \
+    }
         NOBLE_PAIR_CASE(false, false)
         NOBLE_PAIR_CASE(false, true)
         NOBLE_PAIR_CASE(true, true)

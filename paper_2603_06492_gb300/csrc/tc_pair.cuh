@@ -63,6 +63,18 @@ __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap
         : "memory");
 }
 
+// 4-D variant for MN-major operands stored with the 64-wide chunks of each
+// 8-row K group side by side (see make_map_mn4 on the host).
+__device__ __forceinline__ void tma_load_4d_pair(uint32_t dst, const CUtensorMap *map, uint32_t bar_cluster, int c2,
+                                                 int c3)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2 [%0], [%1, {%3, "
+        "%3, %4, %5}], [%2];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(0), "r"(c2), "r"(c3)
+        : "memory");
+}
+
 __device__ __forceinline__ void tmem_alloc2(uint32_t dst_smem, uint32_t ncols)
 {
     asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst_smem), "r"(ncols)
@@ -154,7 +166,11 @@ struct PairSmem {
 };
 
 // Problems of a launch must use bn in {128, 256} (64 or 128 B columns per CTA).
-template <bool A_MN, bool B_MN, int STAGES, class Epi>
+// MN4: MN-major operand tiles are loaded by one 4-D TMA each into the layout
+//   [8-row K group][64-wide MN chunk][8 rows][128 B]
+// (chunk stride 1 KB, group stride nchunks KB) instead of two or more 2-D
+// boxes giving [MN chunk][64 K rows][128 B] (chunk stride 8 KB, group 1 KB).
+template <bool A_MN, bool B_MN, int STAGES, class Epi, bool MN4 = false>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
 gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupArgs<typename Epi::Params> g)
 {
@@ -230,13 +246,17 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     const CUtensorMap *mB = &maps.m[tr.prob][seg1 ? 3 : 1];
                     const int k = (seg1 ? kb - P.kb0 : kb) * kBK;
                     const int nb = (int)tr.n0 + (int)rank * bh;
-                    if (A_MN) {
+                    if (A_MN && MN4) {
+                        tma_load_4d_pair(sA, mA, fb, (int)(tr.m0 / 64), k / 8);
+                    } else if (A_MN) {
                         tma_load_2d_pair(sA, mA, fb, (int)tr.m0, k);
                         tma_load_2d_pair(sA + kChunkBytes, mA, fb, (int)tr.m0 + 64, k);
                     } else {
                         tma_load_2d_pair(sA, mA, fb, k, (int)tr.m0);
                     }
-                    if (B_MN) {
+                    if (B_MN && MN4) {
+                        tma_load_4d_pair(sB, mB, fb, nb / 64, k / 8);
+                    } else if (B_MN) {
                         for (int c = 0; c < bh / 64; ++c) tma_load_2d_pair(sB + c * kChunkBytes, mB, fb, nb + 64 * c, k);
                     } else {
                         tma_load_2d_pair(sB, mB, fb, k, nb);
@@ -276,12 +296,16 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     }
                     ptx::tc_fence_after();
                     const uint32_t sA = sbase + s * S::kStage, sB = sA + S::kA;
+                    const uint32_t nchB = (uint32_t)P.bn / 128;  // 64-wide B chunks held per CTA
 #pragma unroll
                     for (int kk = 0; kk < kBK / 16; ++kk) {
-                        const uint64_t ad = A_MN ? ptx::smem_desc_sw128(sA + kk * 2048, kChunkBytes, 1024)
-                                                 : ptx::smem_desc_sw128(sA + kk * 32, 16, 1024);
-                        const uint64_t bd = B_MN ? ptx::smem_desc_sw128(sB + kk * 2048, kChunkBytes, 1024)
-                                                 : ptx::smem_desc_sw128(sB + kk * 32, 16, 1024);
+                        uint64_t ad, bd;
+                        if (A_MN && MN4) ad = ptx::smem_desc_sw128(sA + kk * 4096, 1024, 2048);
+                        else if (A_MN) ad = ptx::smem_desc_sw128(sA + kk * 2048, kChunkBytes, 1024);
+                        else ad = ptx::smem_desc_sw128(sA + kk * 32, 16, 1024);
+                        if (B_MN && MN4) bd = ptx::smem_desc_sw128(sB + kk * 2048 * nchB, 1024, 1024 * nchB);
+                        else if (B_MN) bd = ptx::smem_desc_sw128(sB + kk * 2048, kChunkBytes, 1024);
+                        else bd = ptx::smem_desc_sw128(sB + kk * 32, 16, 1024);
                         mma2_bf16(d_tmem, ad, bd, idesc, first ? 0u : 1u);
                         first = false;
                     }

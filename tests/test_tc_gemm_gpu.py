@@ -100,3 +100,15 @@ def test_split_k():
 
 def test_large_square():
     run_case(1024, 1024, 2048, 0, 0, 0, 256, 1, seed=5)
+
+
+@pytest.mark.parametrize("amn,bmn,cf", [(0, 1, 0), (1, 1, 1), (1, 1, 0)])
+def test_mnmajor_tiled_layout(amn, bmn, cf):
+    # extents that tile by 64 (MN) and 8 (K): MN-major operands use the 4-D
+    # TMA layout with interleaved 64-wide chunks
+    run_case(384, 512, 1032, 0, amn, bmn, 256, cf, seed=11)
+    run_case(256, 128, 520, 0, amn, bmn, 128, cf, seed=12)
+
+
+def test_mnmajor_tiled_two_segments():
+    run_case(256, 512, 1024, 128, 0, 1, 256, 0, seed=13)
