@@ -3,7 +3,9 @@
 // Host side only: argument validation, buffer carving and kernel dispatch.
 // Forward = Eq. 1 (Section 3.1) with CosNet (Eq. 2, Section 3.2; Eqs. 5-7,
 // Appendix A); backward = the chain rule through the same definitions.
+#include <algorithm>
 #include <atomic>
+#include <vector>
 #include <mutex>
 #include <initializer_list>
 #include <type_traits>
@@ -516,6 +518,61 @@ noble_status tc_group(cudaStream_t st, const char *name, int n, const ProbSpec *
 }
 
 
+
+// Static longest-processing-time-first assignment of the tiles of a grouped
+// launch to its clusters.  A tile's cost is its MMA work (N tile x k-blocks).
+// When all tiles cost the same, round-robin is already balanced and no
+// schedule is built.  Otherwise tiles are taken heaviest first (keeping the
+// L2-friendly order among equal costs) and each goes to the least-loaded
+// cluster; slot j * clusters + c of the schedule holds cluster c's j-th tile.
+template <class GA>
+noble_status pair_schedule(GA &g, int clusters)
+{
+    g.sched_len = 0;
+    struct Item {
+        int id;
+        double cost;
+    };
+    std::vector<Item> items;
+    items.reserve(g.total_tiles);
+    for (int p = 0; p < g.nproblems; ++p) {
+        const auto &P = g.p[p];
+        const int pairs_m = (P.tiles_m + 1) / 2;
+        const int per_split = pairs_m * P.tiles_n;
+        const int kbt = P.kb0 + P.kb1;
+        for (int z = 0; z < P.nsplit; ++z) {
+            int kb = kbt;
+            if (P.kb_per_split > 0) {
+                const int b = z * P.kb_per_split;
+                kb = (b + P.kb_per_split < kbt ? b + P.kb_per_split : kbt) - b;
+            }
+            const double cost = (double)P.bn * kb;
+            for (int i = 0; i < per_split; ++i) items.push_back({P.tile_begin + z * per_split + i, cost});
+        }
+    }
+    bool uniform = true;
+    for (const Item &it : items) uniform = uniform && it.cost == items[0].cost;
+    if (uniform || clusters < 1) return NOBLE_OK;
+    std::stable_sort(items.begin(), items.end(), [](const Item &a, const Item &b) { return a.cost > b.cost; });
+    std::vector<double> load(clusters, 0.0);
+    std::vector<std::vector<int>> lists(clusters);
+    for (const Item &it : items) {
+        int c = 0;
+        for (int k = 1; k < clusters; ++k)
+            if (load[k] < load[c]) c = k;
+        lists[c].push_back(it.id);
+        load[c] += it.cost;
+    }
+    size_t maxlen = 0;
+    for (const auto &l : lists) maxlen = l.size() > maxlen ? l.size() : maxlen;
+    if (maxlen * clusters > (size_t)tc::kMaxSched) return NOBLE_OK;  // too long: round-robin
+    for (size_t j = 0; j < maxlen; ++j)
+        for (int c = 0; c < clusters; ++c)
+            g.sched[j * clusters + c] = j < lists[c].size() ? (uint16_t)lists[c][j] : (uint16_t)0xFFFF;
+    g.sched_len = (int)(maxlen * clusters);
+    return NOBLE_OK;
+}
+
 // Grouped GEMM on CTA pairs (tc_pair.cuh): every problem's tile width must be
 // 128 or 256.  Tiles are 256 rows (a pair of 128-row halves).
 template <bool A_MN, bool B_MN, class Epi, bool MN4 = false>
@@ -596,6 +653,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         if (dev >= 0 && dev < 64) max_clusters_cache[dev] = max_clusters;
     }
     const int clusters = tiles < max_clusters ? tiles : max_clusters;
+    NOBLE_TRY(pair_schedule(g, clusters));
     const KernelInfo ki{name, kBoundTensor, flops, bytes};
     return run(st, ki, [&] { kern<<<2 * clusters, tc::kThreads, SM::kDynamic, st>>>(maps, g); });
 }

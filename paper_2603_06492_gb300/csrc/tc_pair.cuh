@@ -154,6 +154,15 @@ __device__ __forceinline__ PairTile locate_pair(const GroupArgs<EpiParams> &g, i
     return r;
 }
 
+// Tile of the given slot (see GroupArgs::sched); -1 when the slot is empty.
+template <class EpiParams>
+__device__ __forceinline__ int slot_tile(const GroupArgs<EpiParams> &g, int slot)
+{
+    if (g.sched_len == 0) return slot;
+    const int t = g.sched[slot];
+    return t == 0xFFFF ? -1 : t;
+}
+
 template <int STAGES>
 struct PairSmem {
     static constexpr uint32_t kA = kBM * kBK * 2;         // 128 rows of A
@@ -226,7 +235,10 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             // ---------------- producer (both CTAs)
             uint32_t it = 0;
             bool ok = true;
-            for (int t = cluster; ok && t < g.total_tiles; t += nclusters) {
+            const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
+            for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
+                const int t = slot_tile(g, slot);
+                if (t < 0) continue;
                 const PairTile tr = locate_pair(g, t, rank);
                 const auto &P = g.p[tr.prob];
                 const int bh = P.bn / 2;  // B columns held by this CTA
@@ -277,7 +289,10 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             uint32_t it = 0;
             int j = 0;
             bool ok = true;
-            for (int t = cluster; ok && t < g.total_tiles; t += nclusters, ++j) {
+            const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
+            for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
+                const int t = slot_tile(g, slot);
+                if (t < 0) continue;
                 const PairTile tr = locate_pair(g, t, 0);
                 const auto &P = g.p[tr.prob];
                 const int b = j & 1;
@@ -312,6 +327,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     mma2_commit_mc(empty_bar(s), 0x3);
                 }
                 mma2_commit_mc(tfull_bar(b), 0x3);
+                ++j;
             }
             mma2_commit_mc(mma_done, 0x1);
             ptx::mbar_wait(mma_done, 0, nullptr);
@@ -322,7 +338,10 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
         const uint32_t leader_tempty1 = map_to_rank(tempty_bar(1), 0);
         int j = 0;
-        for (int t = cluster; t < g.total_tiles; t += nclusters, ++j) {
+        const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
+        for (int slot = cluster; slot < nslots; slot += nclusters) {
+            const int t = slot_tile(g, slot);
+            if (t < 0) continue;
             const PairTile tr = locate_pair(g, t, rank);
             const auto &P = g.p[tr.prob];
             const int b = j & 1;
@@ -335,6 +354,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(b ? leader_tempty1 : leader_tempty0);
+            ++j;
         }
     }
 

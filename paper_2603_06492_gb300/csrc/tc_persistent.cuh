@@ -30,12 +30,19 @@ struct Problem {
     EpiParams ep;
 };
 
+// Optional explicit schedule (CTA-pair launches): slot j * nclusters + c
+// holds the j-th tile of cluster c, 0xFFFF for none.  sched_len = 0 means
+// plain round-robin over tile indices.
+constexpr int kMaxSched = 2048;
+
 template <class EpiParams>
 struct GroupArgs {
     Problem<EpiParams> p[kMaxProblems];
     int nproblems;
     int total_tiles;
     uint32_t *status;
+    int sched_len;
+    uint16_t sched[kMaxSched];
 };
 
 struct GroupMaps {
