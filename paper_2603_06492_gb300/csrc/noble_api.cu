@@ -748,7 +748,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
     const KernelInfo ki{name, kBoundHbm, 2.0 * T * R * (K + R), 2.0 * T * K + 2.0 * R * K + (BWD ? 14.0 : 10.0) * T * R};
     return run(st, ki, [&] {
-        kern<<<(unsigned)ceil_div(T, tc::kBM), tc::kThreads, Cfg::kDynamic, st>>>(mA, mB, mM, args);
+        kern<<<(unsigned)ceil_div(T, tc::kBM), tc::kCosnetThreads, Cfg::kDynamic, st>>>(mA, mB, mM, args);
     });
 }
 

@@ -139,8 +139,12 @@ __device__ __forceinline__ uint4 store_hi_lo_impl(uint8_t *tile, int row, int co
     return hi;
 }
 
+// Warps 0 (TMA) and 1 (MMA, TMEM owner) plus eight epilogue warps: two per
+// TMEM lane quarter, taking alternate 32-column chunks of their 32 rows.
+constexpr int kCosnetThreads = 320;
+
 template <int R, bool BWD>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kCosnetThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mM, const CosnetArgs args)
 {
@@ -247,8 +251,10 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             ptx::mbar_wait(tmem_full, 0, nullptr);
         }
     } else {
-        // ---------------- epilogue: 4 warps, one token row per thread
+        // ---------------- epilogue: 8 warps; a thread owns one token row and
+        // the 32-column chunks c with (c / 32) % 2 == half
         const int quarter = warp % 4;
+        const int half = (warp - 2) / 4;
         const int row = quarter * 32 + lane;
         const int64_t t = m0 + row;
         const bool live = t < args.T;
@@ -262,7 +268,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             ptx::tc_fence_after();
             // ---- phase 1: first accumulator -> bf16 operand tile (+ outputs)
 #pragma unroll 1
-            for (int c = 0; c < R; c += 32) {
+            for (int c = 32 * half; c < R; c += 64) {
                 float v[32];
                 if constexpr (R >= 32) {
                     ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
@@ -331,7 +337,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
             // ---- second MMA: (128 x r operand tile) x (r x r mixing matrix)
             ptx::fence_proxy_async_smem();
-            ptx::named_barrier_sync(1, 128);
+            ptx::named_barrier_sync(1, 256);
             if (threadIdx.x == 64) {
                 constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
                 const uint32_t acc = tmem + C::kRCols;
@@ -368,7 +374,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             ptx::tc_fence_after();
             // ---- phase 2: second accumulator
 #pragma unroll 1
-            for (int c = 0; c < R; c += 32) {
+            for (int c = 32 * half; c < R; c += 64) {
                 float v[32];
                 if constexpr (R >= 32) {
                     ptx::tmem_ld_32x32b_x32(acc2 + c, v);
@@ -452,8 +458,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
             if constexpr (BWD) {
                 // per-CTA column sums: the four warps added in warp order
-                ptx::named_barrier_sync(1, 128);
-                for (int k = threadIdx.x - 64; k < 4 * R; k += 128) {
+                ptx::named_barrier_sync(1, 256);
+                for (int k = threadIdx.x - 64; k < 4 * R; k += 256) {
                     const int q = k / R, col = k % R;
                     float s = 0.f;
 #pragma unroll

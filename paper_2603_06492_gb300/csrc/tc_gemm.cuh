@@ -76,10 +76,12 @@ struct EpiStore {
                 q.y = ptx::pack_bf16x2(f[2], f[3]);
                 q.z = ptx::pack_bf16x2(f[4], f[5]);
                 q.w = ptx::pack_bf16x2(f[6], f[7]);
-                *reinterpret_cast<uint4 *>(out + n) = q;
+                // streaming stores: outputs are not read again by this kernel
+                // and should not push its operands out of L2
+                __stcs(reinterpret_cast<uint4 *>(out + n), q);
             } else {
-                *reinterpret_cast<float4 *>(out + n) = make_float4(f[0], f[1], f[2], f[3]);
-                *reinterpret_cast<float4 *>(out + n + 4) = make_float4(f[4], f[5], f[6], f[7]);
+                __stcs(reinterpret_cast<float4 *>(out + n), make_float4(f[0], f[1], f[2], f[3]));
+                __stcs(reinterpret_cast<float4 *>(out + n + 4), make_float4(f[4], f[5], f[6], f[7]));
             }
         }
     }
