@@ -34,7 +34,19 @@ sys.path.insert(0, ROOT)
 from paper_2603_06492_gb300.inputs import CONFIGS, layer_seed, make_layer_inputs  # noqa: E402
 
 CONFIG_INDEX = 3
-WORKLOAD = "1.5B-scale FFN up/down + QKV, T=16384, d=2048, r=128, CosNet, fwd+bwd"
+WORKLOADS = {
+    0: "tiny correctness case, T=256, 128->128, r=16, fp32, fwd+bwd",
+    1: "250M-scale attention QKV + output, T=8192, d=1024, r=64, CosNet, fwd+bwd",
+    2: "250M-scale FFN up + down, T=8192, d=1024, r=64, CosNet, fwd+bwd",
+    3: "1.5B-scale FFN up/down + QKV, T=16384, d=2048, r=128, CosNet, fwd+bwd",
+    4: "ViT-Base-shaped QKV + FFN up/down, T=50432, d=768, r in {16..256}, CosNet, fwd+bwd",
+}
+
+# DRAM bytes per launch of each tensor-core kernel class on the 1.5B-scale
+# workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, mean over the
+# three layers' launches of one fwd+bwd).  Valid for the kernels as they are
+# built now; a kernel change invalidates its entry.
+TRAFFIC_PER_LAUNCH = {3: {"tc_wgrad": 1015.8e6, "tc_main_up_fwd": 485.6e6, "tc_dx": 540.4e6}}
 METRIC = "NOBLE linear fwd+bwd TFLOP/s"
 
 
@@ -135,7 +147,7 @@ def run_reference(args, rank):
     """--impl reference: the oracle as it stands, on host cores, rank 0 only."""
     if rank != 0:
         return
-    layers = CONFIGS[CONFIG_INDEX]
+    layers = CONFIGS[args.config]
     import oracle
     oracle.build()
     for _ in range(args.warmup):
@@ -146,13 +158,13 @@ def run_reference(args, rank):
         secs += t
         flops += f
     v = flops / secs / 1e12
-    sample = (f"first {args.ref_tokens} of 16384 tokens of each of the 3 layers per step "
-              f"(fwd+bwd, fp64)")
+    sample = (f"first {args.ref_tokens} of {layers[0].T} tokens of each of the {len(layers)} layers "
+              f"per step (fwd+bwd, fp64)")
     line = {"impl": "reference", "metric": METRIC, "value": v, "unit": "TFLOP/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOAD, "sample": sample},
+            "config": {"workload": WORKLOADS[args.config], "config_index": args.config, "sample": sample},
             "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": host_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
@@ -176,6 +188,10 @@ def main():
     ap.add_argument("--profile-run", action="store_true",
                     help="fwd+bwd of the selected layers only, for ncu; prints no bench line")
     ap.add_argument("--layers", default="", help="comma-separated layer names (default: all)")
+    ap.add_argument("--config", type=int, default=CONFIG_INDEX,
+                    help="workload: configuration 0-4 (default 3, the headline)")
+    ap.add_argument("--per-layer", action="store_true",
+                    help="also time every layer alone (NOBLE and plain) and report each")
     args = ap.parse_args()
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -200,14 +216,15 @@ def main():
     binding.load()
     assert args.profile_run or args.warmup >= 3, "at least 3 warm-up steps"
 
-    layers = CONFIGS[CONFIG_INDEX]
+    cfg = args.config
+    layers = CONFIGS[cfg]
     if args.layers:
         keep = set(args.layers.split(","))
         layers = [l for l in layers if l.name in keep]
     dev_inputs, bufs, plain_bufs = [], [], []
     for layer in layers:
-        li = [l.name for l in CONFIGS[CONFIG_INDEX]].index(layer.name)
-        inp = make_layer_inputs(layer, layer_seed(CONFIG_INDEX, li))
+        li = [l.name for l in CONFIGS[cfg]].index(layer.name)
+        inp = make_layer_inputs(layer, layer_seed(cfg, li))
         dev_inputs.append(binding.params_to_device(inp, layer.dtype))
         del inp
         bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype))
@@ -284,7 +301,8 @@ def main():
         else:  # fp32 FMA pipe: 152 SMs x 128 lanes x 2 FLOP x max SM clock
             peak, unit = 152 * 128 * 2 * pk["sm_max_mhz"] * 1e6 / 1e12, "TFLOP/s"
         roof = {"bound": top["bound"], "kernel": top["name"], "achieved": achieved, "peak": peak,
-                "unit": unit, "frac": achieved / peak, "traffic": None,
+                "unit": unit, "frac": achieved / peak,
+                "traffic": TRAFFIC_PER_LAUNCH.get(cfg, {}).get(top["name"]) if not args.layers else None,
                 "peak_src": ("measured sustained" if top["bound"] == "tensor" else
                              "measured" if top["bound"] == "hbm" else "derived from unit counts"),
                 "share_of_step": top["ms"] / ms, "launches_per_step": top["launches"] / args.steps}
@@ -376,6 +394,28 @@ def main():
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e,
                "copies": "pinned host buffers, copy streams overlapping compute"}
 
+    per_layer = None
+    if args.per_layer:
+        per_layer = {}
+        for li, layer in enumerate(layers):
+            d, b, bp = dev_inputs[li], bufs[li], plain_bufs[li]
+
+            def one(plain=False, d=d, b=b, bp=bp):
+                p = {k: d[k] for k in ("W", "bias")} if plain else d
+                bb = bp if plain else b
+                binding.forward(bb, d["x"], p, stream)
+                binding.backward(bb, d["x"], d["dy"], p, stream)
+
+            for _ in range(2):
+                one()
+                one(True)
+            t_n = timed(one, args.steps) / args.steps
+            t_p = timed(lambda: one(True), args.steps) / args.steps
+            per_layer[layer.name] = {
+                "ms": t_n, "tflops": world * layer.flops() / (t_n * 1e-3) / 1e12,
+                "plain_ms": t_p, "plain_tflops": world * layer.plain().flops() / (t_p * 1e-3) / 1e12,
+                "overhead_vs_plain": t_n / t_p - 1.0}
+
     # cuBLAS reference timing of the plain layer (torch.matmul x3), context only
     def cublas_step():
         for d in dev_inputs:
@@ -391,16 +431,17 @@ def main():
     if rank == 0 and not args.no_cpu_baseline:
         secs, fl = oracle_sample(layers, args.cpu_tokens)
         cpu = {"value": fl / secs / 1e12, "unit": "TFLOP/s", "cores": host_cores(), "kind": "oracle",
-               "sample": f"fwd+bwd of the first {args.cpu_tokens} of 16384 tokens of each layer, fp64",
+               "sample": f"fwd+bwd of the first {args.cpu_tokens} of {layers[0].T} tokens of each layer, fp64",
                "seconds": secs}
 
     if rank == 0:
         line = {
             "metric": METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_step,
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16" if layers[0].dtype == "bf16" else "f32",
             "data": "synthetic",
-            "config": {"workload": WORKLOAD, "layers": [
+            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "layers": [
                 {"name": l.name, "T": l.T, "d_in": l.d_in, "d_out": l.d_out, "r": l.r} for l in layers],
                 "l2": "inputs larger than L2: each step streams ~1.8 GB of activations",
                 "parallelism": f"replicas x{world}"},
@@ -412,7 +453,7 @@ def main():
             "overhead_vs_plain": ms_step / (ms_plain / args.steps) - 1.0,
             "cublas_plain_ms_per_step": ms_cublas,
             "overhead_vs_cublas_plain": ms_step / ms_cublas - 1.0,
-            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e,
+            "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "per_layer": per_layer,
             "gpu_launches": launches,
             "kernel_breakdown": {k: {"ms_per_step": v["ms"] / args.steps,
                                      "launches_per_step": v["launches"] / args.steps}
