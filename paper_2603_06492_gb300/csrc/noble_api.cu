@@ -149,6 +149,33 @@ constexpr int64_t kBiasChunk = 128;    // tokens per dbias partial (CUDA-core pa
 constexpr int64_t kOnesCols = 64;      // width of the all-ones operand that yields dbias
 int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
 
+// K split of the grouped weight-gradient launch (tensor-core path).  When the
+// launch has fewer than two waves of 256 x N tile pairs for a GB300 (74
+// resident CTA pairs), K = T is cut into s chunks of at least 16 k-blocks;
+// each chunk writes an fp32 partial and one reduction adds them in chunk
+// order.  A function of the shape only, so buffer sizes do not depend on the
+// device.
+constexpr int kAssumedPairs = 74;
+int wgrad_tiles(int64_t M, int64_t N, int bn) { return (int)(ceil_div(ceil_div(M, 128), 2) * ceil_div(N, bn)); }
+int wgrad_split(const noble_linear_desc *d)
+{
+    const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
+    const int rb = r < 128 ? 128 : (int)r;
+    int tiles = wgrad_tiles(dout, di, 256) + wgrad_tiles(dout, kOnesCols, 128);
+    if (r > 0) tiles += wgrad_tiles(r, di, 256) + wgrad_tiles(dout, r, rb) + wgrad_tiles(r, r, rb);
+    const int64_t kb = ceil_div(T, 64);
+    int s = (int)ceil_div(2 * kAssumedPairs, tiles);
+    if (s > kb / 16) s = (int)(kb / 16);
+    return s < 1 ? 1 : s;
+}
+// Sizes of the five token-summed products (M x N), in launch order.
+void wgrad_shapes(const noble_linear_desc *d, int64_t (&mn)[5][2])
+{
+    const int64_t di = d->d_in, dout = d->d_out, r = d->r;
+    const int64_t v[5][2] = {{dout, di}, {r, di}, {dout, r}, {r, r}, {dout, 1}};
+    for (int i = 0; i < 5; ++i) mn[i][0] = v[i][0], mn[i][1] = v[i][1];
+}
+
 // Backward scratch.
 //   CUDA-core path: dh (dtype), dc, a, db (fp32) [T][r]; M^T fp32; per-block
 //     partials of the CosNet sums, of dM and of dbias.
@@ -156,7 +183,8 @@ int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
 //     M as bf16 high and low parts [2][r][r]; an all-ones [T][8] bf16
 //     operand; per-tile CosNet partials.
 struct WorkLayout {
-    size_t dh, dc, a, db, mt, wupt, mb, ones, cos_part, dm_part, bias_part, total;
+    size_t dh, dc, a, db, mt, wupt, mb, ones, cos_part, dm_part, bias_part, wsplit[5], total;
+    int split;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
 };
 WorkLayout work_layout(const noble_linear_desc *d)
@@ -175,6 +203,12 @@ WorkLayout work_layout(const noble_linear_desc *d)
         L.ones = take((size_t)T * kOnesCols * 2);
         L.n_cos_blocks = r ? ceil_div(T, 128) : 0;
         L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
+        L.split = wgrad_split(d);
+        if (L.split > 1) {
+            int64_t mn[5][2];
+            wgrad_shapes(d, mn);
+            for (int i = 0; i < 5; ++i) L.wsplit[i] = take((size_t)L.split * mn[i][0] * mn[i][1] * 4);
+        }
     } else {
         L.dc = take(tr * 4);
         L.a = take(tr * 4);
@@ -637,7 +671,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
     if (max_clusters <= 0) {
         cudaLaunchConfig_t cfg = {};
         cfg.gridDim = dim3(2 * 64, 1, 1);
-        cfg.blockDim = dim3(tc::kThreads, 1, 1);
+        cfg.blockDim = dim3(tc::pair::kPairThreads, 1, 1);
         cfg.dynamicSmemBytes = SM::kDynamic;
         cudaLaunchAttribute attr;
         attr.id = cudaLaunchAttributeClusterDimension;
@@ -655,7 +689,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
     const int clusters = tiles < max_clusters ? tiles : max_clusters;
     NOBLE_TRY(pair_schedule(g, clusters));
     const KernelInfo ki{name, kBoundTensor, flops, bytes};
-    return run(st, ki, [&] { kern<<<2 * clusters, tc::kThreads, SM::kDynamic, st>>>(maps, g); });
+    return run(st, ki, [&] { kern<<<2 * clusters, tc::pair::kPairThreads, SM::kDynamic, st>>>(maps, g); });
 }
 
 // Runtime r -> compile-time N tile for the r-wide products.
@@ -727,6 +761,27 @@ noble_status prep_bf16(cudaStream_t st, int64_t d_out, int64_t r, const bf16 *W_
         prep_bf16_kernel<<<nt + nm + no, 256, 0, st>>>(d_out, (int)r, W_up, wupt, nt, M, mt, mb, nm,
                                                        ones ? ones_n : 0, ones);
     });
+}
+
+// Sum of K-split partials: out_j[i] = sum_z part_j[z][i] (z ascending) for
+// up to five outputs in one launch.
+struct SplitJobs {
+    const float *part[5];
+    float *out[5];
+    int64_t n[5], begin[6];
+    int nparts;
+    int njobs;
+};
+__global__ void reduce_split_kernel(SplitJobs J)
+{
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= J.begin[J.njobs]) return;
+    int j = 0;
+    while (idx >= J.begin[j + 1]) ++j;
+    const int64_t i = idx - J.begin[j];
+    float s = 0.f;
+    for (int z = 0; z < J.nparts; ++z) s += J.part[j][(int64_t)z * J.n[j] + i];
+    J.out[j][i] = s;
 }
 
 // Fused r-wide GEMM + CosNet launch (forward or backward), one tile per CTA.
@@ -829,28 +884,60 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         const bf16 *c = r > 0 ? (const bf16 *)(saved + SL.c) : nullptr;
         ProbSpec P[5];
         tc::EpiStore<float>::Params E[5];
+        float *final_out[5];
+        int64_t mn[5][2];
+        wgrad_shapes(d, mn);
+        int which[5];
         int n = 0;
+        auto add = [&](int k, ProbSpec ps, float *out, int64_t ldc, bool col0) {
+            P[n] = ps;
+            E[n] = {out, ldc, nullptr, 0};
+            E[n].col0 = col0 ? 1 : 0;
+            final_out[n] = out;
+            which[n++] = k;
+        };
         // heaviest tiles first: the round-robin tile walk then fills the
         // CTAs that drew fewer full tiles with the small ones
-        P[n] = ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256};
-        E[n++] = {dW, di, nullptr, 0};
+        add(0, ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256}, dW, di, false);
         if (r > 0) {
-            P[n] = ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256};
-            E[n++] = {dW_down, di, nullptr, 0};
-            P[n] = ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r};
-            E[n++] = {dW_up, r, nullptr, 0};
-            P[n] = ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r};
-            E[n++] = {dM, r, nullptr, 0};
+            add(1, ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256}, dW_down, di, false);
+            add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false);
+            add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);
         }
-        if (dbias) {
-            P[n] = ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128};
-            E[n] = {dbias, 1, nullptr, 0};
-            E[n++].col0 = 1;
+        if (dbias) add(4, ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128}, dbias, 1, true);
+        const int split = WL.split;
+        SplitJobs J{};
+        if (split > 1) {
+            const int kbt = (int)ceil_div(T, tc::kBK);
+            const int per = (int)ceil_div(kbt, split);
+            J.nparts = (int)ceil_div(kbt, per);
+            J.begin[0] = 0;
+            for (int i = 0; i < n; ++i) {
+                const int k = which[i];
+                float *part = (float *)(ws + WL.wsplit[k]);
+                P[i].nsplit = J.nparts;
+                P[i].kb_per_split = per;
+                E[i].C = part;
+                E[i].split_stride = mn[k][0] * mn[k][1];
+                J.part[i] = part;
+                J.out[i] = final_out[i];
+                J.n[i] = mn[k][0] * mn[k][1];
+                J.begin[i + 1] = J.begin[i] + J.n[i];
+            }
+            J.njobs = n;
         }
         if (mn4_ok({di, dout, r, kOnesCols}, {T}))
             NOBLE_TRY((tc_pair_group<true, true, tc::EpiStore<float>, true>(st, "tc_wgrad", n, P, E)));
         else
             NOBLE_TRY((tc_pair_group<true, true, tc::EpiStore<float>>(st, "tc_wgrad", n, P, E)));
+        if (split > 1) {
+            const int64_t total = J.begin[J.njobs];
+            const KernelInfo kr{"reduce_wgrad_split", kBoundHbm, (double)total * J.nparts,
+                                4.0 * total * (J.nparts + 1)};
+            NOBLE_TRY(run(st, kr, [&] {
+                reduce_split_kernel<<<(unsigned)ceil_div(total, 256), 256, 0, st>>>(J);
+            }));
+        }
     }
     return NOBLE_OK;
 }

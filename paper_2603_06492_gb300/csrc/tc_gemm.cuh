@@ -86,21 +86,23 @@ struct EpiStore {
         }
     }
 
-    // Runtime tile width bn (a multiple of 32), for the persistent kernel.
+    // Runtime tile width bn (a multiple of 32), for the persistent kernels.
+    // This warp stores the 32-column chunks c0, c0 + cstep, ... of its rows.
     __device__ static void run_dyn(const Params &p, uint32_t tmem, int bn, int quarter, int lane, int64_t m0,
-                                   int64_t n0, int64_t M, int64_t N, int z)
+                                   int64_t n0, int64_t M, int64_t N, int z, int c0 = 0, int cstep = 32)
     {
         const int64_t row = m0 + quarter * 32 + lane;
         OutT *out = p.C + (int64_t)z * p.split_stride + row * p.ldc;
         const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
         if (p.col0) {
+            if (c0 != 0) return;
             float v[32];
             ptx::tmem_ld_32x32b_x32(lane_addr, v);
             if (row < M && n0 == 0) *out = (OutT)v[0];
             return;
         }
 #pragma unroll 1
-        for (int c = 0; c < bn; c += 32) {
+        for (int c = c0; c < bn; c += cstep) {
             if (n0 + c >= N) break;  // warp-uniform: whole chunk past the edge
             float v[32];
             ptx::tmem_ld_32x32b_x32(lane_addr + c, v);

@@ -15,8 +15,9 @@
 //   * MMA (warp 1 of the leader only): waits `full`, issues the pair MMAs,
 //     commits to `empty` of both CTAs (multicast) and, per tile, to `tfull`
 //     of both CTAs.
-//   * epilogue (warps 2-5 of each CTA): reads its own accumulator rows and
-//     arrives on the LEADER's `tempty` (8 arrivals: 4 warps x 2 CTAs).
+//   * epilogue (warps 2-9 of each CTA, two per TMEM lane quarter taking
+//     alternate 32-column chunks): reads its own accumulator rows and
+//     arrives on the LEADER's `tempty` (16 arrivals: 8 warps x 2 CTAs).
 // All waits are bounded as in the single-CTA kernels.
 #pragma once
 
@@ -163,6 +164,9 @@ __device__ __forceinline__ int slot_tile(const GroupArgs<EpiParams> &g, int slot
     return t == 0xFFFF ? -1 : t;
 }
 
+// Warps 0 (TMA), 1 (MMA, TMEM owner) and eight epilogue warps.
+constexpr int kPairThreads = 320;
+
 template <int STAGES>
 struct PairSmem {
     static constexpr uint32_t kA = kBM * kBK * 2;         // 128 rows of A
@@ -180,7 +184,7 @@ struct PairSmem {
 // (chunk stride 1 KB, group stride nchunks KB) instead of two or more 2-D
 // boxes giving [MN chunk][64 K rows][128 B] (chunk stride 8 KB, group 1 KB).
 template <bool A_MN, bool B_MN, int STAGES, class Epi, bool MN4 = false>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupArgs<typename Epi::Params> g)
 {
     using S = PairSmem<STAGES>;
@@ -215,7 +219,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(tfull_bar(b), 1);
-            ptx::mbar_init(tempty_bar(b), 8);  // 4 epilogue warps in each CTA of the pair
+            ptx::mbar_init(tempty_bar(b), 16);  // 8 epilogue warps in each CTA of the pair
         }
         ptx::mbar_init(mma_done, 1);
         ptx::fence_barrier_init();
@@ -335,6 +339,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
     } else {
         // ---------------- epilogue (both CTAs): own 128 accumulator rows
         const int quarter = warp % 4;
+        const int half = (warp - 2) / 4;  // two warps per TMEM lane quarter split the columns
         const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
         const uint32_t leader_tempty1 = map_to_rank(tempty_bar(1), 0);
         int j = 0;
@@ -350,7 +355,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             ptx::tc_fence_after();
-            Epi::run_dyn(P.ep, tmem + b * kAccCols, P.bn, quarter, lane, tr.m0, tr.n0, P.M, P.N, tr.z);
+            Epi::run_dyn(P.ep, tmem + b * kAccCols, P.bn, quarter, lane, tr.m0, tr.n0, P.M, P.N, tr.z, 32 * half, 64);
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(b ? leader_tempty1 : leader_tempty0);
