@@ -201,7 +201,9 @@ WorkLayout work_layout(const noble_linear_desc *d)
         L.wupt = take((size_t)r * d->d_out * 2);
         L.mb = take(2 * (size_t)r * r * 2);
         L.ones = take((size_t)T * kOnesCols * 2);
-        L.n_cos_blocks = r ? ceil_div(T, 128) : 0;
+        // one partial per CTA of the CosNet kernel, whose grid is a whole number
+        // of CTA pairs (a padding CTA contributes exact zeros)
+        L.n_cos_blocks = r ? 2 * ceil_div(ceil_div(T, 128), 2) : 0;
         L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
         L.split = wgrad_split(d);
         if (L.split > 1) {
@@ -792,7 +794,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     using Cfg = tc::CosnetCfg<R>;
     CUtensorMap mA, mB, mM;
     NOBLE_TRY(make_map(&mA, A, T, K, tc::kBM));
-    NOBLE_TRY(make_map(&mB, B, R, K, R));
+    NOBLE_TRY(make_map(&mB, B, R, K, R / 2));  // each CTA of a pair loads half of the rows
     NOBLE_TRY(make_map(&mM, Mx, 2 * R, R, R));  // [2][R][R]: high then low part
     tc::CosnetArgs args = args_in;
     args.T = T;
@@ -803,7 +805,10 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
     const KernelInfo ki{name, kBoundHbm, 2.0 * T * R * (K + R), 2.0 * T * K + 2.0 * R * K + (BWD ? 14.0 : 10.0) * T * R};
     return run(st, ki, [&] {
-        kern<<<(unsigned)ceil_div(T, tc::kBM), tc::kCosnetThreads, Cfg::kDynamic, st>>>(mA, mB, mM, args);
+        // clusters of two tiles; an odd tile count gets one tile past the end,
+        // whose rows are all out of range (zero-filled, never stored)
+        const unsigned grid = (unsigned)(2 * ceil_div(ceil_div(T, tc::kBM), 2));
+        kern<<<grid, tc::kCosnetThreads, Cfg::kDynamic, st>>>(mA, mB, mM, args);
     });
 }
 

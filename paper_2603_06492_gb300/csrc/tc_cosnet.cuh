@@ -143,8 +143,40 @@ __device__ __forceinline__ uint4 store_hi_lo_impl(uint8_t *tile, int row, int co
 // TMEM lane quarter, taking alternate 32-column chunks of their 32 rows.
 constexpr int kCosnetThreads = 320;
 
+// Cluster of two CTAs (consecutive 128-token tiles).  The r-row B operand
+// of the main loop is the same for both, so each CTA loads half of every B
+// stage and multicasts it to both: a stage is refilled only once the MMAs of
+// both CTAs have released it (empty barriers count two arrivals, each CTA's
+// MMA commit arrives on both).
+__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0, int c1,
+                                               uint16_t mask)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster "
+        "[%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "h"(mask)
+        : "memory");
+}
+__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t mask)
+{
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::
+                     "r"(bar),
+                 "h"(mask)
+                 : "memory");
+}
+__device__ __forceinline__ void cluster_sync_all()
+{
+    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ uint32_t cta_rank_in_cluster()
+{
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
 template <int R, bool BWD>
-__global__ void __launch_bounds__(kCosnetThreads, 1)
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kCosnetThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const __grid_constant__ CUtensorMap mM, const CosnetArgs args)
 {
@@ -176,7 +208,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ptx::tma_prefetch_desc(&mB);
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(full_bar(s), 1);
-            ptx::mbar_init(empty_bar(s), 1);
+            ptx::mbar_init(empty_bar(s), 2);  // released by the MMAs of both CTAs
         }
         ptx::mbar_init(tmem_full, 1);
         ptx::mbar_init(m_full, 1);
@@ -196,8 +228,10 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
     }
     ptx::tc_fence_before();
     __syncthreads();
+    cluster_sync_all();  // both CTAs' barriers exist before any multicast
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    const uint32_t rank = cta_rank_in_cluster();
 
     if (warp == 0) {
         if (lane == 0) {
@@ -210,7 +244,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 ptx::mbar_arrive_expect_tx(fb, C::kStage);
                 const uint32_t sA = sbase + s * C::kStage;
                 ptx::tma_load_2d(sA, &mA, fb, i * kBK, (int)m0);
-                ptx::tma_load_2d(sA + C::kA, &mB, fb, i * kBK, 0);
+                // this CTA's half of the B rows, to the same offset in both CTAs
+                tma_load_2d_mc(sA + C::kA + rank * (R / 2) * 128, &mB, fb, i * kBK, (int)rank * (R / 2), 0x3);
                 ++issued;
             }
             for (int i = issued > STAGES ? issued - STAGES : 0; i < issued; ++i)
@@ -245,7 +280,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 for (int kk = 0; kk < kBK / 16; ++kk)
                     ptx::mma_bf16(tmem, ptx::smem_desc_sw128(sA + kk * 32, 16, 1024),
                                   ptx::smem_desc_sw128(sB + kk * 32, 16, 1024), idesc, (i > 0 || kk > 0) ? 1u : 0u);
-                ptx::mma_commit(empty_bar(s));
+                mma_commit_mc(empty_bar(s), 0x3);
             }
             ptx::mma_commit(tmem_full);
             ptx::mbar_wait(tmem_full, 0, nullptr);
@@ -472,6 +507,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 
     ptx::tc_fence_before();
     __syncthreads();
+    cluster_sync_all();  // no CTA leaves while its peer may still signal it
     if (warp == 1) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, C::kTmemCols);
