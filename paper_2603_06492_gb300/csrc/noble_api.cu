@@ -490,9 +490,7 @@ struct ProbSpec {
     int bn;           // N tile (multiple of 32; of 64 when B is MN-major)
     int nsplit = 1;
     int kb_per_split = 0;
-    uint8_t hint[4] = {0, 0, 0, 0};  // L2 policy of A0, B0, A1, B1: 0 none, 1 evict-first, 2 evict-last
 };
-constexpr uint8_t kEvictFirst = 1, kEvictLast = 2;
 
 template <int BN_MAX> struct PStagesFor { static constexpr int value = BN_MAX >= 256 ? 4 : 6; };
 
@@ -653,7 +651,6 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         q.nsplit = P.nsplit;
         q.kb_per_split = P.kb_per_split;
         q.tile_begin = tiles;
-        for (int h = 0; h < 4; ++h) q.hint[h] = P.hint[h];
         q.ep = eps[i];
         tiles += (int)ceil_div(q.tiles_m, 2) * q.tiles_n * q.nsplit;
         const double K = (double)P.s0.K + (P.s1 ? (double)P.s1->K : 0.0);
@@ -834,8 +831,7 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     const TcSeg main{x, W, di};
     const tc::EpiStore<bf16>::Params py{y, dout, bias, 0};
     if (r == 0) {
-        ProbSpec P{T, dout, main, nullptr, 256};
-        P.hint[0] = kEvictFirst, P.hint[1] = kEvictLast;  // activations stream, weights stay
+        const ProbSpec P{T, dout, main, nullptr, 256};
         return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
     }
     const SavedLayout SL = saved_layout(d);
@@ -849,8 +845,7 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
         return cosnet_launch<decltype(bn)::value, false>(st, "tc_down_cosnet_fwd", T, x, di, W_down, mt, a);
     }));
     const TcSeg up{c, W_up, r};
-    ProbSpec P{T, dout, main, &up, 256};
-    P.hint[0] = kEvictFirst, P.hint[1] = kEvictLast, P.hint[2] = kEvictFirst, P.hint[3] = kEvictLast;
+    const ProbSpec P{T, dout, main, &up, 256};
     return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
 }
 
@@ -882,8 +877,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     {
         const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
         const TcSeg sdx2{dh, W_down, r};
-        ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
-        P.hint[0] = kEvictFirst, P.hint[1] = kEvictLast, P.hint[2] = kEvictFirst, P.hint[3] = kEvictLast;
+        const ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
         if (mn4_ok({di}, {dout, r}))
             NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>, true>(st, "tc_dx", 1, &P, &px)));
         else
@@ -900,12 +894,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         wgrad_shapes(d, mn);
         int which[5];
         int n = 0;
-        // Each wave of tiles re-reads the narrower of dy and x and streams the
-        // wider one once: keep the narrow one (and the r-wide operands) in L2.
-        const uint8_t h_dy = dout >= di ? kEvictFirst : kEvictLast;
-        const uint8_t h_x = dout >= di ? kEvictLast : kEvictFirst;
-        auto add = [&](int k, ProbSpec ps, float *out, int64_t ldc, bool col0, uint8_t ha, uint8_t hb) {
-            ps.hint[0] = ha, ps.hint[1] = hb;
+        auto add = [&](int k, ProbSpec ps, float *out, int64_t ldc, bool col0) {
             P[n] = ps;
             E[n] = {out, ldc, nullptr, 0};
             E[n].col0 = col0 ? 1 : 0;
@@ -914,16 +903,13 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         };
         // heaviest tiles first: the round-robin tile walk then fills the
         // CTAs that drew fewer full tiles with the small ones
-        add(0, ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256}, dW, di, false, h_dy, h_x);
+        add(0, ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256}, dW, di, false);
         if (r > 0) {
-            add(1, ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256}, dW_down, di, false, kEvictLast, h_x);
-            add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false, h_dy,
-                kEvictLast);
-            add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false, kEvictLast,
-                kEvictLast);
+            add(1, ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256}, dW_down, di, false);
+            add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false);
+            add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);
         }
-        if (dbias)
-            add(4, ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128}, dbias, 1, true, h_dy, kEvictLast);
+        if (dbias) add(4, ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128}, dbias, 1, true);
         const int split = WL.split;
         SplitJobs J{};
         if (split > 1) {

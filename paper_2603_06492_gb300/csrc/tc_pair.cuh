@@ -54,38 +54,6 @@ __device__ __forceinline__ void mbar_arrive_cluster(uint32_t cluster_addr)
 
 // TMA load into this CTA's shared memory, completing on an mbarrier that may
 // live in the peer CTA of the pair (cluster address).
-// L2 eviction policies for TMA loads (created once per thread that issues them).
-__device__ __forceinline__ uint64_t policy_evict_first()
-{
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-__device__ __forceinline__ uint64_t policy_evict_last()
-{
-    uint64_t p;
-    asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
-    return p;
-}
-__device__ __forceinline__ void tma_load_2d_pair_hint(uint32_t dst, const CUtensorMap *map, uint32_t bar_cluster,
-                                                      int c0, int c1, uint64_t policy)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint "
-        "[%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(c0), "r"(c1), "l"(policy)
-        : "memory");
-}
-__device__ __forceinline__ void tma_load_4d_pair_hint(uint32_t dst, const CUtensorMap *map, uint32_t bar_cluster,
-                                                      int c2, int c3, uint64_t policy)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cta.global.tile.mbarrier::complete_tx::bytes.cta_group::2.L2::cache_hint "
-        "[%0], [%1, {%3, %3, %4, %5}], [%2], %6;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(0), "r"(c2), "r"(c3), "l"(policy)
-        : "memory");
-}
-
 __device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap *map, uint32_t bar_cluster, int c0,
                                                  int c1)
 {
@@ -269,7 +237,6 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
     if (warp == 0) {
         if (lane == 0) {
             // ---------------- producer (both CTAs)
-            const uint64_t pol_first = policy_evict_first(), pol_last = policy_evict_last();
             uint32_t it = 0;
             bool ok = true;
             const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
@@ -295,30 +262,20 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     const CUtensorMap *mB = &maps.m[tr.prob][seg1 ? 3 : 1];
                     const int k = (seg1 ? kb - P.kb0 : kb) * kBK;
                     const int nb = (int)tr.n0 + (int)rank * bh;
-                    const int ha = P.hint[seg1 ? 2 : 0], hb = P.hint[seg1 ? 3 : 1];
-                    const uint64_t pa = ha == 1 ? pol_first : pol_last, pb = hb == 1 ? pol_first : pol_last;
-                    auto ld2 = [&](uint32_t dst, const CUtensorMap *m, int c0, int c1, int h, uint64_t pol) {
-                        if (h) tma_load_2d_pair_hint(dst, m, fb, c0, c1, pol);
-                        else tma_load_2d_pair(dst, m, fb, c0, c1);
-                    };
-                    auto ld4 = [&](uint32_t dst, const CUtensorMap *m, int c2, int c3, int h, uint64_t pol) {
-                        if (h) tma_load_4d_pair_hint(dst, m, fb, c2, c3, pol);
-                        else tma_load_4d_pair(dst, m, fb, c2, c3);
-                    };
                     if (A_MN && MN4) {
-                        ld4(sA, mA, (int)(tr.m0 / 64), k / 8, ha, pa);
+                        tma_load_4d_pair(sA, mA, fb, (int)(tr.m0 / 64), k / 8);
                     } else if (A_MN) {
-                        ld2(sA, mA, (int)tr.m0, k, ha, pa);
-                        ld2(sA + kChunkBytes, mA, (int)tr.m0 + 64, k, ha, pa);
+                        tma_load_2d_pair(sA, mA, fb, (int)tr.m0, k);
+                        tma_load_2d_pair(sA + kChunkBytes, mA, fb, (int)tr.m0 + 64, k);
                     } else {
-                        ld2(sA, mA, k, (int)tr.m0, ha, pa);
+                        tma_load_2d_pair(sA, mA, fb, k, (int)tr.m0);
                     }
                     if (B_MN && MN4) {
-                        ld4(sB, mB, nb / 64, k / 8, hb, pb);
+                        tma_load_4d_pair(sB, mB, fb, nb / 64, k / 8);
                     } else if (B_MN) {
-                        for (int c = 0; c < bh / 64; ++c) ld2(sB + c * kChunkBytes, mB, nb + 64 * c, k, hb, pb);
+                        for (int c = 0; c < bh / 64; ++c) tma_load_2d_pair(sB + c * kChunkBytes, mB, fb, nb + 64 * c, k);
                     } else {
-                        ld2(sB, mB, k, nb, hb, pb);
+                        tma_load_2d_pair(sB, mB, fb, k, nb);
                     }
                 }
             }

@@ -27,7 +27,6 @@ struct Problem {
     int tiles_m, tiles_n;  // output tiles
     int nsplit, kb_per_split;
     int tile_begin;        // first global tile index of this problem
-    uint8_t hint[4];       // L2 policy per operand map (A0, B0, A1, B1): 0 none, 1 evict-first, 2 evict-last
     EpiParams ep;
 };
 
