@@ -200,11 +200,13 @@ WorkLayout work_layout(const noble_linear_desc *d)
         L.db = take(tr * 2);
         L.wupt = take((size_t)r * d->d_out * 2);
         L.mb = take(2 * (size_t)r * r * 2);
-        L.ones = take((size_t)T * kOnesCols * 2);
+        L.ones = r ? 0 : take((size_t)T * kOnesCols * 2);  // dbias = dy^T 1 without a branch
         // one partial per CTA of the CosNet kernel, whose grid is a whole number
         // of CTA pairs (a padding CTA contributes exact zeros)
         L.n_cos_blocks = r ? 2 * ceil_div(ceil_div(T, 128), 2) : 0;
         L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
+        // with a branch, dbias is summed from the dy tiles of the CosNet kernel
+        L.bias_part = take((size_t)L.n_cos_blocks * d->d_out * 4);
         L.split = wgrad_split(d);
         if (L.split > 1) {
             int64_t mn[5][2];
@@ -765,12 +767,12 @@ noble_status prep_bf16(cudaStream_t st, int64_t d_out, int64_t r, const bf16 *W_
     });
 }
 
-// Sum of K-split partials: out_j[i] = sum_z part_j[z][i] (z ascending) for
-// up to five outputs in one launch.
+// Fixed-order sums of partial results: out_j[i] = sum_z part_j[z * stride_j + i]
+// (z ascending) for up to five outputs in one launch.
 struct SplitJobs {
     const float *part[5];
     float *out[5];
-    int64_t n[5], begin[6];
+    int64_t n[5], stride[5], begin[6];  // stride: elements between consecutive partials
     int nparts;
     int njobs;
 };
@@ -782,7 +784,7 @@ __global__ void reduce_split_kernel(SplitJobs J)
     while (idx >= J.begin[j + 1]) ++j;
     const int64_t i = idx - J.begin[j];
     float s = 0.f;
-    for (int z = 0; z < J.nparts; ++z) s += J.part[j][(int64_t)z * J.n[j] + i];
+    for (int z = 0; z < J.nparts; ++z) s += J.part[j][(int64_t)z * J.stride[j] + i];
     J.out[j][i] = s;
 }
 
@@ -860,18 +862,45 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     const WorkLayout WL = work_layout(d);
     bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
     bf16 *wupt = (bf16 *)(ws + WL.wupt), *mb = (bf16 *)(ws + WL.mb), *ones = (bf16 *)(ws + WL.ones);
+    const bool ones_dbias = dbias && r == 0;
     NOBLE_TRY(prep_bf16(st, dout, r, r ? W_up : nullptr, r ? wupt : nullptr, M, nullptr, r ? mb : nullptr,
-                        dbias ? T * kOnesCols : 0, dbias ? ones : nullptr));
+                        ones_dbias ? T * kOnesCols : 0, ones_dbias ? ones : nullptr));
     if (r > 0) {
         float *cpart = (float *)(ws + WL.cos_part);
         tc::CosnetArgs ca{};
         ca.om1 = om1, ca.ph1 = ph1, ca.om2 = om2, ca.ph2 = ph2;
         ca.h_in = (const float *)(saved + SL.h), ca.b_in = (const float *)(saved + SL.b);
         ca.dh_out = dh, ca.a_out = a, ca.db_out = db, ca.part = cpart;
+        float *bpart = (float *)(ws + WL.bias_part);
+        ca.bias_part = dbias ? bpart : nullptr;
+        ca.kdim = dout;
         NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
             return cosnet_launch<decltype(bn)::value, true>(st, "tc_dc_cosnet_bwd", T, dy, dout, wupt, mb, ca);
         }));
-        NOBLE_TRY(reduce(st, WL.n_cos_blocks, 4 * r, r, cpart, dom1, dph1, dom2, dph2));
+        // domega1, dphi1, domega2, dphi2 (and dbias) from the per-CTA partials
+        SplitJobs J{};
+        float *outs[4] = {dom1, dph1, dom2, dph2};
+        J.nparts = (int)WL.n_cos_blocks;
+        J.begin[0] = 0;
+        for (int q = 0; q < 4; ++q) {
+            J.part[q] = cpart + q * r;
+            J.out[q] = outs[q];
+            J.n[q] = r;
+            J.stride[q] = 4 * r;
+            J.begin[q + 1] = J.begin[q] + r;
+        }
+        J.njobs = 4;
+        if (dbias) {
+            J.part[4] = bpart;
+            J.out[4] = dbias;
+            J.n[4] = dout;
+            J.stride[4] = dout;
+            J.begin[5] = J.begin[4] + dout;
+            J.njobs = 5;
+        }
+        const int64_t total = J.begin[J.njobs];
+        const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
+        NOBLE_TRY(run(st, kr, [&] { reduce_split_kernel<<<(unsigned)ceil_div(total, 256), 256, 0, st>>>(J); }));
     }
     // dx = [dy | dh] [W ; W_down]
     {
@@ -909,7 +938,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false);
             add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);
         }
-        if (dbias) add(4, ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128}, dbias, 1, true);
+        if (ones_dbias) add(4, ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128}, dbias, 1, true);
         const int split = WL.split;
         SplitJobs J{};
         if (split > 1) {
@@ -927,6 +956,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
                 J.part[i] = part;
                 J.out[i] = final_out[i];
                 J.n[i] = mn[k][0] * mn[k][1];
+                J.stride[i] = J.n[i];
                 J.begin[i + 1] = J.begin[i] + J.n[i];
             }
             J.njobs = n;

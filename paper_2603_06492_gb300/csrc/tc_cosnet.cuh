@@ -42,6 +42,10 @@ struct CosnetArgs {
     const float *h_in, *b_in;
     __nv_bfloat16 *dh_out, *a_out, *db_out;
     float *part;         // [gridDim.x][4][r]
+    // backward, optional: column sums of dy over this CTA's tokens,
+    // [gridDim.x][kdim], accumulated from the dy tiles of the main loop
+    float *bias_part;
+    int64_t kdim;
     uint32_t *status;
 };
 
@@ -56,7 +60,7 @@ struct CosnetCfg {
     static constexpr int kKSteps = R < 64 ? R / 16 : 4;   // MMA K-steps per k-block
     static constexpr uint32_t kMkbBytes = 2 * R * 128;    // one k-block of M_hi and M_lo
     static constexpr uint32_t kTileBytes = kMkb * kBM * 128;  // epilogue row-operand tile, bf16
-    static constexpr uint32_t kExtra = 4 * R * 4 + 4 * 4 * R * 4 + 256;  // params, column sums, barriers
+    static constexpr uint32_t kExtra = 4 * R * 4 + 4 * 4 * R * 4 + 2048 + 256;  // params, column sums, barriers
     static constexpr uint32_t kFit = (227u * 1024u - 1024u - kExtra) / kStage;
     static constexpr int kStages = kFit > 8 ? 8 : (int)kFit;
     static_assert(kStages >= 2, "pipeline depth");
@@ -70,7 +74,8 @@ struct CosnetCfg {
     static constexpr uint32_t kMOff = 2 * kTileBytes;  // 1024-aligned
     static constexpr uint32_t kParamOff = kRing;        // omega/phi copies, 4 x R floats
     static constexpr uint32_t kPartOff = kParamOff + 4 * R * 4;  // [4 warps][4][R] floats
-    static constexpr uint32_t kBarOff = kPartOff + 4 * 4 * R * 4;
+    static constexpr uint32_t kBiasRedOff = kPartOff + 4 * 4 * R * 4;  // [8 warps][64] floats
+    static constexpr uint32_t kBarOff = kBiasRedOff + 8 * 64 * 4;
     static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 4) + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
@@ -208,7 +213,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ptx::tma_prefetch_desc(&mB);
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(full_bar(s), 1);
-            ptx::mbar_init(empty_bar(s), 2);  // released by the MMAs of both CTAs
+            // released by the MMAs of both CTAs and, when dbias is summed from the
+            // dy stages, by this CTA's eight epilogue warps
+            ptx::mbar_init(empty_bar(s), (BWD && args.bias_part) ? 10 : 2);
         }
         ptx::mbar_init(tmem_full, 1);
         ptx::mbar_init(m_full, 1);
@@ -297,8 +304,54 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         const uint32_t acc2 = lane_addr + C::kRCols;
         const float *om1 = prm, *ph1 = prm + R, *om2 = prm + 2 * R, *ph2 = prm + 3 * R;
         uint8_t *tile = smem;  // the ring is free once the main accumulator is complete
-        bool ok = ptx::mbar_wait(tmem_full, 0, args.status);
-        ok = __all_sync(0xffffffffu, ok);
+        bool bias_ok = true;
+        if constexpr (BWD) {
+            if (args.bias_part) {
+                // dbias partials while the main loop runs: warp ew sums rows
+                // [16 ew, 16 ew + 16) of each dy stage for columns 2 lane, 2 lane + 1
+                // (rows ascending), then the eight warps' sums are added in order.
+                const int ew = warp - 2;
+                float *red = reinterpret_cast<float *>(smem + C::kBiasRedOff);
+                for (int i = 0; i < args.kb; ++i) {
+                    const int s = i % STAGES;
+                    const uint32_t ph = (i / STAGES) & 1;
+                    bool w = bias_ok && ptx::mbar_wait(full_bar(s), ph, args.status);
+                    w = __all_sync(0xffffffffu, w);
+                    float s0 = 0.f, s1 = 0.f;
+                    if (w) {
+                        const uint8_t *sA = smem + s * C::kStage;
+#pragma unroll
+                        for (int rr = 0; rr < 16; ++rr) {
+                            const int rw = ew * 16 + rr;
+                            const uint32_t off =
+                                rw * 128 + ((((uint32_t)lane >> 2) ^ (rw & 7)) << 4) + ((lane & 3) << 2);
+                            const float2 f =
+                                __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(sA + off));
+                            s0 += f.x;
+                            s1 += f.y;
+                        }
+                        __syncwarp();
+                        if (lane == 0) ptx::mbar_arrive(empty_bar(s));
+                    }
+                    red[ew * 64 + 2 * lane] = s0;
+                    red[ew * 64 + 2 * lane + 1] = s1;
+                    // every epilogue warp reaches this barrier once per k-block,
+                    // whatever its waits returned
+                    bias_ok = ptx::named_barrier_and(2, 256, w);
+                    if (bias_ok && ew < 2) {
+                        const int cl = ew * 32 + lane;
+                        float sum = 0.f;
+#pragma unroll
+                        for (int w8 = 0; w8 < 8; ++w8) sum += red[w8 * 64 + cl];
+                        const int64_t col = (int64_t)i * 64 + cl;
+                        if (col < args.kdim) args.bias_part[(int64_t)blockIdx.x * args.kdim + col] = sum;
+                    }
+                    ptx::named_barrier_sync(2, 256);
+                }
+            }
+        }
+        bool ok = bias_ok && ptx::mbar_wait(tmem_full, 0, args.status);
+        ok = ptx::named_barrier_and(3, 256, ok);  // uniform over the epilogue warps
         if (ok) {
             ptx::tc_fence_after();
             // ---- phase 1: first accumulator -> bf16 operand tile (+ outputs)
@@ -403,7 +456,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 ptx::mma_commit(mma2_done);
             }
             ok = ptx::mbar_wait(mma2_done, 0, args.status);
-            ok = __all_sync(0xffffffffu, ok);
+            ok = ptx::named_barrier_and(3, 256, ok);
         }
         if (ok) {
             ptx::tc_fence_after();
