@@ -258,8 +258,14 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             for (int i = issued > STAGES ? issued - STAGES : 0; i < issued; ++i)
                 ptx::mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1, nullptr);
             // mixing matrix (rows [0, r) = hi, [r, 2r) = lo) into the ring once
-            // every main-loop MMA is done, kChunkKb k-blocks per pass
-            if (issued == args.kb && ptx::mbar_wait(tmem_full, 0, args.status)) {
+            // every main-loop MMA is done and every stage has been released
+            // (in the backward also by the epilogue warps that sum dy for
+            // dbias, which may still be reading the last stages), kChunkKb
+            // k-blocks per pass
+            bool released = issued == args.kb;
+            for (int i = issued > STAGES ? issued - STAGES : 0; released && i < issued; ++i)
+                released = ptx::mbar_wait(empty_bar(i % STAGES), (i / STAGES) & 1, args.status);
+            if (released && ptx::mbar_wait(tmem_full, 0, args.status)) {
                 for (int pass = 0; pass < C::kPasses; ++pass) {
                     if (pass > 0 && !ptx::mbar_wait(m_empty, (pass - 1) & 1, args.status)) break;
                     const uint32_t mf = m_full;
