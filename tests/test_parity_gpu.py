@@ -169,3 +169,24 @@ def test_launch_counter_advances():
     n0 = binding.noble_kernel_launch_count()
     run_gpu(layer, inp)
     assert binding.noble_kernel_launch_count() > n0
+
+
+@pytest.mark.parametrize("d_out,r", [(768, 256), (2304, 16), (6144, 128), (1024, 64)])
+def test_dbias_from_cosnet_kernel(d_out, r):
+    """dbias is summed from the dy tiles streamed by the CosNet backward
+    kernel; check it against an fp64 column sum on shapes with many k-blocks
+    per tile, three times in a row (the sums race with the ring reuse that
+    follows the main loop if its ordering is wrong)."""
+    import torch
+    layer = Layer("dbias", 4096, 256, d_out, r, "bf16")
+    inp = make_layer_inputs(layer, 31)
+    ref = inp["dy"].sum(axis=0)
+    dev = binding.params_to_device(inp, "bf16")
+    buf = binding.NobleLinearBuffers(4096, 256, d_out, r, "bf16")
+    binding.forward(buf, dev["x"], dev)
+    for _ in range(3):
+        buf.grads["dbias"].fill_(float("nan"))
+        binding.backward(buf, dev["x"], dev["dy"], dev)
+        torch.cuda.synchronize()
+        got = buf.grads["dbias"].cpu().numpy().astype(np.float64)
+        assert rel_err(got, ref) < 1e-5, rel_err(got, ref)
