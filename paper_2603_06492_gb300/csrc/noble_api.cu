@@ -125,11 +125,9 @@ size_t esize(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 ? 2 : 4
 // True when the bf16 tensor-core path runs (the default for bf16 operands).
 bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->flags & kFlagSimtOnly); }
 
-// Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r],
-// then (tensor-core path) the mixing matrix transposed, Mt[j][i] = M[i][j],
-// as bf16 high and low parts [2][r][r].
+// Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r].
 struct SavedLayout {
-    size_t h, b, c, mt, total;
+    size_t h, b, c, total;
 };
 SavedLayout saved_layout(const noble_linear_desc *d)
 {
@@ -139,8 +137,7 @@ SavedLayout saved_layout(const noble_linear_desc *d)
     L.h = 0;
     L.b = align_up(L.h + tr * 4, 256);
     L.c = align_up(L.b + tr * 4, 256);
-    L.mt = align_up(L.c + tr * esize(d), 256);
-    L.total = align_up(L.mt + (use_tc(d) ? 2 * (size_t)d->r * d->r * 2 : 0), 256);
+    L.total = align_up(L.c + tr * esize(d), 256);
     return L;
 }
 
@@ -180,10 +177,10 @@ void wgrad_shapes(const noble_linear_desc *d, int64_t (&mn)[5][2])
 //   CUDA-core path: dh (dtype), dc, a, db (fp32) [T][r]; M^T fp32; per-block
 //     partials of the CosNet sums, of dM and of dbias.
 //   tensor-core path: dh, a, db (bf16) [T][r]; W_up^T (bf16 [r][d_out]);
-//     M as bf16 high and low parts [2][r][r]; an all-ones [T][8] bf16
-//     operand; per-tile CosNet partials.
+//     per-CTA CosNet and dbias partials; without a branch an all-ones
+//     [T][64] bf16 operand (dbias = dy^T 1).
 struct WorkLayout {
-    size_t dh, dc, a, db, mt, wupt, mb, ones, cos_part, dm_part, bias_part, wsplit[5], total;
+    size_t dh, dc, a, db, mt, wupt, ones, cos_part, dm_part, bias_part, wsplit[5], total;
     int split;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
 };
@@ -199,7 +196,6 @@ WorkLayout work_layout(const noble_linear_desc *d)
         L.a = take(tr * 2);
         L.db = take(tr * 2);
         L.wupt = take((size_t)r * d->d_out * 2);
-        L.mb = take(2 * (size_t)r * r * 2);
         L.ones = r ? 0 : take((size_t)T * kOnesCols * 2);  // dbias = dy^T 1 without a branch
         // one partial per CTA of the CosNet kernel, whose grid is a whole number
         // of CTA pairs (a padding CTA contributes exact zeros)
@@ -710,13 +706,12 @@ noble_status with_rank_tile(int64_t r, F &&f)
     return fail(NOBLE_ERR_UNSUPPORTED, "rank %lld", (long long)r);
 }
 
-// Preparation of the small bf16 operands of the tensor-core path, in one
-// launch: blocks [0, nt) transpose W_up [d_out][r] into wupt [r][d_out] in
-// 32 x 32 tiles; the following blocks split M (fp32) into bf16 high and low
-// parts, transposed (mt, forward) and/or as is (mb, backward); the rest fill
-// the all-ones [T][kOnesCols] operand.
-__global__ void prep_bf16_kernel(int64_t d_out, int r, const bf16 *W_up, bf16 *wupt, int nt, const float *M,
-                                 bf16 *mt, bf16 *mb, int nm, int64_t ones_n, bf16 *ones)
+// Preparation of the small bf16 operands of the backward tensor-core path,
+// in one launch: blocks [0, nt) transpose W_up [d_out][r] into wupt
+// [r][d_out] in 32 x 32 tiles; the rest fill the all-ones [T][kOnesCols]
+// operand.
+__global__ void prep_bf16_kernel(int64_t d_out, int r, const bf16 *W_up, bf16 *wupt, int nt, int64_t ones_n,
+                                 bf16 *ones)
 {
     __shared__ bf16 tile[32][33];
     const int b = blockIdx.x;
@@ -734,36 +729,19 @@ __global__ void prep_bf16_kernel(int64_t d_out, int r, const bf16 *W_up, bf16 *w
         }
         return;
     }
-    if (b < nt + nm) {
-        const int64_t idx = (int64_t)(b - nt) * blockDim.x + threadIdx.x;
-        if (idx < (int64_t)r * r) {
-            // high and low bf16 parts, stored as [2][r][r] (rows [0,r) hi, [r,2r) lo)
-            const int i = (int)(idx / r), j = (int)(idx % r);
-            const float m = M[idx];
-            const bf16 hi = __float2bfloat16_rn(m);
-            const bf16 lo = __float2bfloat16_rn(m - __bfloat162float(hi));
-            const int64_t rr = (int64_t)r * r;
-            if (mb) mb[idx] = hi, mb[rr + idx] = lo;
-            if (mt) mt[(int64_t)j * r + i] = hi, mt[rr + (int64_t)j * r + i] = lo;
-        }
-        return;
-    }
-    const int64_t idx = (int64_t)(b - nt - nm) * blockDim.x + threadIdx.x;
+    const int64_t idx = (int64_t)(b - nt) * blockDim.x + threadIdx.x;
     if (idx < ones_n) ones[idx] = __float2bfloat16_rn(1.f);
 }
 
-noble_status prep_bf16(cudaStream_t st, int64_t d_out, int64_t r, const bf16 *W_up, bf16 *wupt, const float *M,
-                       bf16 *mt, bf16 *mb, int64_t ones_n, bf16 *ones)
+noble_status prep_bf16(cudaStream_t st, int64_t d_out, int64_t r, const bf16 *W_up, bf16 *wupt, int64_t ones_n,
+                       bf16 *ones)
 {
     const int nt = wupt ? (int)(ceil_div(d_out, 32) * ceil_div(r, 32)) : 0;
-    const int nm = (mt || mb) ? (int)ceil_div(r * r, 256) : 0;
     const int no = ones ? (int)ceil_div(ones_n, 256) : 0;
-    if (nt + nm + no == 0) return NOBLE_OK;
-    const KernelInfo ki{"prep_bf16", kBoundHbm, 0.0,
-                        4.0 * (wupt ? d_out * r : 0) + 6.0 * (nm ? r * r : 0) + 2.0 * (ones ? ones_n : 0)};
+    if (nt + no == 0) return NOBLE_OK;
+    const KernelInfo ki{"prep_bf16", kBoundHbm, 0.0, 4.0 * (wupt ? d_out * r : 0) + 2.0 * (ones ? ones_n : 0)};
     return run(st, ki, [&] {
-        prep_bf16_kernel<<<nt + nm + no, 256, 0, st>>>(d_out, (int)r, W_up, wupt, nt, M, mt, mb, nm,
-                                                       ones ? ones_n : 0, ones);
+        prep_bf16_kernel<<<nt + no, 256, 0, st>>>(d_out, (int)r, W_up, wupt, nt, ones ? ones_n : 0, ones);
     });
 }
 
@@ -776,28 +754,43 @@ struct SplitJobs {
     int nparts;
     int njobs;
 };
-__global__ void reduce_split_kernel(SplitJobs J)
+// Block = 8 warps over 32 consecutive outputs: warp w adds partials
+// [w P/8, (w+1) P/8) in ascending order for its lane's output, then the eight
+// warp sums are added in warp order -- deterministic.
+__global__ void __launch_bounds__(256) reduce_split_kernel(SplitJobs J)
 {
-    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= J.begin[J.njobs]) return;
+    __shared__ float sm[8][33];
+    const int lane = threadIdx.x % 32, w = threadIdx.x / 32;
+    const int64_t idx = (int64_t)blockIdx.x * 32 + lane;
+    const bool in = idx < J.begin[J.njobs];
     int j = 0;
-    while (idx >= J.begin[j + 1]) ++j;
-    const int64_t i = idx - J.begin[j];
+    if (in)
+        while (idx >= J.begin[j + 1]) ++j;
+    const int64_t i = in ? idx - J.begin[j] : 0;
+    const int per = (J.nparts + 7) / 8;
+    const int zb = w * per, ze = min(J.nparts, zb + per);
     float s = 0.f;
-    for (int z = 0; z < J.nparts; ++z) s += J.part[j][(int64_t)z * J.stride[j] + i];
-    J.out[j][i] = s;
+    if (in)
+        for (int z = zb; z < ze; ++z) s += J.part[j][(int64_t)z * J.stride[j] + i];
+    sm[w][lane] = s;
+    __syncthreads();
+    if (w == 0 && in) {
+        float t = 0.f;
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t += sm[k][lane];
+        J.out[j][i] = t;
+    }
 }
 
 // Fused r-wide GEMM + CosNet launch (forward or backward), one tile per CTA.
 template <int R, bool BWD>
 noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const bf16 *A, int64_t K, const bf16 *B,
-                           const bf16 *Mx, const tc::CosnetArgs &args_in)
+                           const tc::CosnetArgs &args_in)
 {
     using Cfg = tc::CosnetCfg<R>;
-    CUtensorMap mA, mB, mM;
+    CUtensorMap mA, mB;
     NOBLE_TRY(make_map(&mA, A, T, K, tc::kBM));
     NOBLE_TRY(make_map(&mB, B, R, K, R / 2));  // each CTA of a pair loads half of the rows
-    NOBLE_TRY(make_map(&mM, Mx, 2 * R, R, R));  // [2][R][R]: high then low part
     tc::CosnetArgs args = args_in;
     args.T = T;
     args.kb = (int)ceil_div(K, tc::kBK);
@@ -810,7 +803,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
         // clusters of two tiles; an odd tile count gets one tile past the end,
         // whose rows are all out of range (zero-filled, never stored)
         const unsigned grid = (unsigned)(2 * ceil_div(ceil_div(T, tc::kBM), 2));
-        kern<<<grid, tc::kCosnetThreads, Cfg::kDynamic, st>>>(mA, mB, mM, args);
+        kern<<<grid, tc::kCosnetThreads, Cfg::kDynamic, st>>>(mA, mB, args);
     });
 }
 
@@ -838,13 +831,12 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     }
     const SavedLayout SL = saved_layout(d);
     float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
-    bf16 *c = (bf16 *)(saved + SL.c), *mt = (bf16 *)(saved + SL.mt);
-    NOBLE_TRY(prep_bf16(st, dout, r, nullptr, nullptr, M, mt, nullptr, 0, nullptr));
+    bf16 *c = (bf16 *)(saved + SL.c);
     tc::CosnetArgs a{};
-    a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2;
+    a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2, a.M = M;
     a.h_out = h, a.b_out = b, a.c_out = c;
     NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-        return cosnet_launch<decltype(bn)::value, false>(st, "tc_down_cosnet_fwd", T, x, di, W_down, mt, a);
+        return cosnet_launch<decltype(bn)::value, false>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
     }));
     const TcSeg up{c, W_up, r};
     const ProbSpec P{T, dout, main, &up, 256};
@@ -861,21 +853,21 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     const SavedLayout SL = saved_layout(d);
     const WorkLayout WL = work_layout(d);
     bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
-    bf16 *wupt = (bf16 *)(ws + WL.wupt), *mb = (bf16 *)(ws + WL.mb), *ones = (bf16 *)(ws + WL.ones);
+    bf16 *wupt = (bf16 *)(ws + WL.wupt), *ones = (bf16 *)(ws + WL.ones);
     const bool ones_dbias = dbias && r == 0;
-    NOBLE_TRY(prep_bf16(st, dout, r, r ? W_up : nullptr, r ? wupt : nullptr, M, nullptr, r ? mb : nullptr,
-                        ones_dbias ? T * kOnesCols : 0, ones_dbias ? ones : nullptr));
+    NOBLE_TRY(prep_bf16(st, dout, r, r ? W_up : nullptr, r ? wupt : nullptr, ones_dbias ? T * kOnesCols : 0,
+                        ones_dbias ? ones : nullptr));
     if (r > 0) {
         float *cpart = (float *)(ws + WL.cos_part);
         tc::CosnetArgs ca{};
-        ca.om1 = om1, ca.ph1 = ph1, ca.om2 = om2, ca.ph2 = ph2;
+        ca.om1 = om1, ca.ph1 = ph1, ca.om2 = om2, ca.ph2 = ph2, ca.M = M;
         ca.h_in = (const float *)(saved + SL.h), ca.b_in = (const float *)(saved + SL.b);
         ca.dh_out = dh, ca.a_out = a, ca.db_out = db, ca.part = cpart;
         float *bpart = (float *)(ws + WL.bias_part);
         ca.bias_part = dbias ? bpart : nullptr;
         ca.kdim = dout;
         NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-            return cosnet_launch<decltype(bn)::value, true>(st, "tc_dc_cosnet_bwd", T, dy, dout, wupt, mb, ca);
+            return cosnet_launch<decltype(bn)::value, true>(st, "tc_dc_cosnet_bwd", T, dy, dout, wupt, ca);
         }));
         // domega1, dphi1, domega2, dphi2 (and dbias) from the per-CTA partials
         SplitJobs J{};
@@ -900,7 +892,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         }
         const int64_t total = J.begin[J.njobs];
         const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
-        NOBLE_TRY(run(st, kr, [&] { reduce_split_kernel<<<(unsigned)ceil_div(total, 256), 256, 0, st>>>(J); }));
+        NOBLE_TRY(run(st, kr, [&] { reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J); }));
     }
     // dx = [dy | dh] [W ; W_down]
     {
@@ -970,7 +962,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             const KernelInfo kr{"reduce_wgrad_split", kBoundHbm, (double)total * J.nparts,
                                 4.0 * total * (J.nparts + 1)};
             NOBLE_TRY(run(st, kr, [&] {
-                reduce_split_kernel<<<(unsigned)ceil_div(total, 256), 256, 0, st>>>(J);
+                reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J);
             }));
         }
     }

@@ -14,9 +14,10 @@
 //             part[cta][0] = sum du1*h, [1] = sum du1, [2] = sum du2*b, [3] = sum du2
 //   (each [r]), reduced over the 128 tokens of the tile in a fixed order.
 //
-// The mixing matrix enters as a bf16 K-major operand loaded by TMA once the
-// main loop is done: Mt[j][i] = M[i][j] for the forward (b_j = sum_i a_i
-// M[i][j]) and M itself for the backward (da_i = sum_j db_j M[i][j]).  Both
+// The mixing matrix enters as a bf16 K-major operand that the epilogue
+// threads build in shared memory from the fp32 M once the main loop is done:
+// Mt[j][i] = M[i][j] for the forward (b_j = sum_i a_i M[i][j]) and M itself
+// for the backward (da_i = sum_j db_j M[i][j]).  Both
 // the row operand (a or db) and the matrix are split into bf16 high and low
 // parts, x = x_hi + x_lo, and the product is formed as
 //     x_hi M_hi + x_lo M_hi + x_hi M_lo
@@ -35,6 +36,7 @@ struct CosnetArgs {
     int64_t T;
     int kb;              // k-blocks of the main operand (d_in or d_out)
     const float *om1, *ph1, *om2, *ph2;
+    const float *M;      // mixing matrix, fp32 [r][r] (b_j = sum_i a_i M[i][j])
     // forward outputs
     float *h_out, *b_out;
     __nv_bfloat16 *c_out;
@@ -76,7 +78,7 @@ struct CosnetCfg {
     static constexpr uint32_t kPartOff = kParamOff + 4 * R * 4;  // [4 warps][4][R] floats
     static constexpr uint32_t kBiasRedOff = kPartOff + 4 * 4 * R * 4;  // [8 warps][64] floats
     static constexpr uint32_t kBarOff = kBiasRedOff + 8 * 64 * 4;
-    static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 4) + 16;
+    static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 3) + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
 
@@ -183,7 +185,7 @@ __device__ __forceinline__ uint32_t cta_rank_in_cluster()
 template <int R, bool BWD>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kCosnetThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-                   const __grid_constant__ CUtensorMap mM, const CosnetArgs args)
+                   const CosnetArgs args)
 {
     using C = CosnetCfg<R>;
     constexpr int STAGES = C::kStages;
@@ -198,10 +200,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
     auto full_bar = [&](int s) { return bar0 + 8u * s; };
     auto empty_bar = [&](int s) { return bar0 + 8u * (STAGES + s); };
     const uint32_t tmem_full = bar0 + 8u * (2 * STAGES);
-    const uint32_t m_full = bar0 + 8u * (2 * STAGES + 1);
-    const uint32_t mma2_done = bar0 + 8u * (2 * STAGES + 2);
-    const uint32_t m_empty = bar0 + 8u * (2 * STAGES + 3);
-    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kBarOff + 8 * (2 * STAGES + 4));
+    const uint32_t mma2_done = bar0 + 8u * (2 * STAGES + 1);
+    const uint32_t m_empty = bar0 + 8u * (2 * STAGES + 2);
+    uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + C::kBarOff + 8 * (2 * STAGES + 3));
     float *prm = reinterpret_cast<float *>(smem + C::kParamOff);  // om1 | ph1 | om2 | ph2
     float *cpart = reinterpret_cast<float *>(smem + C::kPartOff);  // [4][4][R]
 
@@ -218,7 +219,6 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             ptx::mbar_init(empty_bar(s), (BWD && args.bias_part) ? 10 : 2);
         }
         ptx::mbar_init(tmem_full, 1);
-        ptx::mbar_init(m_full, 1);
         ptx::mbar_init(mma2_done, 1);
         ptx::mbar_init(m_empty, 1);
         ptx::fence_barrier_init();
@@ -257,28 +257,6 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
             for (int i = issued > STAGES ? issued - STAGES : 0; i < issued; ++i)
                 ptx::mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1, nullptr);
-            // mixing matrix (rows [0, r) = hi, [r, 2r) = lo) into the ring once
-            // every main-loop MMA is done and every stage has been released
-            // (in the backward also by the epilogue warps that sum dy for
-            // dbias, which may still be reading the last stages), kChunkKb
-            // k-blocks per pass
-            bool released = issued == args.kb;
-            for (int i = issued > STAGES ? issued - STAGES : 0; released && i < issued; ++i)
-                released = ptx::mbar_wait(empty_bar(i % STAGES), (i / STAGES) & 1, args.status);
-            if (released && ptx::mbar_wait(tmem_full, 0, args.status)) {
-                for (int pass = 0; pass < C::kPasses; ++pass) {
-                    if (pass > 0 && !ptx::mbar_wait(m_empty, (pass - 1) & 1, args.status)) break;
-                    const uint32_t mf = m_full;
-                    ptx::mbar_arrive_expect_tx(mf, C::kChunkKb * C::kMkbBytes);
-                    for (int j = 0; j < C::kChunkKb; ++j) {
-                        const int kb = pass * C::kChunkKb + j;
-                        const uint32_t dst = sbase + C::kMOff + j * C::kMkbBytes;
-                        ptx::tma_load_2d(dst, &mM, mf, kb * 64, 0);
-                        ptx::tma_load_2d(dst + R * 128, &mM, mf, kb * 64, R);
-                    }
-                    ptx::mbar_wait(mf, pass & 1, nullptr);
-                }
-            }
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -310,6 +288,64 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         const uint32_t acc2 = lane_addr + C::kRCols;
         const float *om1 = prm, *ph1 = prm + R, *om2 = prm + 2 * R, *ph2 = prm + 3 * R;
         uint8_t *tile = smem;  // the ring is free once the main accumulator is complete
+        // The mixing matrix, bf16 high and low parts, K-major in the SW128
+        // layout: group gi covers operand row n (an output column) and k-columns
+        // [c, c + 8) of k-block j of a pass.  n runs fastest, so a warp reads
+        // whole 128-byte rows of M in the forward.
+        const int et = threadIdx.x - 64;  // 0..255
+        constexpr int kGroups = R * 8 * C::kChunkKb;
+        constexpr int kIters = (kGroups + 255) / 256;
+        float mraw[kIters][8];
+        auto m_group = [&](int it, int pass, int &j, int &n, int &cg, int &c) {
+            const int gi = et + it * 256;
+            j = gi / (R * 8);
+            n = gi % R;
+            cg = ((gi / R) % 8) * 8;
+            c = (pass * C::kChunkKb + j) * 64 + cg;  // k index
+            return gi < kGroups && c < R;
+        };
+        // loads only: the values are first used in m_store, so the loads stay
+        // in flight across whatever runs in between
+        auto m_load = [&](int pass) {
+#pragma unroll
+            for (int it = 0; it < kIters; ++it) {
+                int j, n, cg, c;
+                if (!m_group(it, pass, j, n, cg, c)) continue;
+                if constexpr (BWD) {
+                    const float4 *src = reinterpret_cast<const float4 *>(args.M + (int64_t)n * R + c);  // M[n][c+q]
+                    const float4 u = __ldg(src), w = __ldg(src + 1);
+                    mraw[it][0] = u.x, mraw[it][1] = u.y, mraw[it][2] = u.z, mraw[it][3] = u.w;
+                    mraw[it][4] = w.x, mraw[it][5] = w.y, mraw[it][6] = w.z, mraw[it][7] = w.w;
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) mraw[it][q] = __ldg(args.M + (int64_t)(c + q) * R + n);  // M[c+q][n]
+                }
+            }
+        };
+        auto m_store = [&](int pass) {
+#pragma unroll
+            for (int it = 0; it < kIters; ++it) {
+                int j, n, cg, c;
+                if (!m_group(it, pass, j, n, cg, c)) continue;
+                uint4 hi, lo;
+                uint32_t *ph = &hi.x, *pl = &lo.x;
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    const __nv_bfloat162 h2 = __floats2bfloat162_rn(mraw[it][2 * q], mraw[it][2 * q + 1]);
+                    const float2 hf = __bfloat1622float2(h2);
+                    const __nv_bfloat162 l2 =
+                        __floats2bfloat162_rn(mraw[it][2 * q] - hf.x, mraw[it][2 * q + 1] - hf.y);
+                    ph[q] = *reinterpret_cast<const uint32_t *>(&h2);
+                    pl[q] = *reinterpret_cast<const uint32_t *>(&l2);
+                }
+                const uint32_t off =
+                    C::kMOff + j * C::kMkbBytes + n * 128 + ((((uint32_t)cg >> 3) ^ (n & 7)) << 4);
+                *reinterpret_cast<uint4 *>(smem + off) = hi;
+                *reinterpret_cast<uint4 *>(smem + off + R * 128) = lo;
+            }
+        };
+        // the first pass's part of M is read while the main loop runs
+        m_load(0);
         bool bias_ok = true;
         if constexpr (BWD) {
             if (args.bias_part) {
@@ -359,6 +395,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         bool ok = bias_ok && ptx::mbar_wait(tmem_full, 0, args.status);
         ok = ptx::named_barrier_and(3, 256, ok);  // uniform over the epilogue warps
         if (ok) {
+            // the ring is free once the main accumulator is complete
+            m_store(0);
             ptx::tc_fence_after();
             // ---- phase 1: first accumulator -> bf16 operand tile (+ outputs)
 #pragma unroll 1
@@ -429,17 +467,24 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     }
                 }
             }
-            // ---- second MMA: (128 x r operand tile) x (r x r mixing matrix)
-            ptx::fence_proxy_async_smem();
-            ptx::named_barrier_sync(1, 256);
-            if (threadIdx.x == 64) {
-                constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
-                const uint32_t acc = tmem + C::kRCols;
-                bool mok = true;
-                for (int pass = 0; pass < C::kPasses && mok; ++pass) {
-                    mok = ptx::mbar_wait(m_full, pass & 1, args.status);
+            // ---- second MMA: (128 x r operand tile) x (r x r mixing matrix), the
+            // matrix converted to bf16 hi/lo operand blocks by these threads,
+            // kChunkKb k-blocks per pass
+            constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
+            for (int pass = 0; ok && pass < C::kPasses; ++pass) {
+                if (pass > 0) {
+                    // the previous pass's MMAs have read the operand blocks
+                    ok = ptx::mbar_wait(m_empty, (pass - 1) & 1, args.status);
+                    ok = ptx::named_barrier_and(3, 256, ok);
+                    if (!ok) break;
+                    m_load(pass);
+                    m_store(pass);
+                }
+                ptx::fence_proxy_async_smem();
+                ptx::named_barrier_sync(1, 256);
+                if (threadIdx.x == 64) {
                     ptx::tc_fence_after();
-                    if (!mok) break;
+                    const uint32_t acc = tmem + C::kRCols;
                     for (int j = 0; j < C::kChunkKb; ++j) {
                         const int kb = pass * C::kChunkKb + j;
 #pragma unroll
@@ -459,10 +504,12 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     }
                     if (pass + 1 < C::kPasses) ptx::mma_commit(m_empty);
                 }
-                ptx::mma_commit(mma2_done);
             }
-            ok = ptx::mbar_wait(mma2_done, 0, args.status);
-            ok = ptx::named_barrier_and(3, 256, ok);
+            // also after a failed wait: the MMAs already issued finish before
+            // the tile and the accumulator are given up
+            if (threadIdx.x == 64) ptx::mma_commit(mma2_done);
+            const bool done = ptx::mbar_wait(mma2_done, 0, args.status);
+            ok = ptx::named_barrier_and(3, 256, ok && done);
         }
         if (ok) {
             ptx::tc_fence_after();
