@@ -176,11 +176,11 @@ void wgrad_shapes(const noble_linear_desc *d, int64_t (&mn)[5][2])
 // Backward scratch.
 //   CUDA-core path: dh (dtype), dc, a, db (fp32) [T][r]; M^T fp32; per-block
 //     partials of the CosNet sums, of dM and of dbias.
-//   tensor-core path: dh, a, db (bf16) [T][r]; W_up^T (bf16 [r][d_out]);
-//     per-CTA CosNet and dbias partials; without a branch an all-ones
+//   tensor-core path: dh, a, db (bf16) [T][r]; per-CTA CosNet and dbias
+//     partials; without a branch an all-ones
 //     [T][64] bf16 operand (dbias = dy^T 1).
 struct WorkLayout {
-    size_t dh, dc, a, db, mt, wupt, ones, cos_part, dm_part, bias_part, wsplit[5], total;
+    size_t dh, dc, a, db, mt, ones, cos_part, dm_part, bias_part, wsplit[5], total;
     int split;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
 };
@@ -195,7 +195,6 @@ WorkLayout work_layout(const noble_linear_desc *d)
     if (use_tc(d)) {
         L.a = take(tr * 2);
         L.db = take(tr * 2);
-        L.wupt = take((size_t)r * d->d_out * 2);
         L.ones = r ? 0 : take((size_t)T * kOnesCols * 2);  // dbias = dy^T 1 without a branch
         // one partial per CTA of the CosNet kernel, whose grid is a whole number
         // of CTA pairs (a padding CTA contributes exact zeros)
@@ -706,43 +705,19 @@ noble_status with_rank_tile(int64_t r, F &&f)
     return fail(NOBLE_ERR_UNSUPPORTED, "rank %lld", (long long)r);
 }
 
-// Preparation of the small bf16 operands of the backward tensor-core path,
-// in one launch: blocks [0, nt) transpose W_up [d_out][r] into wupt
-// [r][d_out] in 32 x 32 tiles; the rest fill the all-ones [T][kOnesCols]
-// operand.
-__global__ void prep_bf16_kernel(int64_t d_out, int r, const bf16 *W_up, bf16 *wupt, int nt, int64_t ones_n,
-                                 bf16 *ones)
+// The all-ones [T][kOnesCols] bf16 operand of the backward without a branch
+// (dbias = dy^T 1 as extra weight-gradient columns).
+__global__ void fill_ones_kernel(int64_t n, bf16 *ones)
 {
-    __shared__ bf16 tile[32][33];
-    const int b = blockIdx.x;
-    if (b < nt) {
-        const int tiles_c = (r + 31) / 32;
-        const int64_t r0 = (int64_t)(b / tiles_c) * 32, c0 = (int64_t)(b % tiles_c) * 32;
-        for (int i = threadIdx.x / 32; i < 32; i += blockDim.x / 32) {
-            const int64_t rr = r0 + i, cc = c0 + threadIdx.x % 32;
-            if (rr < d_out && cc < r) tile[i][threadIdx.x % 32] = W_up[rr * r + cc];
-        }
-        __syncthreads();
-        for (int i = threadIdx.x / 32; i < 32; i += blockDim.x / 32) {
-            const int64_t cc = c0 + i, rr = r0 + threadIdx.x % 32;
-            if (rr < d_out && cc < r) wupt[cc * d_out + rr] = tile[threadIdx.x % 32][i];
-        }
-        return;
-    }
-    const int64_t idx = (int64_t)(b - nt) * blockDim.x + threadIdx.x;
-    if (idx < ones_n) ones[idx] = __float2bfloat16_rn(1.f);
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx < n) ones[idx] = __float2bfloat16_rn(1.f);
 }
 
-noble_status prep_bf16(cudaStream_t st, int64_t d_out, int64_t r, const bf16 *W_up, bf16 *wupt, int64_t ones_n,
-                       bf16 *ones)
+noble_status fill_ones(cudaStream_t st, int64_t n, bf16 *ones)
 {
-    const int nt = wupt ? (int)(ceil_div(d_out, 32) * ceil_div(r, 32)) : 0;
-    const int no = ones ? (int)ceil_div(ones_n, 256) : 0;
-    if (nt + no == 0) return NOBLE_OK;
-    const KernelInfo ki{"prep_bf16", kBoundHbm, 0.0, 4.0 * (wupt ? d_out * r : 0) + 2.0 * (ones ? ones_n : 0)};
-    return run(st, ki, [&] {
-        prep_bf16_kernel<<<nt + no, 256, 0, st>>>(d_out, (int)r, W_up, wupt, nt, ones ? ones_n : 0, ones);
-    });
+    if (n == 0) return NOBLE_OK;
+    const KernelInfo ki{"fill_ones", kBoundHbm, 0.0, 2.0 * n};
+    return run(st, ki, [&] { fill_ones_kernel<<<(unsigned)ceil_div(n, 256), 256, 0, st>>>(n, ones); });
 }
 
 // Fixed-order sums of partial results: out_j[i] = sum_z part_j[z * stride_j + i]
@@ -787,10 +762,13 @@ template <int R, bool BWD>
 noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const bf16 *A, int64_t K, const bf16 *B,
                            const tc::CosnetArgs &args_in)
 {
-    using Cfg = tc::CosnetCfg<R>;
+    using Cfg = tc::CosnetCfg<R, BWD>;
     CUtensorMap mA, mB;
     NOBLE_TRY(make_map(&mA, A, T, K, tc::kBM));
-    NOBLE_TRY(make_map(&mB, B, R, K, R / 2));  // each CTA of a pair loads half of the rows
+    if (BWD)  // B = W_up [K = d_out][R], MN-major; each CTA of a pair loads half of the K rows
+        NOBLE_TRY(make_map(&mB, B, K, R, tc::kBK / 2));
+    else  // B = W_down [R][K], K-major; each CTA of a pair loads half of the rows
+        NOBLE_TRY(make_map(&mB, B, R, K, R / 2));
     tc::CosnetArgs args = args_in;
     args.T = T;
     args.kb = (int)ceil_div(K, tc::kBK);
@@ -853,10 +831,9 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     const SavedLayout SL = saved_layout(d);
     const WorkLayout WL = work_layout(d);
     bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
-    bf16 *wupt = (bf16 *)(ws + WL.wupt), *ones = (bf16 *)(ws + WL.ones);
+    bf16 *ones = (bf16 *)(ws + WL.ones);
     const bool ones_dbias = dbias && r == 0;
-    NOBLE_TRY(prep_bf16(st, dout, r, r ? W_up : nullptr, r ? wupt : nullptr, ones_dbias ? T * kOnesCols : 0,
-                        ones_dbias ? ones : nullptr));
+    if (ones_dbias) NOBLE_TRY(fill_ones(st, T * kOnesCols, ones));
     if (r > 0) {
         float *cpart = (float *)(ws + WL.cos_part);
         tc::CosnetArgs ca{};
@@ -867,7 +844,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         ca.bias_part = dbias ? bpart : nullptr;
         ca.kdim = dout;
         NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-            return cosnet_launch<decltype(bn)::value, true>(st, "tc_dc_cosnet_bwd", T, dy, dout, wupt, ca);
+            return cosnet_launch<decltype(bn)::value, true>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
         }));
         // domega1, dphi1, domega2, dphi2 (and dbias) from the per-CTA partials
         SplitJobs J{};

@@ -51,12 +51,21 @@ struct CosnetArgs {
     uint32_t *status;
 };
 
-template <int R>
+// B_MN: the main loop's B operand is MN-major (W_up [d_out][r] as stored, in
+// the backward), loaded as 64-wide column chunks of 64 K rows each; otherwise
+// it is K-major with R rows (W_down [r][d_in], in the forward).
+template <int R, bool B_MN>
 struct CosnetCfg {
-    static constexpr int kRCols = R < 32 ? 32 : R;         // TMEM columns per accumulator
+    // N of the main MMA: an MN-major B is read in whole 64-wide swizzle atoms,
+    // so for r < 64 the MMA runs 64 columns wide (the columns past r are
+    // zero-filled by the copy and never read back)
+    static constexpr int kMainN = B_MN && R < 64 ? 64 : R;
+    static constexpr int kRCols = kMainN < 32 ? 32 : kMainN;  // TMEM columns per accumulator
     static constexpr uint32_t kTmemCols = 2 * kRCols;     // h|dc and b|da
+    static constexpr int kBChunks = (R + 63) / 64;         // MN-major B: 64-wide column chunks
+    static constexpr uint32_t kChunkBytes = kBK * 128;     // one chunk: 64 K rows of 128 bytes
     static constexpr uint32_t kA = kBM * kBK * 2;
-    static constexpr uint32_t kB = R * kBK * 2;
+    static constexpr uint32_t kB = B_MN ? kBChunks * kChunkBytes : R * kBK * 2;
     static constexpr uint32_t kStage = kA + kB;
     static constexpr int kMkb = (R + 63) / 64;            // k-blocks of the r x r operand
     static constexpr int kKSteps = R < 64 ? R / 16 : 4;   // MMA K-steps per k-block
@@ -187,7 +196,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kCosnetThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const CosnetArgs args)
 {
-    using C = CosnetCfg<R>;
+    using C = CosnetCfg<R, BWD>;
     constexpr int STAGES = C::kStages;
     auto store_hi_lo = [](uint8_t *tile, int row, int col, const float(&o)[8]) {
         return store_hi_lo_impl<C::kTileBytes>(tile, row, col, o);
@@ -251,8 +260,16 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 ptx::mbar_arrive_expect_tx(fb, C::kStage);
                 const uint32_t sA = sbase + s * C::kStage;
                 ptx::tma_load_2d(sA, &mA, fb, i * kBK, (int)m0);
-                // this CTA's half of the B rows, to the same offset in both CTAs
-                tma_load_2d_mc(sA + C::kA + rank * (R / 2) * 128, &mB, fb, i * kBK, (int)rank * (R / 2), 0x3);
+                if constexpr (BWD) {
+                    // this CTA's half of the 64 K rows of every column chunk, to
+                    // the same offsets in both CTAs
+                    for (int c = 0; c < C::kBChunks; ++c)
+                        tma_load_2d_mc(sA + C::kA + c * C::kChunkBytes + rank * (kBK / 2) * 128, &mB, fb, c * 64,
+                                       i * kBK + (int)rank * (kBK / 2), 0x3);
+                } else {
+                    // this CTA's half of the B rows, to the same offset in both CTAs
+                    tma_load_2d_mc(sA + C::kA + rank * (R / 2) * 128, &mB, fb, i * kBK, (int)rank * (R / 2), 0x3);
+                }
                 ++issued;
             }
             for (int i = issued > STAGES ? issued - STAGES : 0; i < issued; ++i)
@@ -260,7 +277,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         }
     } else if (warp == 1) {
         if (lane == 0) {
-            constexpr uint32_t idesc = ptx::idesc_bf16(kBM, R, false, false);
+            constexpr uint32_t idesc = ptx::idesc_bf16(kBM, C::kMainN, false, BWD);
             for (int i = 0; i < args.kb; ++i) {
                 const int s = i % STAGES;
                 const uint32_t ph = (i / STAGES) & 1;
@@ -268,9 +285,14 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 ptx::tc_fence_after();
                 const uint32_t sA = sbase + s * C::kStage, sB = sA + C::kA;
 #pragma unroll
-                for (int kk = 0; kk < kBK / 16; ++kk)
-                    ptx::mma_bf16(tmem, ptx::smem_desc_sw128(sA + kk * 32, 16, 1024),
-                                  ptx::smem_desc_sw128(sB + kk * 32, 16, 1024), idesc, (i > 0 || kk > 0) ? 1u : 0u);
+                for (int kk = 0; kk < kBK / 16; ++kk) {
+                    // MN-major B: 16 K rows are two 8-row groups (2048 bytes);
+                    // the column chunks are kChunkBytes apart
+                    const uint64_t bd = BWD ? ptx::smem_desc_sw128(sB + kk * 2048, C::kChunkBytes, 1024)
+                                            : ptx::smem_desc_sw128(sB + kk * 32, 16, 1024);
+                    ptx::mma_bf16(tmem, ptx::smem_desc_sw128(sA + kk * 32, 16, 1024), bd, idesc,
+                                  (i > 0 || kk > 0) ? 1u : 0u);
+                }
                 mma_commit_mc(empty_bar(s), 0x3);
             }
             ptx::mma_commit(tmem_full);
