@@ -406,6 +406,28 @@ noble_status make_map_mn4(CUtensorMap *m, const void *ptr, int64_t K, int64_t MN
     return NOBLE_OK;
 }
 
+// 3-D TMA map for the pair kernel's stores into C: dimensions (inner first)
+// {N, M, nsplit} with row pitch ldc and split pitch split_stride (elements),
+// box {128 bytes of columns, 32 rows, 1}, 128-byte swizzle.
+noble_status make_store_map(CUtensorMap *m, void *C, bool fp32, int64_t M, int64_t N, int64_t ldc, int64_t nsplit,
+                            int64_t split_stride)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    const cuuint64_t es = fp32 ? 4 : 2;
+    cuuint64_t dims[3] = {(cuuint64_t)N, (cuuint64_t)M, (cuuint64_t)nsplit};
+    cuuint64_t strides[2] = {(cuuint64_t)ldc * es, (cuuint64_t)(nsplit > 1 ? split_stride : M * ldc) * es};
+    cuuint32_t box[3] = {(cuuint32_t)(128 / es), 32, 1};
+    cuuint32_t estr[3] = {1, 1, 1};
+    CUresult r = enc(m, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, C, dims, strides,
+                     box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                     CU_TENSOR_MAP_L2_PROMOTION_NONE, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS)
+        return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled (store) failed (%d): M=%lld N=%lld ldc=%lld", (int)r,
+                    (long long)M, (long long)N, (long long)ldc);
+    return NOBLE_OK;
+}
+
 // Device address of this device's status word (looked up once per device).
 uint32_t *status_ptr()
 {
@@ -649,6 +671,17 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         q.kb_per_split = P.kb_per_split;
         q.tile_begin = tiles;
         q.ep = eps[i];
+        {
+            // TMA-store epilogue where C's layout allows it
+            using OutT = typename Epi::out_type;
+            constexpr int64_t es = sizeof(OutT);
+            const auto &e = eps[i];
+            const bool ok = !e.col0 && reinterpret_cast<uintptr_t>(e.C) % 16 == 0 && (e.ldc * es) % 16 == 0 &&
+                            P.N % 4 == 0 && (P.nsplit == 1 || (e.split_stride * es) % 16 == 0);
+            q.ep.tma = ok ? 1 : 0;
+            if (ok)
+                NOBLE_TRY(make_store_map(&maps.m[np][4], e.C, es == 4, P.M, P.N, e.ldc, P.nsplit, e.split_stride));
+        }
         tiles += (int)ceil_div(q.tiles_m, 2) * q.tiles_n * q.nsplit;
         const double K = (double)P.s0.K + (P.s1 ? (double)P.s1->K : 0.0);
         flops += 2.0 * P.M * P.N * K;

@@ -51,12 +51,14 @@ struct TmemCols {
 // Plain store: C[z][m][n] = acc (+ bias[n]) in OutT.  N must be a multiple of 8.
 template <typename OutT>
 struct EpiStore {
+    using out_type = OutT;
     struct Params {
         OutT *C;
         int64_t ldc;
         const float *bias;
         int64_t split_stride;  // elements between blockIdx.z partial outputs
         int col0 = 0;          // store only column 0 of each row, to C[row * ldc]
+        int tma = 0;           // pair kernel: store through a 3-D TMA map of C (run_tma)
     };
 
     // 32 accumulator columns [c, c+32) of this thread's row -> C (+ bias)
@@ -107,6 +109,66 @@ struct EpiStore {
             float v[32];
             ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
             if (row < M) store32(p, out, v, n0 + c, N);
+        }
+    }
+
+    // TMA-store epilogue of the pair kernel.  The warp's 32 rows are written
+    // in boxes of kBoxCols columns (128 bytes per row): the accumulator chunk
+    // (+ bias) is converted into the warp's 4 KB staging buffer in the
+    // 128-byte-swizzled layout and stored by one 3-D TMA copy at
+    // (column, row, split); rows >= M and columns >= N are clipped by the copy.
+    // The warp's boxes start at column half * kBoxCols and step by 2 kBoxCols.
+    // Requires N % 4 == 0 (whole float4 groups of bias).
+    static constexpr int kBoxCols = 128 / (int)sizeof(OutT);
+    __device__ static void run_tma(const Params &p, const CUtensorMap *map, uint8_t *stg_ptr, uint32_t stg,
+                                   uint32_t tmem, int bn, int quarter, int lane, int64_t m0, int64_t n0, int64_t N,
+                                   int z, int half)
+    {
+        const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+        uint8_t *my_row = stg_ptr + lane * 128;
+#pragma unroll 1
+        for (int c = half * kBoxCols; c < bn; c += 2 * kBoxCols) {
+            if (n0 + c >= N) break;  // warp-uniform
+            if (lane == 0) ptx::bulk_wait_read_all();  // the previous box has left the buffer
+            __syncwarp();
+#pragma unroll
+            for (int h = 0; h < kBoxCols / 32; ++h) {
+                float v[32];
+                ptx::tmem_ld_32x32b_x32(lane_addr + c + 32 * h, v);
+                const int64_t n = n0 + c + 32 * h;
+                if (p.bias) {
+#pragma unroll
+                    for (int q = 0; q < 8; ++q) {
+                        if (n + 4 * q < N) {
+                            const float4 b = __ldg(reinterpret_cast<const float4 *>(p.bias + n) + q);
+                            v[4 * q] += b.x, v[4 * q + 1] += b.y, v[4 * q + 2] += b.z, v[4 * q + 3] += b.w;
+                        }
+                    }
+                }
+                if constexpr (sizeof(OutT) == 2) {
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        const int j = h * 4 + g;  // 16-byte piece of the 128-byte row
+                        uint4 q;
+                        q.x = ptx::pack_bf16x2(v[8 * g], v[8 * g + 1]);
+                        q.y = ptx::pack_bf16x2(v[8 * g + 2], v[8 * g + 3]);
+                        q.z = ptx::pack_bf16x2(v[8 * g + 4], v[8 * g + 5]);
+                        q.w = ptx::pack_bf16x2(v[8 * g + 6], v[8 * g + 7]);
+                        *reinterpret_cast<uint4 *>(my_row + ((j ^ (lane & 7)) << 4)) = q;
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 8; ++j)
+                        *reinterpret_cast<float4 *>(my_row + ((j ^ (lane & 7)) << 4)) =
+                            make_float4(v[4 * j], v[4 * j + 1], v[4 * j + 2], v[4 * j + 3]);
+                }
+            }
+            ptx::fence_proxy_async_smem();
+            __syncwarp();
+            if (lane == 0) {
+                ptx::tma_store_3d(map, stg, (int)(n0 + c), (int)(m0 + quarter * 32), z);
+                ptx::bulk_commit_group();
+            }
         }
     }
 

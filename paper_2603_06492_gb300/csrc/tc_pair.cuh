@@ -172,7 +172,9 @@ struct PairSmem {
     static constexpr uint32_t kA = kBM * kBK * 2;         // 128 rows of A
     static constexpr uint32_t kB = 128 * kBK * 2;         // up to 128 columns of B
     static constexpr uint32_t kStage = kA + kB;
-    static constexpr uint32_t kBarOff = STAGES * kStage;
+    static constexpr uint32_t kStgOff = STAGES * kStage;  // epilogue staging, 4 KB per epilogue warp
+    static constexpr uint32_t kStgBytes = 8 * 4096;
+    static constexpr uint32_t kBarOff = kStgOff + kStgBytes;
     static constexpr uint32_t kNumBars = 2 * STAGES + 5;  // full, empty, tfull[2], tempty[2], mma_done
     static constexpr uint32_t kBytes = kBarOff + 8 * kNumBars + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
@@ -342,6 +344,8 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         const int half = (warp - 2) / 4;  // two warps per TMEM lane quarter split the columns
         const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
         const uint32_t leader_tempty1 = map_to_rank(tempty_bar(1), 0);
+        const uint32_t stg = sbase + S::kStgOff + (uint32_t)(warp - 2) * 4096u;
+        uint8_t *stg_ptr = smem + S::kStgOff + (warp - 2) * 4096;
         int j = 0;
         const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
         for (int slot = cluster; slot < nslots; slot += nclusters) {
@@ -355,12 +359,18 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             ok = __all_sync(0xffffffffu, ok);
             if (!ok) break;
             ptx::tc_fence_after();
-            Epi::run_dyn(P.ep, tmem + b * kAccCols, P.bn, quarter, lane, tr.m0, tr.n0, P.M, P.N, tr.z, 32 * half, 64);
+            if (P.ep.tma)
+                Epi::run_tma(P.ep, &maps.m[tr.prob][4], stg_ptr, stg, tmem + b * kAccCols, P.bn, quarter, lane, tr.m0,
+                             tr.n0, P.N, tr.z, half);
+            else
+                Epi::run_dyn(P.ep, tmem + b * kAccCols, P.bn, quarter, lane, tr.m0, tr.n0, P.M, P.N, tr.z, 32 * half,
+                             64);
             ptx::tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive_cluster(b ? leader_tempty1 : leader_tempty0);
             ++j;
         }
+        if (lane == 0) ptx::bulk_wait_all();  // stores done before the staging buffer goes away
     }
 
     ptx::tc_fence_before();

@@ -46,7 +46,7 @@ struct GroupArgs {
 };
 
 struct GroupMaps {
-    CUtensorMap m[kMaxProblems][4];  // A0, B0, A1, B1
+    CUtensorMap m[kMaxProblems][5];  // A0, B0, A1, B1, C (pair kernel's TMA-store epilogue)
 };
 
 struct TileRef {
