@@ -291,10 +291,18 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         }
     } else if (warp == 1) {
         if (lane == 0 && leader) {
-            // ---------------- MMA issuer (leader CTA only)
-            uint32_t it = 0;
+            // ---------------- MMA issuer (leader CTA only).  The loop keeps the
+            // work between consecutive k-blocks small: operand descriptors are
+            // a per-tile base plus additive offsets (start addresses are below
+            // 256 KB, so the 14-bit address field never carries), and the ring
+            // position advances incrementally.
+            int s = 0;
+            uint32_t ph = 0;
             int j = 0;
             bool ok = true;
+            // descriptor address-field steps (16-byte units) per K-step of 16
+            constexpr uint32_t kStepA = A_MN ? (MN4 ? 4096 / 16 : 2048 / 16) : 32 / 16;
+            constexpr uint32_t kStageUnits = S::kStage / 16;
             const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
             for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
                 const int t = slot_tile(g, slot);
@@ -307,30 +315,32 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                 ptx::tc_fence_after();
                 const uint32_t d_tmem = tmem + b * kAccCols;
                 const uint32_t idesc = ptx::idesc_bf16(2 * kBM, P.bn, A_MN, B_MN);
-                bool first = true;
-                for (int kb = tr.kb_begin; kb < tr.kb_end; ++kb, ++it) {
-                    const int s = it % STAGES;
-                    const uint32_t ph = (it / STAGES) & 1;
+                const uint32_t nchB = (uint32_t)P.bn / 128;  // 64-wide B chunks held per CTA
+                const uint64_t a0 = A_MN ? (MN4 ? ptx::smem_desc_sw128(sbase, 1024, 2048)
+                                                : ptx::smem_desc_sw128(sbase, kChunkBytes, 1024))
+                                         : ptx::smem_desc_sw128(sbase, 16, 1024);
+                const uint64_t b0 = B_MN ? (MN4 ? ptx::smem_desc_sw128(sbase + S::kA, 1024, 1024 * nchB)
+                                                : ptx::smem_desc_sw128(sbase + S::kA, kChunkBytes, 1024))
+                                         : ptx::smem_desc_sw128(sbase + S::kA, 16, 1024);
+                const uint32_t stepB = B_MN ? (MN4 ? 128u * nchB : 2048u / 16) : 32u / 16;
+                const int nkb = tr.kb_end - tr.kb_begin;
+                for (int i = 0; i < nkb; ++i) {
                     if (!ptx::mbar_wait(full_bar(s), ph, g.status)) {
                         ok = false;
                         break;
                     }
                     ptx::tc_fence_after();
-                    const uint32_t sA = sbase + s * S::kStage, sB = sA + S::kA;
-                    const uint32_t nchB = (uint32_t)P.bn / 128;  // 64-wide B chunks held per CTA
+                    const uint64_t so = (uint64_t)((uint32_t)s * kStageUnits);
+                    const uint64_t ad = a0 + so, bd = b0 + so;
+                    mma2_bf16(d_tmem, ad, bd, idesc, i > 0 ? 1u : 0u);
 #pragma unroll
-                    for (int kk = 0; kk < kBK / 16; ++kk) {
-                        uint64_t ad, bd;
-                        if (A_MN && MN4) ad = ptx::smem_desc_sw128(sA + kk * 4096, 1024, 2048);
-                        else if (A_MN) ad = ptx::smem_desc_sw128(sA + kk * 2048, kChunkBytes, 1024);
-                        else ad = ptx::smem_desc_sw128(sA + kk * 32, 16, 1024);
-                        if (B_MN && MN4) bd = ptx::smem_desc_sw128(sB + kk * 2048 * nchB, 1024, 1024 * nchB);
-                        else if (B_MN) bd = ptx::smem_desc_sw128(sB + kk * 2048, kChunkBytes, 1024);
-                        else bd = ptx::smem_desc_sw128(sB + kk * 32, 16, 1024);
-                        mma2_bf16(d_tmem, ad, bd, idesc, first ? 0u : 1u);
-                        first = false;
-                    }
+                    for (int kk = 1; kk < kBK / 16; ++kk)
+                        mma2_bf16(d_tmem, ad + kk * kStepA, bd + kk * stepB, idesc, 1u);
                     mma2_commit_mc(empty_bar(s), 0x3);
+                    if (++s == STAGES) {
+                        s = 0;
+                        ph ^= 1;
+                    }
                 }
                 mma2_commit_mc(tfull_bar(b), 0x3);
                 ++j;
