@@ -324,8 +324,15 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                                          : ptx::smem_desc_sw128(sbase + S::kA, 16, 1024);
                 const uint32_t stepB = B_MN ? (MN4 ? 128u * nchB : 2048u / 16) : 32u / 16;
                 const int nkb = tr.kb_end - tr.kb_begin;
-                for (int i = 0; i < nkb; ++i) {
-                    if (!ptx::mbar_wait(full_bar(s), ph, g.status)) {
+                for (int i = 0; i < nkb; i += 2) {
+                    const bool two = i + 1 < nkb;
+                    int s2 = s + 1;
+                    uint32_t ph2 = ph;
+                    if (s2 == STAGES) {
+                        s2 = 0;
+                        ph2 ^= 1;
+                    }
+                    if (!ptx::mbar_wait(full_bar(s), ph, g.status) || (two && !ptx::mbar_wait(full_bar(s2), ph2, g.status))) {
                         ok = false;
                         break;
                     }
@@ -337,9 +344,22 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     for (int kk = 1; kk < kBK / 16; ++kk)
                         mma2_bf16(d_tmem, ad + kk * kStepA, bd + kk * stepB, idesc, 1u);
                     mma2_commit_mc(empty_bar(s), 0x3);
-                    if (++s == STAGES) {
-                        s = 0;
-                        ph ^= 1;
+                    if (two) {
+                        const uint64_t so2 = (uint64_t)((uint32_t)s2 * kStageUnits);
+                        const uint64_t ad2 = a0 + so2, bd2 = b0 + so2;
+#pragma unroll
+                        for (int kk = 0; kk < kBK / 16; ++kk)
+                            mma2_bf16(d_tmem, ad2 + kk * kStepA, bd2 + kk * stepB, idesc, 1u);
+                        mma2_commit_mc(empty_bar(s2), 0x3);
+                        s = s2 + 1;
+                        ph = ph2;
+                        if (s == STAGES) {
+                            s = 0;
+                            ph ^= 1;
+                        }
+                    } else {
+                        s = s2;
+                        ph = ph2;
                     }
                 }
                 mma2_commit_mc(tfull_bar(b), 0x3);
