@@ -126,6 +126,63 @@ __device__ __forceinline__ float warp_colsum32(float (&v)[32])
     return v[0];
 }
 
+// Coalesced row segments for the epilogue.  Lane l of a warp owns row
+// t0 + l and holds P 16-byte pieces of it (one segment of P * 16 bytes).
+// transpose_pieces swaps the lane and piece index bits within groups of P
+// lanes (log2 P xor-shuffle stages): afterwards lane l holds, in slot i,
+// piece l % P of row (l & ~(P - 1)) + i, so each memory instruction covers
+// 32 / P whole row segments instead of 32 scattered 16-byte pieces.  The
+// exchange is its own inverse, which the loads use.
+template <int P>
+__device__ __forceinline__ void transpose_pieces(uint32_t (&w)[P][4])
+{
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int m = P / 2; m >= 1; m >>= 1) {
+        const bool hi = (lane & m) != 0;
+#pragma unroll
+        for (int a = 0; a < P; ++a) {
+            if (a & m) continue;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint32_t send = hi ? w[a][q] : w[a | m][q];
+                const uint32_t recv = __shfl_xor_sync(0xffffffffu, send, m);
+                if (hi) w[a][q] = recv;
+                else w[a | m][q] = recv;
+            }
+        }
+    }
+}
+// Store the warp's segments: dst = address of the first piece of row t0;
+// rows at or past T are skipped.
+template <int P>
+__device__ __forceinline__ void store_segments(uint32_t (&w)[P][4], void *dst, int64_t pitch, int64_t t0, int64_t T)
+{
+    transpose_pieces<P>(w);
+    const int lane = threadIdx.x & 31;
+    const int gb = lane & ~(P - 1);
+    uint8_t *p = reinterpret_cast<uint8_t *>(dst) + (lane & (P - 1)) * 16;
+#pragma unroll
+    for (int i = 0; i < P; ++i)
+        if (t0 + gb + i < T)
+            *reinterpret_cast<uint4 *>(p + (int64_t)(gb + i) * pitch) = make_uint4(w[i][0], w[i][1], w[i][2], w[i][3]);
+}
+// Load the warp's segments (zeros for rows at or past T).
+template <int P>
+__device__ __forceinline__ void load_segments(uint32_t (&w)[P][4], const void *src, int64_t pitch, int64_t t0, int64_t T)
+{
+    const int lane = threadIdx.x & 31;
+    const int gb = lane & ~(P - 1);
+    const uint8_t *p = reinterpret_cast<const uint8_t *>(src) + (lane & (P - 1)) * 16;
+#pragma unroll
+    for (int i = 0; i < P; ++i) {
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (t0 + gb + i < T) v = __ldg(reinterpret_cast<const uint4 *>(p + (int64_t)(gb + i) * pitch));
+        w[i][0] = v.x, w[i][1] = v.y, w[i][2] = v.z, w[i][3] = v.w;
+    }
+    transpose_pieces<P>(w);
+}
+
 // Byte offset of element (row, col) in a 128-row bf16 K-major tile stored as
 // 64-column blocks with the 128-byte swizzle (what TMA writes and UMMA reads).
 __device__ __forceinline__ uint32_t sw128_offset(int row, int col)
@@ -306,6 +363,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         const int row = quarter * 32 + lane;
         const int64_t t = m0 + row;
         const bool live = t < args.T;
+        const int64_t t0 = m0 + quarter * 32;  // the warp's first row
         const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
         const uint32_t acc2 = lane_addr + C::kRCols;
         const float *om1 = prm, *ph1 = prm + R, *om2 = prm + 2 * R, *ph2 = prm + 3 * R;
@@ -368,6 +426,17 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         };
         // the first pass's part of M is read while the main loop runs
         m_load(0);
+        if constexpr (BWD) {
+            // the tile's saved h and b rows are read after the main loop: bring
+            // them into L2 meanwhile
+            const int64_t nbytes = (min((int64_t)kBM, args.T - m0) > 0 ? min((int64_t)kBM, args.T - m0) : 0) * R * 4;
+            const uint8_t *hrow = reinterpret_cast<const uint8_t *>(args.h_in + m0 * R);
+            const uint8_t *brow = reinterpret_cast<const uint8_t *>(args.b_in + m0 * R);
+            for (int64_t off = (int64_t)et * 128; off < nbytes; off += 256 * 128) {
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(hrow + off));
+                asm volatile("prefetch.global.L2 [%0];" ::"l"(brow + off));
+            }
+        }
         bool bias_ok = true;
         if constexpr (BWD) {
             if (args.bias_part) {
@@ -435,11 +504,13 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 constexpr int W = R < 32 ? R : 32;
                 if constexpr (!BWD) {
                     // v = h: store h, operand a = cos(omega1 h + phi1)
-                    if (live) {
-                        float4 *dst = reinterpret_cast<float4 *>(args.h_out + t * R + c);
+                    {
+                        uint32_t w[W / 4][4];
 #pragma unroll
                         for (int i = 0; i < W / 4; ++i)
-                            dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
+                        store_segments<W / 4>(w, args.h_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
                     }
 #pragma unroll
                     for (int g = 0; g < W / 8; ++g) {
@@ -456,15 +527,16 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     float bv[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) bv[i] = 0.f;
-                    if (live) {
-                        const float4 *src = reinterpret_cast<const float4 *>(args.b_in + t * R + c);
+                    {
+                        uint32_t w[W / 4][4];
+                        load_segments<W / 4>(w, args.b_in + t0 * R + c, (int64_t)R * 4, t0, args.T);
 #pragma unroll
-                        for (int i = 0; i < W / 4; ++i) {
-                            const float4 q = __ldg(src + i);
-                            bv[4 * i] = q.x, bv[4 * i + 1] = q.y, bv[4 * i + 2] = q.z, bv[4 * i + 3] = q.w;
-                        }
+                        for (int i = 0; i < W / 4; ++i)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) bv[4 * i + q] = __uint_as_float(w[i][q]);
                     }
                     float q2[32], q3[32];
+                    uint32_t wdb[W / 8][4];
 #pragma unroll
                     for (int i = W; i < 32; ++i) q2[i] = 0.f, q3[i] = 0.f;
 #pragma unroll
@@ -479,8 +551,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                             q3[j] = du2;
                         }
                         const uint4 q = store_hi_lo(tile, row, c + 8 * g, o);
-                        if (live) *reinterpret_cast<uint4 *>(args.db_out + t * R + c + 8 * g) = q;
+                        wdb[g][0] = q.x, wdb[g][1] = q.y, wdb[g][2] = q.z, wdb[g][3] = q.w;
                     }
+                    store_segments<W / 8>(wdb, args.db_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                     const float s2 = warp_colsum32(q2);
                     const float s3 = warp_colsum32(q3);
                     if (c + lane < R) {
@@ -550,37 +623,39 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 constexpr int W = R < 32 ? R : 32;
                 if constexpr (!BWD) {
                     // v = b
-                    if (live) {
-                        float4 *dst = reinterpret_cast<float4 *>(args.b_out + t * R + c);
+                    uint32_t wc[W / 8][4];
 #pragma unroll
-                        for (int i = 0; i < W / 4; ++i) dst[i] = make_float4(v[4 * i], v[4 * i + 1], v[4 * i + 2], v[4 * i + 3]);
+                    for (int g = 0; g < W / 8; ++g) {
+                        float cc[8];
 #pragma unroll
-                        for (int g = 0; g < W / 8; ++g) {
-                            float cc[8];
+                        for (int i = 0; i < 8; ++i) cc[i] = cos_reduced(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
 #pragma unroll
-                            for (int i = 0; i < 8; ++i) cc[i] = cos_reduced(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
-                            uint4 q;
-                            q.x = ptx::pack_bf16x2(cc[0], cc[1]);
-                            q.y = ptx::pack_bf16x2(cc[2], cc[3]);
-                            q.z = ptx::pack_bf16x2(cc[4], cc[5]);
-                            q.w = ptx::pack_bf16x2(cc[6], cc[7]);
-                            *reinterpret_cast<uint4 *>(args.c_out + t * R + c + 8 * g) = q;
-                        }
+                        for (int q = 0; q < 4; ++q) wc[g][q] = ptx::pack_bf16x2(cc[2 * q], cc[2 * q + 1]);
                     }
+                    {
+                        uint32_t w[W / 4][4];
+#pragma unroll
+                        for (int i = 0; i < W / 4; ++i)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
+                        store_segments<W / 4>(w, args.b_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                    }
+                    store_segments<W / 8>(wc, args.c_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                 } else {
                     // v = da; with h of this row: du1, dh = omega1 du1, a = cos(u1)
                     float hv[32];
 #pragma unroll
                     for (int i = 0; i < 32; ++i) hv[i] = 0.f;
-                    if (live) {
-                        const float4 *src = reinterpret_cast<const float4 *>(args.h_in + t * R + c);
+                    {
+                        uint32_t w[W / 4][4];
+                        load_segments<W / 4>(w, args.h_in + t0 * R + c, (int64_t)R * 4, t0, args.T);
 #pragma unroll
-                        for (int i = 0; i < W / 4; ++i) {
-                            const float4 q = __ldg(src + i);
-                            hv[4 * i] = q.x, hv[4 * i + 1] = q.y, hv[4 * i + 2] = q.z, hv[4 * i + 3] = q.w;
-                        }
+                        for (int i = 0; i < W / 4; ++i)
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) hv[4 * i + q] = __uint_as_float(w[i][q]);
                     }
                     float q0[32], q1[32];
+                    uint32_t wdh[W / 8][4], wa[W / 8][4];
 #pragma unroll
                     for (int i = W; i < 32; ++i) q0[i] = 0.f, q1[i] = 0.f;
 #pragma unroll
@@ -597,20 +672,14 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                             q0[j] = du1 * hv[j];
                             q1[j] = du1;
                         }
-                        if (live) {
-                            uint4 q;
-                            q.x = ptx::pack_bf16x2(dh[0], dh[1]);
-                            q.y = ptx::pack_bf16x2(dh[2], dh[3]);
-                            q.z = ptx::pack_bf16x2(dh[4], dh[5]);
-                            q.w = ptx::pack_bf16x2(dh[6], dh[7]);
-                            *reinterpret_cast<uint4 *>(args.dh_out + t * R + c + 8 * g) = q;
-                            q.x = ptx::pack_bf16x2(av[0], av[1]);
-                            q.y = ptx::pack_bf16x2(av[2], av[3]);
-                            q.z = ptx::pack_bf16x2(av[4], av[5]);
-                            q.w = ptx::pack_bf16x2(av[6], av[7]);
-                            *reinterpret_cast<uint4 *>(args.a_out + t * R + c + 8 * g) = q;
+#pragma unroll
+                        for (int q = 0; q < 4; ++q) {
+                            wdh[g][q] = ptx::pack_bf16x2(dh[2 * q], dh[2 * q + 1]);
+                            wa[g][q] = ptx::pack_bf16x2(av[2 * q], av[2 * q + 1]);
                         }
                     }
+                    store_segments<W / 8>(wdh, args.dh_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                    store_segments<W / 8>(wa, args.a_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                     const float s0 = warp_colsum32(q0);
                     const float s1 = warp_colsum32(q1);
                     if (c + lane < R) {
