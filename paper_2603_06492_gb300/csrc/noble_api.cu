@@ -384,10 +384,11 @@ noble_status make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t col
 // 4-D TMA map over a row-major bf16 matrix [K][MN] (MN contiguous) that loads
 // MN-major tiles in the layout [8-row K group][64-wide MN chunk][8 rows][128 B]:
 // dimensions (inner first) {64 elements, 8 rows, MN/64 chunks, K/8 groups} with
-// strides {P, 128 B, 8 P} for the row pitch P, box {64, 8, nchunks, 8}.
+// strides {P, 128 B, 8 P} for the row pitch P, box {64, 8, nchunks, kgroups}.
 // Requires MN % 64 == 0 and K % 8 == 0, so that every in-range coordinate of
 // the 4-D description is an element of the matrix.
-noble_status make_map_mn4(CUtensorMap *m, const void *ptr, int64_t K, int64_t MN, uint32_t nchunks)
+noble_status make_map_mn4(CUtensorMap *m, const void *ptr, int64_t K, int64_t MN, uint32_t nchunks,
+                          uint32_t kgroups = 8)
 {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
@@ -395,7 +396,7 @@ noble_status make_map_mn4(CUtensorMap *m, const void *ptr, int64_t K, int64_t MN
     const cuuint64_t P = (cuuint64_t)MN * 2;
     cuuint64_t dims[4] = {64, 8, (cuuint64_t)MN / 64, (cuuint64_t)K / 8};
     cuuint64_t strides[3] = {P, 128, 8 * P};
-    cuuint32_t box[4] = {64, 8, nchunks, 8};
+    cuuint32_t box[4] = {64, 8, nchunks, kgroups};
     cuuint32_t estr[4] = {1, 1, 1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void *>(ptr), dims, strides, box, estr,
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -798,7 +799,9 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     using Cfg = tc::CosnetCfg<R, BWD>;
     CUtensorMap mA, mB;
     NOBLE_TRY(make_map(&mA, A, T, K, tc::kBM));
-    if (BWD)  // B = W_up [K = d_out][R], MN-major; each CTA of a pair loads half of the K rows
+    if (Cfg::kBInterleaved)  // B = W_up [K = d_out][R], MN-major, 4 of the 8 K groups per CTA
+        NOBLE_TRY(make_map_mn4(&mB, B, K, R, (uint32_t)(R / 64), 4));
+    else if (BWD)  // B = W_up [K = d_out][R], MN-major; each CTA of a pair loads half of the K rows
         NOBLE_TRY(make_map(&mB, B, K, R, tc::kBK / 2));
     else  // B = W_down [R][K], K-major; each CTA of a pair loads half of the rows
         NOBLE_TRY(make_map(&mB, B, R, K, R / 2));

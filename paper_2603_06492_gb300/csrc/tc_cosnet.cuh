@@ -63,6 +63,10 @@ struct CosnetCfg {
     static constexpr int kRCols = kMainN < 32 ? 32 : kMainN;  // TMEM columns per accumulator
     static constexpr uint32_t kTmemCols = 2 * kRCols;     // h|dc and b|da
     static constexpr int kBChunks = (R + 63) / 64;         // MN-major B: 64-wide column chunks
+    // MN-major B with r a multiple of 64 is copied in the interleaved layout
+    // [8-row K group][column chunk][8 rows][128 B] (one 4-D copy per CTA and
+    // stage); otherwise as column chunks of 64 K rows.
+    static constexpr bool kBInterleaved = B_MN && R % 64 == 0;
     static constexpr uint32_t kChunkBytes = kBK * 128;     // one chunk: 64 K rows of 128 bytes
     static constexpr uint32_t kA = kBM * kBK * 2;
     static constexpr uint32_t kB = B_MN ? kBChunks * kChunkBytes : R * kBK * 2;
@@ -221,6 +225,15 @@ constexpr int kCosnetThreads = 320;
 // stage and multicasts it to both: a stage is refilled only once the MMAs of
 // both CTAs have released it (empty barriers count two arrivals, each CTA's
 // MMA commit arrives on both).
+__device__ __forceinline__ void tma_load_4d_mc(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c2, int c3,
+                                               uint16_t mask)
+{
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster "
+        "[%0], [%1, {%3, %3, %4, %5}], [%2], %6;" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(0), "r"(c2), "r"(c3), "h"(mask)
+        : "memory");
+}
 __device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0, int c1,
                                                uint16_t mask)
 {
@@ -317,7 +330,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 ptx::mbar_arrive_expect_tx(fb, C::kStage);
                 const uint32_t sA = sbase + s * C::kStage;
                 ptx::tma_load_2d(sA, &mA, fb, i * kBK, (int)m0);
-                if constexpr (BWD) {
+                if constexpr (C::kBInterleaved) {
+                    // this CTA's four 8-row K groups (of eight) across all column
+                    // chunks, to the same offset in both CTAs
+                    tma_load_4d_mc(sA + C::kA + rank * 4 * C::kBChunks * 1024, &mB, fb, 0, i * 8 + (int)rank * 4, 0x3);
+                } else if constexpr (BWD) {
                     // this CTA's half of the 64 K rows of every column chunk, to
                     // the same offsets in both CTAs
                     for (int c = 0; c < C::kBChunks; ++c)
@@ -345,8 +362,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 for (int kk = 0; kk < kBK / 16; ++kk) {
                     // MN-major B: 16 K rows are two 8-row groups (2048 bytes);
                     // the column chunks are kChunkBytes apart
-                    const uint64_t bd = BWD ? ptx::smem_desc_sw128(sB + kk * 2048, C::kChunkBytes, 1024)
-                                            : ptx::smem_desc_sw128(sB + kk * 32, 16, 1024);
+                    const uint64_t bd =
+                        C::kBInterleaved
+                            ? ptx::smem_desc_sw128(sB + kk * 2048 * C::kBChunks, 1024, 1024 * C::kBChunks)
+                        : BWD ? ptx::smem_desc_sw128(sB + kk * 2048, C::kChunkBytes, 1024)
+                              : ptx::smem_desc_sw128(sB + kk * 32, 16, 1024);
                     ptx::mma_bf16(tmem, ptx::smem_desc_sw128(sA + kk * 32, 16, 1024), bd, idesc,
                                   (i > 0 || kk > 0) ? 1u : 0u);
                 }
