@@ -791,6 +791,30 @@ __global__ void __launch_bounds__(256) reduce_split_kernel(SplitJobs J)
     }
 }
 
+// Split-K sums (few partials, long outputs): thread q handles outputs
+// [4q, 4q + 4) of the concatenated jobs and adds the partials z = 0, 1, ... in
+// order -- deterministic, and the same association as reduce_split_kernel
+// for up to eight partials.  Every job length and partial stride is a
+// multiple of 4 and every pointer 16-byte aligned.
+__global__ void __launch_bounds__(256) reduce_split_vec4_kernel(SplitJobs J)
+{
+    const int64_t n4 = J.begin[J.njobs] / 4;
+    for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < n4; q += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t idx = q * 4;
+        int j = 0;
+        while (idx >= J.begin[j + 1]) ++j;
+        const int64_t i = idx - J.begin[j];
+        const float4 *p = reinterpret_cast<const float4 *>(J.part[j] + i);
+        const int64_t st4 = J.stride[j] / 4;
+        float4 s = __ldcs(p);
+        for (int z = 1; z < J.nparts; ++z) {
+            const float4 v = __ldcs(p + z * st4);
+            s.x += v.x, s.y += v.y, s.z += v.z, s.w += v.w;
+        }
+        *reinterpret_cast<float4 *>(J.out[j] + i) = s;
+    }
+}
+
 // Fused r-wide GEMM + CosNet launch (forward or backward), one tile per CTA.
 template <int R, bool BWD>
 noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const bf16 *A, int64_t K, const bf16 *B,
@@ -974,8 +998,16 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             const int64_t total = J.begin[J.njobs];
             const KernelInfo kr{"reduce_wgrad_split", kBoundHbm, (double)total * J.nparts,
                                 4.0 * total * (J.nparts + 1)};
+            bool vec4 = J.nparts <= 8;
+            for (int i = 0; i < J.njobs; ++i)
+                vec4 = vec4 && J.n[i] % 4 == 0 && J.stride[i] % 4 == 0 &&
+                       reinterpret_cast<uintptr_t>(J.out[i]) % 16 == 0 && reinterpret_cast<uintptr_t>(J.part[i]) % 16 == 0;
+            const int64_t blocks = std::min<int64_t>(ceil_div(total / 4, 256), 8 * (int64_t)num_sms());
             NOBLE_TRY(run(st, kr, [&] {
-                reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J);
+                if (vec4)
+                    reduce_split_vec4_kernel<<<(unsigned)blocks, 256, 0, st>>>(J);
+                else
+                    reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J);
             }));
         }
     }
