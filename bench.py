@@ -296,7 +296,34 @@ def main():
     ms_profiled = timed(lambda: step(bufs), args.steps)
     lib.noble_profile_enable(0)
     prof = binding.profile_read()
-    ms_plain = timed(lambda: step(plain_bufs, plain=True), args.steps)
+
+    # overhead against the plain (r = 0) layer of this library: NOBLE and
+    # plain runs alternate three times, medians compared (clock and thermal
+    # drift between two single runs is of the size of the effect)
+    reps_n, reps_p = [], []
+    for _ in range(3):
+        reps_n.append(timed(lambda: step(bufs), args.steps))
+        reps_p.append(timed(lambda: step(plain_bufs, plain=True), args.steps))
+    ms_noble_med, ms_plain = statistics.median(reps_n), statistics.median(reps_p)
+
+    # forward and backward passes timed apart
+    def fwd_only(bset, plain=False):
+        for d, b in zip(dev_inputs, bset):
+            binding.forward(b, d["x"], {k: d[k] for k in ("W", "bias")} if plain else d, stream)
+
+    def bwd_only(bset, plain=False):
+        for d, b in zip(dev_inputs, bset):
+            binding.backward(b, d["x"], d["dy"], {k: d[k] for k in ("W", "bias")} if plain else d, stream)
+
+    ms_fwd, ms_bwd = timed(lambda: fwd_only(bufs), args.steps), timed(lambda: bwd_only(bufs), args.steps)
+    # inference forward (NOBLE_FLAG_INFERENCE: h and b not saved)
+    inf_bufs = [binding.NobleLinearBuffers(l.T, l.d_in, l.d_out, l.r, l.dtype, with_grads=False,
+                                           flags=binding.NOBLE_FLAG_INFERENCE) for l in layers]
+    fwd_only(inf_bufs)
+    ms_fwd_inf = timed(lambda: fwd_only(inf_bufs), args.steps)
+    del inf_bufs
+    ms_fwd_p = timed(lambda: fwd_only(plain_bufs, True), args.steps)
+    ms_bwd_p = timed(lambda: bwd_only(plain_bufs, True), args.steps)
     binding.noble_get_device_status(None)
 
     ms_step = ms / args.steps
@@ -468,9 +495,15 @@ def main():
             "peak_src": pk["src"],
             "plain_ms_per_step": ms_plain / args.steps,
             "plain_tflops": world * flops_plain / (ms_plain / args.steps * 1e-3) / 1e12,
-            "overhead_vs_plain": ms_step / (ms_plain / args.steps) - 1.0,
+            "overhead_vs_plain": ms_noble_med / ms_plain - 1.0,
+            "overhead_method": "median of 3 alternating NOBLE / plain runs of the timed steps",
+            "fwd_ms_per_step": ms_fwd / args.steps, "bwd_ms_per_step": ms_bwd / args.steps,
+            "plain_fwd_ms_per_step": ms_fwd_p / args.steps, "plain_bwd_ms_per_step": ms_bwd_p / args.steps,
+            "overhead_fwd": ms_fwd / ms_fwd_p - 1.0, "overhead_bwd": ms_bwd / ms_bwd_p - 1.0,
+            "fwd_inference_ms_per_step": ms_fwd_inf / args.steps,
+            "overhead_fwd_inference": ms_fwd_inf / ms_fwd_p - 1.0,
             "cublas_plain_ms_per_step": ms_cublas,
-            "overhead_vs_cublas_plain": ms_step / ms_cublas - 1.0,
+            "overhead_vs_cublas_plain": ms_noble_med / args.steps / ms_cublas - 1.0,
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "per_layer": per_layer,
             "gpu_launches": launches,
             "profiled_ms_per_step": ms_profiled / args.steps,

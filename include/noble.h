@@ -80,6 +80,16 @@ typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
 #define NOBLE_FLAG_SIMT_ONLY 1u /* bf16: run every step on CUDA cores (fp32
                                    FMA), not tensor cores; a second path for
                                    cross-checking the tensor-core kernels */
+#define NOBLE_FLAG_INFERENCE 2u /* forward only, for inference (the branch
+                                   stays in the model at inference, the
+                                   Limitations section): on the
+                                   tensor-core path h and b are not written
+                                   and `saved` holds only c, the second K
+                                   segment of the output GEMM.  The backward
+                                   entry points reject such a descriptor
+                                   (NOBLE_ERR_INVALID_ARG).  The CUDA-core
+                                   paths (fp32, SIMT_ONLY) use the full saved
+                                   layout as scratch. */
 
 typedef struct {
     int64_t T;      /* tokens (rows of x)                          */
@@ -92,9 +102,10 @@ typedef struct {
 
 /*
  * Bytes of the saved-activation buffer that noble_linear_fwd writes and
- * noble_linear_bwd reads (per token: h and b in fp32, c in the operand dtype,
- * plus a copy of the mixing matrix).  0 when r == 0.  Returns 0 for an
- * invalid descriptor as well; the entry points then report why.
+ * noble_linear_bwd reads (per token: h and b in fp32, c in the operand dtype;
+ * only c with NOBLE_FLAG_INFERENCE on the tensor-core path).  0 when r == 0.
+ * Returns 0 for an invalid descriptor as well; the entry points then report
+ * why.
  */
 size_t noble_linear_saved_bytes(const noble_linear_desc *desc);
 

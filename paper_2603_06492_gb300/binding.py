@@ -20,6 +20,7 @@ LIB_PATH = os.path.join(HERE, "libnoble.so")
 HEADER = os.path.join(os.path.dirname(HERE), "include", "noble.h")
 
 NOBLE_BF16, NOBLE_FP32 = 0, 1
+NOBLE_FLAG_SIMT_ONLY, NOBLE_FLAG_INFERENCE = 1, 2
 STATUS = {0: "NOBLE_OK", 1: "NOBLE_ERR_INVALID_ARG", 2: "NOBLE_ERR_MISALIGNED",
           3: "NOBLE_ERR_UNSUPPORTED", 4: "NOBLE_ERR_BUFFER_TOO_SMALL", 5: "NOBLE_ERR_CUDA",
           6: "NOBLE_ERR_TIMEOUT", 7: "NOBLE_ERR_NO_DEVICE"}
@@ -36,10 +37,10 @@ class Desc(ctypes.Structure):
                 ("r", ctypes.c_int64), ("dtype", ctypes.c_int32), ("flags", ctypes.c_uint32)]
 
 
-def make_desc(T, d_in, d_out, r, dtype) -> Desc:
+def make_desc(T, d_in, d_out, r, dtype, flags=0) -> Desc:
     if isinstance(dtype, str):
         dtype = {"bf16": NOBLE_BF16, "fp32": NOBLE_FP32}[dtype]
-    return Desc(T, d_in, d_out, r, dtype, 0)
+    return Desc(T, d_in, d_out, r, dtype, flags)
 
 
 _lib = None
@@ -204,9 +205,9 @@ def _stream_handle(stream):
 class NobleLinearBuffers:
     """Caller-owned device buffers for one layer shape (allocated with torch)."""
 
-    def __init__(self, T, d_in, d_out, r, dtype, device="cuda", with_grads=True):
+    def __init__(self, T, d_in, d_out, r, dtype, device="cuda", with_grads=True, flags=0):
         import torch
-        self.desc = make_desc(T, d_in, d_out, r, dtype)
+        self.desc = make_desc(T, d_in, d_out, r, dtype, flags)
         tdt = torch.bfloat16 if self.desc.dtype == NOBLE_BF16 else torch.float32
         self.saved_bytes = noble_linear_saved_bytes(self.desc)
         self.workspace_bytes = noble_linear_bwd_workspace_bytes(self.desc)

@@ -70,6 +70,7 @@ noble_status run(cudaStream_t st, const KernelInfo &ki, F &&f)
     } while (0)
 
 constexpr uint32_t kFlagSimtOnly = NOBLE_FLAG_SIMT_ONLY;
+constexpr uint32_t kFlagInference = NOBLE_FLAG_INFERENCE;
 
 bool rank_supported(int64_t r) { return r == 0 || r == 16 || r == 32 || r == 64 || r == 128 || r == 256; }
 
@@ -88,7 +89,8 @@ noble_status validate_desc(const noble_linear_desc *d)
         return fail(NOBLE_ERR_UNSUPPORTED, "r=%lld not in {0,16,32,64,128,256}", (long long)d->r);
     if (d->dtype != NOBLE_BF16 && d->dtype != NOBLE_FP32)
         return fail(NOBLE_ERR_UNSUPPORTED, "dtype %d not supported", (int)d->dtype);
-    if (d->flags & ~kFlagSimtOnly) return fail(NOBLE_ERR_UNSUPPORTED, "unknown flags 0x%x", d->flags);
+    if (d->flags & ~(kFlagSimtOnly | kFlagInference))
+        return fail(NOBLE_ERR_UNSUPPORTED, "unknown flags 0x%x", d->flags);
     return NOBLE_OK;
 }
 
@@ -125,15 +127,23 @@ size_t esize(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 ? 2 : 4
 // True when the bf16 tensor-core path runs (the default for bf16 operands).
 bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->flags & kFlagSimtOnly); }
 
-// Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r].
+// Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r];
+// only c for an inference forward on the tensor-core path.
 struct SavedLayout {
     size_t h, b, c, total;
+    bool only_c;
 };
 SavedLayout saved_layout(const noble_linear_desc *d)
 {
     SavedLayout L{};
     if (d->r == 0 || d->T == 0) return L;
     const size_t tr = (size_t)d->T * (size_t)d->r;
+    if ((d->flags & kFlagInference) && use_tc(d)) {
+        L.only_c = true;
+        L.c = 0;
+        L.total = align_up(tr * esize(d), 256);
+        return L;
+    }
     L.h = 0;
     L.b = align_up(L.h + tr * 4, 256);
     L.c = align_up(L.b + tr * 4, 256);
@@ -872,7 +882,7 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     bf16 *c = (bf16 *)(saved + SL.c);
     tc::CosnetArgs a{};
     a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2, a.M = M;
-    a.h_out = h, a.b_out = b, a.c_out = c;
+    a.h_out = SL.only_c ? nullptr : h, a.b_out = SL.only_c ? nullptr : b, a.c_out = c;
     NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
         return cosnet_launch<decltype(bn)::value, false>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
     }));
@@ -1095,6 +1105,8 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, con
 {
     g_last_error[0] = 0;
     NOBLE_TRY(validate_desc(desc));
+    if (desc->flags & kFlagInference)
+        return fail(NOBLE_ERR_INVALID_ARG, "backward of an inference descriptor (NOBLE_FLAG_INFERENCE)");
     const bool br = desc->r > 0, empty = desc->T == 0;
     const char *names[] = {"dy", "x", "dx", "W", "dW", "workspace"};
     const void *req[] = {dy, x, dx, W, dW, workspace};
@@ -1208,6 +1220,8 @@ noble_status noble_linear_bwd_noalloc(const noble_linear_desc *desc, const void 
 {
     g_last_error[0] = 0;
     NOBLE_TRY(validate_desc(desc));
+    if (desc->flags & kFlagInference)
+        return fail(NOBLE_ERR_INVALID_ARG, "backward of an inference descriptor (NOBLE_FLAG_INFERENCE)");
     const size_t need = work_layout(desc).total;
     if (need > kNoallocScratchBytes)
         return fail(NOBLE_ERR_BUFFER_TOO_SMALL,

@@ -37,7 +37,7 @@ struct CosnetArgs {
     int kb;              // k-blocks of the main operand (d_in or d_out)
     const float *om1, *ph1, *om2, *ph2;
     const float *M;      // mixing matrix, fp32 [r][r] (b_j = sum_i a_i M[i][j])
-    // forward outputs
+    // forward outputs (h_out, b_out NULL: not saved, inference)
     float *h_out, *b_out;
     __nv_bfloat16 *c_out;
     // backward inputs / outputs
@@ -530,7 +530,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         for (int i = 0; i < W / 4; ++i)
 #pragma unroll
                             for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
-                        store_segments<W / 4>(w, args.h_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        if (args.h_out) store_segments<W / 4>(w, args.h_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
                     }
 #pragma unroll
                     for (int g = 0; g < W / 8; ++g) {
@@ -658,7 +658,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         for (int i = 0; i < W / 4; ++i)
 #pragma unroll
                             for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
-                        store_segments<W / 4>(w, args.b_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        if (args.b_out) store_segments<W / 4>(w, args.b_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
                     }
                     store_segments<W / 8>(wc, args.c_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                 } else {

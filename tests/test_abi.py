@@ -77,7 +77,7 @@ def test_bad_pointers_rejected(lib):
         _fwd(d, saved_bytes=16)
     assert e.value.status == 4
     bad = binding.make_desc(256, 128, 128, 16, "bf16")
-    bad.flags = 2  # unknown flag bit
+    bad.flags = 0x80  # unknown flag bit
     with pytest.raises(binding.NobleError) as e:
         _fwd(bad)
     assert e.value.status == 3
@@ -97,6 +97,32 @@ def test_branch_pointers_optional_without_rank(lib):
         _fwd(d, W_down=None, omega1=None, phi1=None, M=None, omega2=None, phi2=None,
              W_up=None, saved=None, saved_bytes=0)
     assert e.value.status == 7
+
+
+def test_inference_flag(lib):
+    # the tensor-core forward saves only c; the CUDA-core paths keep the full layout
+    T, r = 256, 16
+    full = binding.noble_linear_saved_bytes(binding.make_desc(T, 128, 128, r, "bf16"))
+    inf = binding.noble_linear_saved_bytes(
+        binding.make_desc(T, 128, 128, r, "bf16", binding.NOBLE_FLAG_INFERENCE))
+    assert inf == T * r * 2 and full >= T * r * (4 + 4 + 2)
+    simt = binding.make_desc(T, 128, 128, r, "bf16", binding.NOBLE_FLAG_INFERENCE | binding.NOBLE_FLAG_SIMT_ONLY)
+    assert binding.noble_linear_saved_bytes(simt) == full
+    f32 = binding.make_desc(T, 128, 128, r, "fp32", binding.NOBLE_FLAG_INFERENCE)
+    assert binding.noble_linear_saved_bytes(f32) == binding.noble_linear_saved_bytes(
+        binding.make_desc(T, 128, 128, r, "fp32"))
+    # the backward of an inference descriptor is rejected before anything runs
+    d = binding.make_desc(T, 128, 128, r, "bf16", binding.NOBLE_FLAG_INFERENCE)
+    kw = dict(dy=FAKE, x=FAKE, W=FAKE, W_down=FAKE, omega1=FAKE, phi1=FAKE, M=FAKE, omega2=FAKE,
+              phi2=FAKE, W_up=FAKE, saved=FAKE, saved_bytes=1 << 40, dx=FAKE, dW=FAKE, dbias=None,
+              dW_down=FAKE, dM=FAKE, domega1=FAKE, dphi1=FAKE, domega2=FAKE, dphi2=FAKE,
+              dW_up=FAKE, stream=None)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_linear_bwd(d, workspace=FAKE, workspace_bytes=1 << 40, **kw)
+    assert e.value.status == 1 and "inference" in str(e.value)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_linear_bwd_noalloc(d, **kw)
+    assert e.value.status == 1
 
 
 def test_bwd_workspace_size_checked(lib):

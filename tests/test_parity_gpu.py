@@ -190,3 +190,27 @@ def test_dbias_from_cosnet_kernel(d_out, r):
         torch.cuda.synchronize()
         got = buf.grads["dbias"].cpu().numpy().astype(np.float64)
         assert rel_err(got, ref) < 1e-5, rel_err(got, ref)
+
+
+@pytest.mark.parametrize("T,d_out", [(4096, 8192), (1000, 264)])
+def test_dbias_without_branch(T, d_out):
+    """r = 0: dbias (the all-ones operand's column of the weight-gradient
+    launch) against an fp64 column sum, and bit-identical over repeated
+    calls."""
+    import torch
+    layer = Layer("dbias0", T, 256, d_out, 0, "bf16")
+    inp = make_layer_inputs(layer, 37)
+    ref = inp["dy"].sum(axis=0)
+    dev = binding.params_to_device(inp, "bf16")
+    buf = binding.NobleLinearBuffers(T, 256, d_out, 0, "bf16")
+    binding.forward(buf, dev["x"], dev)
+    first = None
+    for _ in range(2):
+        buf.grads["dbias"].fill_(float("nan"))
+        binding.backward(buf, dev["x"], dev["dy"], dev)
+        torch.cuda.synchronize()
+        got = buf.grads["dbias"].cpu().numpy().astype(np.float64)
+        assert rel_err(got, ref) < 1e-5, rel_err(got, ref)
+        if first is None:
+            first = got
+        assert np.array_equal(first, got)
