@@ -90,6 +90,17 @@ typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
                                    (NOBLE_ERR_INVALID_ARG).  The CUDA-core
                                    paths (fp32, SIMT_ONLY) use the full saved
                                    layout as scratch. */
+#define NOBLE_FLAG_SIGMA_COS1 4u /* bottleneck sigma(h) = cos(omega1 h + phi1),
+                                    the single-cosine activation of the
+                                    ablation (Section 4.4, Table 5); M,
+                                    omega2, phi2 are not used (may be NULL)
+                                    and dM, domega2, dphi2 are written as 0 */
+#define NOBLE_FLAG_SIGMA_IDENTITY 8u /* bottleneck sigma(h) = h, the linear
+                                    collapse to x (W + W_down W_up)
+                                    (Sections 1 and 3.1); omega, phi and M are
+                                    not used (may be NULL) and their
+                                    gradients are written as 0.  Not together
+                                    with NOBLE_FLAG_SIGMA_COS1. */
 
 typedef struct {
     int64_t T;      /* tokens (rows of x)                          */

@@ -21,7 +21,8 @@
  *     u2 = omega2 * b + phi2
  *     c  = cos(u2)    = sigma(h)
  *
- * Two further sigma modes exist only to pin the oracle:
+ * Two further sigma modes pin the oracle and are the reference for the GPU's
+ * bottleneck variants of the same name:
  *   ORACLE_IDENTITY: sigma(h) = h, where the branch collapses to
  *                    x (W + W_down W_up)   (the LoRA remark in Section 1 and 3.1)
  *   ORACLE_COS1:     sigma(h) = cos(omega1 * h + phi1), the single-cosine

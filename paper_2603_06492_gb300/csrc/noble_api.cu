@@ -71,6 +71,15 @@ noble_status run(cudaStream_t st, const KernelInfo &ki, F &&f)
 
 constexpr uint32_t kFlagSimtOnly = NOBLE_FLAG_SIMT_ONLY;
 constexpr uint32_t kFlagInference = NOBLE_FLAG_INFERENCE;
+constexpr uint32_t kFlagSigmaCos1 = NOBLE_FLAG_SIGMA_COS1;
+constexpr uint32_t kFlagSigmaIdentity = NOBLE_FLAG_SIGMA_IDENTITY;
+
+// Bottleneck activation selected by the descriptor: 0 CosNet (Eq. 2), 1 single
+// cosine, 2 identity (the variants of the ablation, Section 4.4).
+int sigma_mode(const noble_linear_desc *d)
+{
+    return (d->flags & kFlagSigmaCos1) ? 1 : (d->flags & kFlagSigmaIdentity) ? 2 : 0;
+}
 
 bool rank_supported(int64_t r) { return r == 0 || r == 16 || r == 32 || r == 64 || r == 128 || r == 256; }
 
@@ -89,8 +98,10 @@ noble_status validate_desc(const noble_linear_desc *d)
         return fail(NOBLE_ERR_UNSUPPORTED, "r=%lld not in {0,16,32,64,128,256}", (long long)d->r);
     if (d->dtype != NOBLE_BF16 && d->dtype != NOBLE_FP32)
         return fail(NOBLE_ERR_UNSUPPORTED, "dtype %d not supported", (int)d->dtype);
-    if (d->flags & ~(kFlagSimtOnly | kFlagInference))
+    if (d->flags & ~(kFlagSimtOnly | kFlagInference | kFlagSigmaCos1 | kFlagSigmaIdentity))
         return fail(NOBLE_ERR_UNSUPPORTED, "unknown flags 0x%x", d->flags);
+    if ((d->flags & kFlagSigmaCos1) && (d->flags & kFlagSigmaIdentity))
+        return fail(NOBLE_ERR_INVALID_ARG, "NOBLE_FLAG_SIGMA_COS1 and NOBLE_FLAG_SIGMA_IDENTITY together");
     return NOBLE_OK;
 }
 
@@ -276,11 +287,20 @@ noble_status fwd_simt(const noble_linear_desc *d, const TIn *x, const TIn *W, co
         simt::Seg down{{x, di, 1}, {W_down, di, 1}, di};
         NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, down, nullptr, nullptr, h, r)));
         const int tpb = cosnet_tokens_per_block(r);
-        const KernelInfo ki{"simt_cosnet_fwd", kBoundAlu, 2.0 * T * r * r, 0.0};
-        NOBLE_TRY(run(st, ki, [&] {
-            simt::cosnet_fwd_rows<TIn><<<(unsigned)ceil_div(T, tpb), 256, tpb * r * sizeof(float), st>>>(
-                T, (int)r, tpb, h, om1, ph1, M, om2, ph2, b, c);
-        }));
+        const int sig = sigma_mode(d);
+        if (sig == 0) {
+            const KernelInfo ki{"simt_cosnet_fwd", kBoundAlu, 2.0 * T * r * r, 0.0};
+            NOBLE_TRY(run(st, ki, [&] {
+                simt::cosnet_fwd_rows<TIn><<<(unsigned)ceil_div(T, tpb), 256, tpb * r * sizeof(float), st>>>(
+                    T, (int)r, tpb, h, om1, ph1, M, om2, ph2, b, c);
+            }));
+        } else {
+            const KernelInfo ki{"simt_sigma_fwd", kBoundHbm, 0.0, (4.0 + sizeof(TIn)) * T * r};
+            NOBLE_TRY(run(st, ki, [&] {
+                simt::sigma_fwd_rows<TIn><<<(unsigned)std::min<int64_t>(ceil_div(T * r, 256), 4096), 256, 0, st>>>(
+                    T * r, (int)r, sig, h, om1, ph1, c);
+            }));
+        }
         simt::Seg up{{c, r, 1}, {W_up, r, 1}, r};
         return simt_gemm<TIn, TIn>(st, T, dout, main, &up, bias, y, dout);
     }
@@ -304,25 +324,40 @@ noble_status bwd_simt(const noble_linear_desc *d, const TIn *dy, const TIn *x, c
         float *dc = (float *)(ws + WL.dc), *a = (float *)(ws + WL.a), *db = (float *)(ws + WL.db);
         float *Mt = (float *)(ws + WL.mt), *cpart = (float *)(ws + WL.cos_part);
         float *dmpart = (float *)(ws + WL.dm_part);
-        const KernelInfo kt{"transpose_M", kBoundHbm, 0.0, 8.0 * r * r};
-        NOBLE_TRY(run(st, kt, [&] {
-            simt::transpose_square<<<(unsigned)ceil_div(r * r, 256), 256, 0, st>>>((int)r, M, Mt);
-        }));
+        const int sig = sigma_mode(d);
+        if (sig == 0) {
+            const KernelInfo kt{"transpose_M", kBoundHbm, 0.0, 8.0 * r * r};
+            NOBLE_TRY(run(st, kt, [&] {
+                simt::transpose_square<<<(unsigned)ceil_div(r * r, 256), 256, 0, st>>>((int)r, M, Mt);
+            }));
+        }
         // dc = dy W_up
         simt::Seg sdc{{dy, dout, 1}, {W_up, 1, r}, dout};
         NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, sdc, nullptr, nullptr, dc, r)));
         const int tpb = cosnet_tokens_per_block(r);
-        const KernelInfo kc{"simt_cosnet_bwd", kBoundAlu, 2.0 * T * r * r, 0.0};
-        NOBLE_TRY(run(st, kc, [&] {
-            simt::cosnet_bwd_rows<TIn><<<(unsigned)WL.n_cos_blocks, 256, 5 * tpb * r * sizeof(float), st>>>(
-                T, (int)r, tpb, h, b, dc, om1, ph1, Mt, om2, ph2, dh, a, db, cpart);
-        }));
+        if (sig == 0) {
+            const KernelInfo kc{"simt_cosnet_bwd", kBoundAlu, 2.0 * T * r * r, 0.0};
+            NOBLE_TRY(run(st, kc, [&] {
+                simt::cosnet_bwd_rows<TIn><<<(unsigned)WL.n_cos_blocks, 256, 5 * tpb * r * sizeof(float), st>>>(
+                    T, (int)r, tpb, h, b, dc, om1, ph1, Mt, om2, ph2, dh, a, db, cpart);
+            }));
+        } else {
+            const KernelInfo kc{"simt_sigma_bwd", kBoundHbm, 0.0, (12.0 + sizeof(TIn)) * T * r};
+            NOBLE_TRY(run(st, kc, [&] {
+                simt::sigma_bwd_rows<TIn><<<(unsigned)WL.n_cos_blocks, 256, 0, st>>>(T, (int)r, sig, tpb, h, dc,
+                                                                                    om1, ph1, dh, cpart);
+            }));
+        }
         NOBLE_TRY(reduce(st, WL.n_cos_blocks, 4 * r, r, cpart, dom1, dph1, dom2, dph2));
-        // dM = a^T db, fixed token chunks
-        simt::Seg sdm{{a, 1, r}, {db, 1, r}, T};
-        NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
-                                           WL.n_dm_chunks, r * r)));
-        NOBLE_TRY(reduce(st, WL.n_dm_chunks, r * r, r * r, dmpart, dM));
+        if (sig == 0) {
+            // dM = a^T db, fixed token chunks
+            simt::Seg sdm{{a, 1, r}, {db, 1, r}, T};
+            NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
+                                               WL.n_dm_chunks, r * r)));
+            NOBLE_TRY(reduce(st, WL.n_dm_chunks, r * r, r * r, dmpart, dM));
+        } else if (cudaMemsetAsync(dM, 0, (size_t)r * r * 4, st) != cudaSuccess) {
+            return fail(NOBLE_ERR_CUDA, "dM: %s", cudaGetErrorString(cudaGetLastError()));
+        }
         // dW_up = dy^T c ; dW_down = dh^T x
         simt::Seg sup{{dy, 1, dout}, {c, 1, r}, T};
         NOBLE_TRY((simt_gemm<TIn, float>(st, dout, r, sup, nullptr, nullptr, dW_up, r)));
@@ -826,7 +861,7 @@ __global__ void __launch_bounds__(256) reduce_split_vec4_kernel(SplitJobs J)
 }
 
 // Fused r-wide GEMM + CosNet launch (forward or backward), one tile per CTA.
-template <int R, bool BWD>
+template <int R, bool BWD, int SIG>
 noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const bf16 *A, int64_t K, const bf16 *B,
                            const tc::CosnetArgs &args_in)
 {
@@ -843,7 +878,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     args.T = T;
     args.kb = (int)ceil_div(K, tc::kBK);
     args.status = status_ptr();
-    auto kern = tc::cosnet_gemm_kernel<R, BWD>;
+    auto kern = tc::cosnet_gemm_kernel<R, BWD, SIG>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kDynamic) != cudaSuccess)
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
     const KernelInfo ki{name, kBoundHbm, 2.0 * T * R * (K + R), 2.0 * T * K + 2.0 * R * K + (BWD ? 14.0 : 10.0) * T * R};
@@ -884,7 +919,12 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2, a.M = M;
     a.h_out = SL.only_c ? nullptr : h, a.b_out = SL.only_c ? nullptr : b, a.c_out = c;
     NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-        return cosnet_launch<decltype(bn)::value, false>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
+        constexpr int R = decltype(bn)::value;
+        switch (sigma_mode(d)) {
+        case 1: return cosnet_launch<R, false, tc::kSigCos1>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
+        case 2: return cosnet_launch<R, false, tc::kSigIdentity>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
+        default: return cosnet_launch<R, false, tc::kSigCosnet>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
+        }
     }));
     const TcSeg up{c, W_up, r};
     const ProbSpec P{T, dout, main, &up, 256};
@@ -914,7 +954,12 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         ca.bias_part = dbias ? bpart : nullptr;
         ca.kdim = dout;
         NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
-            return cosnet_launch<decltype(bn)::value, true>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
+            constexpr int R = decltype(bn)::value;
+            switch (sigma_mode(d)) {
+            case 1: return cosnet_launch<R, true, tc::kSigCos1>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
+            case 2: return cosnet_launch<R, true, tc::kSigIdentity>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
+            default: return cosnet_launch<R, true, tc::kSigCosnet>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
+            }
         }));
         // domega1, dphi1, domega2, dphi2 (and dbias) from the per-CTA partials
         SplitJobs J{};
@@ -975,7 +1020,10 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         if (r > 0) {
             add(1, ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256}, dW_down, di, false);
             add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false);
-            add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);
+            if (sigma_mode(d) == 0)
+                add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);
+            else if (cudaMemsetAsync(dM, 0, (size_t)r * r * 4, st) != cudaSuccess)
+                return fail(NOBLE_ERR_CUDA, "dM: %s", cudaGetErrorString(cudaGetLastError()));
         }
         if (ones_dbias) add(4, ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128}, dbias, 1, true);
         const int split = WL.split;
@@ -1069,12 +1117,14 @@ noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, cons
     NOBLE_TRY(check_ptr(W, "W", false));
     NOBLE_TRY(check_ptr(bias, "bias", true));
     NOBLE_TRY(check_ptr(y, "y", empty));
+    // parameters the bottleneck variant does not use may be NULL
+    const int sig = sigma_mode(desc);
     NOBLE_TRY(check_ptr(W_down, "W_down", !br));
-    NOBLE_TRY(check_ptr(omega1, "omega1", !br));
-    NOBLE_TRY(check_ptr(phi1, "phi1", !br));
-    NOBLE_TRY(check_ptr(M, "M", !br));
-    NOBLE_TRY(check_ptr(omega2, "omega2", !br));
-    NOBLE_TRY(check_ptr(phi2, "phi2", !br));
+    NOBLE_TRY(check_ptr(omega1, "omega1", !br || sig == 2));
+    NOBLE_TRY(check_ptr(phi1, "phi1", !br || sig == 2));
+    NOBLE_TRY(check_ptr(M, "M", !br || sig != 0));
+    NOBLE_TRY(check_ptr(omega2, "omega2", !br || sig != 0));
+    NOBLE_TRY(check_ptr(phi2, "phi2", !br || sig != 0));
     NOBLE_TRY(check_ptr(W_up, "W_up", !br));
     NOBLE_TRY(check_ptr(saved, "saved", !br || empty));
     if (saved_bytes < saved_layout(desc).total)
@@ -1116,7 +1166,11 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, con
                             "dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2", "dW_up"};
     const void *bptr[] = {W_down, omega1, phi1, M, omega2, phi2, W_up, saved,
                           dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up};
-    for (int i = 0; i < 15; ++i) NOBLE_TRY(check_ptr(bptr[i], bnames[i], !br || (empty && i == 7)));
+    const int sig = sigma_mode(desc);
+    // inputs the bottleneck variant does not use may be NULL; every gradient
+    // output is written (zeros for unused parameters)
+    auto unused = [&](int i) { return (sig == 2 && i >= 1 && i <= 5) || (sig == 1 && i >= 3 && i <= 5); };
+    for (int i = 0; i < 15; ++i) NOBLE_TRY(check_ptr(bptr[i], bnames[i], !br || (empty && i == 7) || unused(i)));
     if (saved_bytes < saved_layout(desc).total)
         return fail(NOBLE_ERR_BUFFER_TOO_SMALL, "saved_bytes=%zu < %zu", saved_bytes, saved_layout(desc).total);
     if (workspace_bytes < work_layout(desc).total)

@@ -130,6 +130,53 @@ cosnet_fwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const fl
     }
 }
 
+// Single-cosine (mode 1) or identity (mode 2) bottleneck on rows, the
+// variants of the ablation (Section 4.4): c = cos(omega1 h + phi1) or c = h,
+// elementwise over h [T][r] (n = T r elements).
+template <typename TOut>
+__global__ void __launch_bounds__(256)
+sigma_fwd_rows(int64_t n, int r, int mode, const float *h, const float *om1, const float *ph1, TOut *c_out)
+{
+    for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < n; idx += (int64_t)gridDim.x * blockDim.x) {
+        const int i = (int)(idx % r);
+        const float v = h[idx];
+        Elem<TOut>::store(c_out + idx, mode == 1 ? cosf(fmaf(om1[i], v, ph1[i])) : v);
+    }
+}
+
+// Backward of sigma_fwd_rows: mode 1: du1 = -sin(omega1 h + phi1) dc,
+// dh = omega1 du1; mode 2: dh = dc.  Per-block column sums over the block's
+// tokens in ascending order: part[blk][0:r] = sum du1*h, [r:2r] = sum du1,
+// [2r:4r] = 0 (no second layer).
+template <typename TOut>
+__global__ void __launch_bounds__(256)
+sigma_bwd_rows(int64_t T, int r, int mode, int tokens_per_block, const float *h, const float *dc,
+               const float *om1, const float *ph1, TOut *dh_out, float *part)
+{
+    const int64_t t0 = (int64_t)blockIdx.x * tokens_per_block;
+    const int64_t t1 = min(T, t0 + tokens_per_block);
+    float *pb = part + (int64_t)blockIdx.x * 4 * r;
+    for (int j = threadIdx.x; j < r; j += blockDim.x) {
+        float so = 0.f, sp = 0.f;
+        for (int64_t t = t0; t < t1; ++t) {
+            const float d = dc[t * r + j];
+            if (mode == 1) {
+                const float hv = h[t * r + j];
+                const float du1 = -sinf(fmaf(om1[j], hv, ph1[j])) * d;
+                Elem<TOut>::store(dh_out + t * r + j, om1[j] * du1);
+                so += du1 * hv;
+                sp += du1;
+            } else {
+                Elem<TOut>::store(dh_out + t * r + j, d);
+            }
+        }
+        pb[j] = so;
+        pb[r + j] = sp;
+        pb[2 * r + j] = 0.f;
+        pb[3 * r + j] = 0.f;
+    }
+}
+
 // CosNet backward on rows (chain rule through Eq. 2).  From saved h, b (fp32),
 // dc = dy W_up (fp32) and Mt = M^T computes per token
 //   du2 = -sin(u2) dc, db = omega2 du2, da = db M^T, du1 = -sin(u1) da,

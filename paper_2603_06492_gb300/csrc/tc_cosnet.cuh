@@ -261,7 +261,14 @@ __device__ __forceinline__ uint32_t cta_rank_in_cluster()
     return r;
 }
 
-template <int R, bool BWD>
+// Bottleneck activation of the kernel: the CosNet of Eq. 2 (default), or two
+// variants of the ablation in Section 4.4 (Table 5): a single cosine
+// sigma(h) = cos(omega1 h + phi1), and the identity sigma(h) = h (the linear
+// collapse of Sections 1 and 3.1).  The variants have no mixing matrix, so
+// their epilogue ends after the first accumulator.
+constexpr int kSigCosnet = 0, kSigCos1 = 1, kSigIdentity = 2;
+
+template <int R, bool BWD, int SIG = kSigCosnet>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kCosnetThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const CosnetArgs args)
@@ -307,10 +314,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ptx::tmem_relinquish();
     }
     for (int i = threadIdx.x; i < R; i += blockDim.x) {
-        prm[i] = args.om1[i];
-        prm[R + i] = args.ph1[i];
-        prm[2 * R + i] = args.om2[i];
-        prm[3 * R + i] = args.ph2[i];
+        // parameters a variant does not use may be NULL
+        prm[i] = args.om1 ? args.om1[i] : 0.f;
+        prm[R + i] = args.ph1 ? args.ph1[i] : 0.f;
+        prm[2 * R + i] = args.om2 ? args.om2[i] : 0.f;
+        prm[3 * R + i] = args.ph2 ? args.ph2[i] : 0.f;
     }
     ptx::tc_fence_before();
     __syncthreads();
@@ -445,7 +453,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
         };
         // the first pass's part of M is read while the main loop runs
-        m_load(0);
+        if constexpr (SIG == kSigCosnet) m_load(0);
         if constexpr (BWD) {
             // the tile's saved h and b rows are read after the main loop: bring
             // them into L2 meanwhile
@@ -507,8 +515,96 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ok = ptx::named_barrier_and(3, 256, ok);  // uniform over the epilogue warps
         if (ok) {
             // the ring is free once the main accumulator is complete
-            m_store(0);
+            if constexpr (SIG == kSigCosnet) m_store(0);
             ptx::tc_fence_after();
+            if constexpr (SIG != kSigCosnet) {
+                // single-cosine or identity bottleneck: c (forward) or dh
+                // (backward) straight from the first accumulator
+#pragma unroll 1
+                for (int c = 32 * half; c < R; c += 64) {
+                    float v[32];
+                    if constexpr (R >= 32) {
+                        ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
+                    } else {
+                        float w[16];
+                        ptx::tmem_ld_32x32b_x16(lane_addr + c, w);
+#pragma unroll
+                        for (int i = 0; i < 16; ++i) v[i] = w[i], v[i + 16] = 0.f;
+                    }
+                    constexpr int W = R < 32 ? R : 32;
+                    if constexpr (!BWD) {
+                        // v = h: store h and c = cos(omega1 h + phi1) or c = h
+                        {
+                            uint32_t w[W / 4][4];
+#pragma unroll
+                            for (int i = 0; i < W / 4; ++i)
+#pragma unroll
+                                for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
+                            if (args.h_out)
+                                store_segments<W / 4>(w, args.h_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        }
+                        uint32_t wc[W / 8][4];
+#pragma unroll
+                        for (int g = 0; g < W / 8; ++g) {
+                            float cc[8];
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const int k = c + 8 * g + i;
+                                cc[i] = SIG == kSigCos1 ? cos_reduced(fmaf(om1[k], v[8 * g + i], ph1[k])) : v[8 * g + i];
+                            }
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) wc[g][q] = ptx::pack_bf16x2(cc[2 * q], cc[2 * q + 1]);
+                        }
+                        store_segments<W / 8>(wc, args.c_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                    } else {
+                        // v = dc; single cosine: du1 = -sin(omega1 h + phi1) dc,
+                        // dh = omega1 du1; identity: dh = dc
+                        float hv[32];
+#pragma unroll
+                        for (int i = 0; i < 32; ++i) hv[i] = 0.f;
+                        if constexpr (SIG == kSigCos1) {
+                            uint32_t w[W / 4][4];
+                            load_segments<W / 4>(w, args.h_in + t0 * R + c, (int64_t)R * 4, t0, args.T);
+#pragma unroll
+                            for (int i = 0; i < W / 4; ++i)
+#pragma unroll
+                                for (int q = 0; q < 4; ++q) hv[4 * i + q] = __uint_as_float(w[i][q]);
+                        }
+                        float q0[32], q1[32];
+                        uint32_t wdh[W / 8][4];
+#pragma unroll
+                        for (int i = W; i < 32; ++i) q0[i] = 0.f, q1[i] = 0.f;
+#pragma unroll
+                        for (int g = 0; g < W / 8; ++g) {
+                            float dh[8];
+#pragma unroll
+                            for (int i = 0; i < 8; ++i) {
+                                const int k = c + 8 * g + i, j = 8 * g + i;
+                                float du1 = 0.f;
+                                if constexpr (SIG == kSigCos1) {
+                                    du1 = live ? -sin_reduced(fmaf(om1[k], hv[j], ph1[k])) * v[j] : 0.f;
+                                    dh[i] = om1[k] * du1;
+                                } else {
+                                    dh[i] = live ? v[j] : 0.f;
+                                }
+                                q0[j] = du1 * hv[j];
+                                q1[j] = du1;
+                            }
+#pragma unroll
+                            for (int q = 0; q < 4; ++q) wdh[g][q] = ptx::pack_bf16x2(dh[2 * q], dh[2 * q + 1]);
+                        }
+                        store_segments<W / 8>(wdh, args.dh_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                        const float s0 = warp_colsum32(q0);
+                        const float s1 = warp_colsum32(q1);
+                        if (c + lane < R) {
+                            cpart[(quarter * 4 + 0) * R + c + lane] = s0;
+                            cpart[(quarter * 4 + 1) * R + c + lane] = s1;
+                            cpart[(quarter * 4 + 2) * R + c + lane] = 0.f;  // no second layer
+                            cpart[(quarter * 4 + 3) * R + c + lane] = 0.f;
+                        }
+                    }
+                }
+            } else {
             // ---- phase 1: first accumulator -> bf16 operand tile (+ outputs)
 #pragma unroll 1
             for (int c = 32 * half; c < R; c += 64) {
@@ -625,12 +721,13 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             if (threadIdx.x == 64) ptx::mma_commit(mma2_done);
             const bool done = ptx::mbar_wait(mma2_done, 0, args.status);
             ok = ptx::named_barrier_and(3, 256, ok && done);
+            }  // SIG == kSigCosnet
         }
         if (ok) {
             ptx::tc_fence_after();
             // ---- phase 2: second accumulator
 #pragma unroll 1
-            for (int c = 32 * half; c < R; c += 64) {
+            for (int c = 32 * half; SIG == kSigCosnet && c < R; c += 64) {
                 float v[32];
                 if constexpr (R >= 32) {
                     ptx::tmem_ld_32x32b_x32(acc2 + c, v);
