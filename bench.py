@@ -201,6 +201,8 @@ def main():
     ap.add_argument("--layers", default="", help="comma-separated layer names (default: all)")
     ap.add_argument("--config", type=int, default=CONFIG_INDEX,
                     help="workload: configuration 0-4 (default 3, the headline)")
+    ap.add_argument("--sigma", default="cosnet", choices=["cosnet", "cos1", "identity"],
+                    help="bottleneck activation (cos1, identity: the variants of the ablation)")
     ap.add_argument("--per-layer", action="store_true",
                     help="also time every layer alone (NOBLE and plain) and report each")
     args = ap.parse_args()
@@ -238,7 +240,10 @@ def main():
         inp = make_layer_inputs(layer, layer_seed(cfg, li))
         dev_inputs.append(binding.params_to_device(inp, layer.dtype))
         del inp
-        bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype))
+        sig_flags = {"cosnet": 0, "cos1": binding.NOBLE_FLAG_SIGMA_COS1,
+                     "identity": binding.NOBLE_FLAG_SIGMA_IDENTITY}[args.sigma]
+        bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype,
+                                               flags=sig_flags))
         plain_bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, 0, layer.dtype))
     flops_step = sum(l.flops() for l in layers)
     flops_plain = sum(l.plain().flops() for l in layers)
@@ -318,7 +323,8 @@ def main():
     ms_fwd, ms_bwd = timed(lambda: fwd_only(bufs), args.steps), timed(lambda: bwd_only(bufs), args.steps)
     # inference forward (NOBLE_FLAG_INFERENCE: h and b not saved)
     inf_bufs = [binding.NobleLinearBuffers(l.T, l.d_in, l.d_out, l.r, l.dtype, with_grads=False,
-                                           flags=binding.NOBLE_FLAG_INFERENCE) for l in layers]
+                                           flags=binding.NOBLE_FLAG_INFERENCE | b.desc.flags)
+                for l, b in zip(layers, bufs)]
     fwd_only(inf_bufs)
     ms_fwd_inf = timed(lambda: fwd_only(inf_bufs), args.steps)
     del inf_bufs
@@ -486,7 +492,7 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if layers[0].dtype == "bf16" else "f32",
             "data": "synthetic",
-            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "layers": [
+            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "sigma": args.sigma, "layers": [
                 {"name": l.name, "T": l.T, "d_in": l.d_in, "d_out": l.d_out, "r": l.r} for l in layers],
                 "l2": "inputs larger than L2: each step streams ~1.8 GB of activations",
                 "parallelism": f"replicas x{world}"},
