@@ -491,6 +491,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                             s0 += f.x;
                             s1 += f.y;
                         }
+                        // the stage is refilled by the copy engine (async proxy)
+                        // once released: order these generic reads before that
+                        ptx::fence_proxy_async_smem();
                         __syncwarp();
                         if (lane == 0) ptx::mbar_arrive(empty_bar(s));
                     }

@@ -175,8 +175,9 @@ def test_launch_counter_advances():
 def test_dbias_from_cosnet_kernel(d_out, r):
     """dbias is summed from the dy tiles streamed by the CosNet backward
     kernel; check it against an fp64 column sum on shapes with many k-blocks
-    per tile, three times in a row (the sums race with the ring reuse that
-    follows the main loop if its ordering is wrong)."""
+    per tile, eight times in a row (the sums race with the ring reuse that
+    follows the main loop, or with the refill of a stage by the copy engine,
+    if their ordering is wrong)."""
     import torch
     layer = Layer("dbias", 4096, 256, d_out, r, "bf16")
     inp = make_layer_inputs(layer, 31)
@@ -184,7 +185,7 @@ def test_dbias_from_cosnet_kernel(d_out, r):
     dev = binding.params_to_device(inp, "bf16")
     buf = binding.NobleLinearBuffers(4096, 256, d_out, r, "bf16")
     binding.forward(buf, dev["x"], dev)
-    for _ in range(3):
+    for _ in range(8):
         buf.grads["dbias"].fill_(float("nan"))
         binding.backward(buf, dev["x"], dev["dy"], dev)
         torch.cuda.synchronize()
