@@ -173,6 +173,53 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy,
                               noble_stream stream);
 
 /*
+ * Optimizer step: AdamW with decoupled weight decay (the optimizer of the
+ * paper's training runs, Section 4.1: beta1 0.9, beta2 0.98, weight decay
+ * 0.01) over a batch of parameter tensors, each with its own learning rate,
+ * in one fused pass per 16 tensors.  For step t >= 1, elementwise with the
+ * tensor's learning rate a = lr * lr_mult:
+ *     p <- p - a * weight_decay * p             (only if `decay`)
+ *     m <- beta1 m + (1 - beta1) g,   v <- beta2 v + (1 - beta2) g^2
+ *     p <- p - a / (1 - beta1^t) * m / (sqrt(v) / sqrt(1 - beta2^t) + eps)
+ * All arrays are device memory, fp32, `n` elements, updated in place (g is
+ * read only).  `param_bf16` (optional) receives the new values rounded to
+ * bf16, e.g. the operand copy of W, W_down or W_up the layer's kernels read.
+ * Pointers must be 16-byte aligned (param_bf16 8-byte aligned).
+ * Errors: NOBLE_ERR_INVALID_ARG for NULL pointers, n < 0, t < 1 or bad
+ * hyperparameters; NOBLE_ERR_MISALIGNED.  Nothing is enqueued on error.
+ */
+typedef struct {
+    float *param;
+    void *param_bf16; /* optional */
+    const float *grad;
+    float *exp_avg;
+    float *exp_avg_sq;
+    int64_t n;
+    float lr_mult;
+    int32_t decay; /* 1: apply weight decay to this tensor */
+} noble_adamw_tensor;
+
+typedef struct {
+    float lr, beta1, beta2, eps, weight_decay;
+    int64_t step; /* t, counted from 1 */
+} noble_adamw_hparams;
+
+noble_status noble_adamw_step(const noble_adamw_tensor *tensors, int n_tensors,
+                              const noble_adamw_hparams *hp, noble_stream stream);
+
+/*
+ * NOBLE's per-group learning-rate multipliers (Section 3.3 and the defaults of
+ * Appendix A), with rho = min(d_in, d_out) / r:
+ *   out[0] W, bias, W_down: 1      out[1] W_up: rho^(2 gamma)
+ *   out[2] M: rho^gamma_M          out[3] omega1, omega2: omega_mult
+ *   out[4] phi1, phi2: phi_mult
+ * Paper defaults: gamma 0.3, gamma_M 0.45, omega_mult 3, phi_mult 5.
+ * Host only.  NOBLE_ERR_INVALID_ARG for r == 0 or a NULL pointer.
+ */
+noble_status noble_linear_lr_multipliers(const noble_linear_desc *desc, float gamma, float gamma_M,
+                                         float omega_mult, float phi_mult, float out[5]);
+
+/*
  * Backward pass without a caller workspace, for callers that cannot allocate
  * device memory: code that runs inside a host framework or plugin which owns
  * every device allocation and hands its extensions no allocator, or a

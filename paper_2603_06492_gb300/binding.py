@@ -38,6 +38,17 @@ class Desc(ctypes.Structure):
                 ("r", ctypes.c_int64), ("dtype", ctypes.c_int32), ("flags", ctypes.c_uint32)]
 
 
+class AdamwTensor(ctypes.Structure):
+    _fields_ = [("param", ctypes.c_void_p), ("param_bf16", ctypes.c_void_p), ("grad", ctypes.c_void_p),
+                ("exp_avg", ctypes.c_void_p), ("exp_avg_sq", ctypes.c_void_p), ("n", ctypes.c_int64),
+                ("lr_mult", ctypes.c_float), ("decay", ctypes.c_int32)]
+
+
+class AdamwHparams(ctypes.Structure):
+    _fields_ = [("lr", ctypes.c_float), ("beta1", ctypes.c_float), ("beta2", ctypes.c_float),
+                ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("step", ctypes.c_int64)]
+
+
 def make_desc(T, d_in, d_out, r, dtype, flags=0) -> Desc:
     if isinstance(dtype, str):
         dtype = {"bf16": NOBLE_BF16, "fp32": NOBLE_FP32}[dtype]
@@ -97,6 +108,11 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.noble_profile_count.restype = ctypes.c_int
         lib.noble_profile_entry.argtypes = [ctypes.c_int, ctypes.c_char_p, ctypes.c_size_t] + [P] * 5
         lib.noble_profile_entry.restype = ctypes.c_int
+        lib.noble_adamw_step.argtypes = [ctypes.POINTER(AdamwTensor), ctypes.c_int,
+                                         ctypes.POINTER(AdamwHparams), P]
+        lib.noble_adamw_step.restype = ctypes.c_int
+        lib.noble_linear_lr_multipliers.argtypes = [D] + [ctypes.c_float] * 4 + [ctypes.POINTER(ctypes.c_float)]
+        lib.noble_linear_lr_multipliers.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -161,6 +177,27 @@ def noble_linear_bwd_noalloc(desc, dy, x, W, W_down, omega1, phi1, M, omega2, ph
 
 
 NOALLOC_SCRATCH_BYTES = 64 << 20
+
+
+def noble_adamw_step(tensors, lr, beta1=0.9, beta2=0.98, eps=1e-8, weight_decay=0.01, step=1,
+                     stream=None):
+    """One fused AdamW step.  ``tensors``: dicts with param, grad, exp_avg,
+    exp_avg_sq (fp32 device tensors or pointers), optional param_bf16,
+    lr_mult (default 1) and decay (default True)."""
+    arr = (AdamwTensor * max(1, len(tensors)))()
+    for i, t in enumerate(tensors):
+        n = t["n"] if "n" in t else t["param"].numel()
+        arr[i] = AdamwTensor(_p(t["param"]), _p(t.get("param_bf16")), _p(t["grad"]), _p(t["exp_avg"]),
+                             _p(t["exp_avg_sq"]), n, float(t.get("lr_mult", 1.0)), int(t.get("decay", True)))
+    hp = AdamwHparams(lr, beta1, beta2, eps, weight_decay, step)
+    _check(load().noble_adamw_step(arr, len(tensors), ctypes.byref(hp), stream))
+
+
+def noble_linear_lr_multipliers(desc, gamma=0.3, gamma_M=0.45, omega_mult=3.0, phi_mult=5.0):
+    """Per-group learning-rate multipliers [W|bias|W_down, W_up, M, omega, phi]."""
+    out = (ctypes.c_float * 5)()
+    _check(load().noble_linear_lr_multipliers(ctypes.byref(desc), gamma, gamma_M, omega_mult, phi_mult, out))
+    return list(out)
 
 
 def noble_get_device_status(stream=None):

@@ -4,6 +4,7 @@
 // Forward = Eq. 1 (Section 3.1) with CosNet (Eq. 2, Section 3.2; Eqs. 5-7,
 // Appendix A); backward = the chain rule through the same definitions.
 #include <algorithm>
+#include <cmath>
 #include <atomic>
 #include <vector>
 #include <mutex>
@@ -17,6 +18,7 @@
 #include "common.cuh"
 #include "profile.cuh"
 #include "simt.cuh"
+#include "adamw.cuh"
 #include "tc_gemm.cuh"
 #include "tc_persistent.cuh"
 #include "tc_cosnet.cuh"
@@ -1288,6 +1290,72 @@ noble_status noble_linear_bwd_noalloc(const noble_linear_desc *desc, const void 
     return noble_linear_bwd(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up, saved, saved_bytes, dx,
                             dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, scratch,
                             kNoallocScratchBytes, stream);
+}
+
+noble_status noble_adamw_step(const noble_adamw_tensor *tensors, int n_tensors, const noble_adamw_hparams *hp,
+                              noble_stream stream)
+{
+    g_last_error[0] = 0;
+    if (n_tensors < 0 || (n_tensors > 0 && !tensors) || !hp) return fail(NOBLE_ERR_INVALID_ARG, "tensors / hparams");
+    if (hp->step < 1 || !(hp->lr >= 0.f) || !(hp->beta1 >= 0.f && hp->beta1 < 1.f) ||
+        !(hp->beta2 >= 0.f && hp->beta2 < 1.f) || !(hp->eps > 0.f) || !(hp->weight_decay >= 0.f))
+        return fail(NOBLE_ERR_INVALID_ARG, "hyperparameters (step %lld)", (long long)hp->step);
+    for (int i = 0; i < n_tensors; ++i) {
+        const noble_adamw_tensor &t = tensors[i];
+        if (t.n < 0 || !(t.lr_mult >= 0.f)) return fail(NOBLE_ERR_INVALID_ARG, "tensor %d: n or lr_mult", i);
+        const bool empty = t.n == 0;
+        NOBLE_TRY(check_ptr(t.param, "param", empty));
+        NOBLE_TRY(check_ptr(t.grad, "grad", empty));
+        NOBLE_TRY(check_ptr(t.exp_avg, "exp_avg", empty));
+        NOBLE_TRY(check_ptr(t.exp_avg_sq, "exp_avg_sq", empty));
+        if (reinterpret_cast<uintptr_t>(t.param_bf16) % 8)
+            return fail(NOBLE_ERR_MISALIGNED, "tensor %d: param_bf16 is not 8-byte aligned", i);
+    }
+    if (n_tensors == 0) return NOBLE_OK;
+    NOBLE_TRY(check_device());
+    cudaStream_t st = (cudaStream_t)stream;
+    const double bc1 = 1.0 - std::pow((double)hp->beta1, (double)hp->step);
+    const double bc2 = 1.0 - std::pow((double)hp->beta2, (double)hp->step);
+    for (int i0 = 0; i0 < n_tensors; i0 += opt::kAdamwMaxTensors) {
+        const int nt = std::min(opt::kAdamwMaxTensors, n_tensors - i0);
+        opt::AdamwBatch b{};
+        b.beta1 = hp->beta1, b.beta2 = hp->beta2, b.eps = hp->eps;
+        b.inv_bc1 = (float)(1.0 / bc1), b.inv_sqrt_bc2 = (float)(1.0 / std::sqrt(bc2));
+        int64_t nmax = 0;
+        double bytes = 0;
+        for (int j = 0; j < nt; ++j) {
+            const noble_adamw_tensor &t = tensors[i0 + j];
+            opt::AdamwTensor &d = b.t[j];
+            d.p = t.param, d.p_bf16 = (__nv_bfloat16 *)t.param_bf16, d.g = t.grad, d.m = t.exp_avg;
+            d.v = t.exp_avg_sq, d.n = t.n;
+            d.lr = hp->lr * t.lr_mult;
+            d.decay = t.decay ? d.lr * hp->weight_decay : 0.f;
+            d.vec4 = t.n % 4 == 0 ? 1 : 0;  // pointers are 16-byte aligned (checked)
+            nmax = std::max(nmax, t.n);
+            bytes += (28.0 + (t.param_bf16 ? 2.0 : 0.0)) * t.n;
+        }
+        const unsigned gx = (unsigned)std::max<int64_t>(1, std::min<int64_t>(ceil_div(ceil_div(nmax, 4), 256),
+                                                                             4 * (int64_t)num_sms()));
+        const KernelInfo ki{"adamw_step", kBoundHbm, 0.0, bytes};
+        NOBLE_TRY(run(st, ki, [&] { opt::adamw_kernel<<<dim3(gx, (unsigned)nt), 256, 0, st>>>(b); }));
+    }
+    return NOBLE_OK;
+}
+
+noble_status noble_linear_lr_multipliers(const noble_linear_desc *desc, float gamma, float gamma_M, float omega_mult,
+                                         float phi_mult, float out[5])
+{
+    g_last_error[0] = 0;
+    if (!desc || !out) return fail(NOBLE_ERR_INVALID_ARG, "desc / out is NULL");
+    NOBLE_TRY(validate_desc(desc));
+    if (desc->r == 0) return fail(NOBLE_ERR_INVALID_ARG, "r == 0: no branch groups");
+    const double rho = (double)std::min(desc->d_in, desc->d_out) / (double)desc->r;
+    out[0] = 1.f;
+    out[1] = (float)std::pow(rho, 2.0 * gamma);
+    out[2] = (float)std::pow(rho, (double)gamma_M);
+    out[3] = omega_mult;
+    out[4] = phi_mult;
+    return NOBLE_OK;
 }
 
 noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, int a_mn, int b_mn, int bn,

@@ -140,3 +140,33 @@ def test_bwd_workspace_size_checked(lib):
     with pytest.raises(binding.NobleError) as e:
         binding.noble_linear_bwd(d, **kw)
     assert e.value.status == 1 and "dM" in str(e.value)
+
+
+def test_lr_multipliers_host(lib):
+    from oracle import adamw
+    for d_in, d_out, r in [(2048, 8192, 128), (1024, 1024, 64), (768, 3072, 16)]:
+        got = binding.noble_linear_lr_multipliers(binding.make_desc(256, d_in, d_out, r, "bf16"))
+        ref = adamw.lr_multipliers(d_in, d_out, r)
+        assert got == pytest.approx([ref["W"], ref["W_up"], ref["M"], ref["omega"], ref["phi"]], rel=1e-6)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_linear_lr_multipliers(binding.make_desc(256, 128, 128, 0, "bf16"))
+    assert e.value.status == 1
+
+
+def test_adamw_arguments_validated(lib):
+    t = dict(param=FAKE, grad=FAKE, exp_avg=FAKE, exp_avg_sq=FAKE, n=64)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_adamw_step([t], lr=1e-3, step=0)
+    assert e.value.status == 1
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_adamw_step([dict(t, grad=None)], lr=1e-3)
+    assert e.value.status == 1
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_adamw_step([dict(t, exp_avg=FAKE + 4)], lr=1e-3)
+    assert e.value.status == 2
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_adamw_step([dict(t, param_bf16=FAKE + 2)], lr=1e-3)
+    assert e.value.status == 2
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_adamw_step([t], lr=1e-3, beta2=1.0)
+    assert e.value.status == 1
