@@ -445,6 +445,44 @@ def main():
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e,
                "copies": "pinned host buffers, copy streams overlapping compute"}
 
+    # optimizer step over the layers' parameters (fused AdamW with NOBLE's
+    # per-group learning rates; fp32 masters and moments, bf16 operand copies
+    # of W, W_down and W_up): HBM-bound, reported against the copy bandwidth
+    adamw = None
+    opt_tensors, opt_bytes = [], 0.0
+    for layer, d, b in zip(layers, dev_inputs, bufs):
+        mult = binding.noble_linear_lr_multipliers(b.desc) if layer.r > 0 else [1.0] * 5
+        groups = [("W", "dW", mult[0], True, True), ("bias", "dbias", mult[0], False, False)]
+        if layer.r > 0:
+            groups += [("W_down", "dW_down", mult[0], True, True), ("W_up", "dW_up", mult[1], True, True),
+                       ("M", "dM", mult[2], True, False), ("omega1", "domega1", mult[3], False, False),
+                       ("omega2", "domega2", mult[3], False, False), ("phi1", "dphi1", mult[4], False, False),
+                       ("phi2", "dphi2", mult[4], False, False)]
+        for name, gname, k, decay, lowp in groups:
+            g = b.grads[gname].reshape(-1)
+            n = g.numel()
+            opt_tensors.append({"param": d[name].float().reshape(-1).clone(), "grad": g,
+                                "exp_avg": torch.zeros(n, device="cuda"), "exp_avg_sq": torch.zeros(n, device="cuda"),
+                                "param_bf16": torch.empty(n, dtype=torch.bfloat16, device="cuda") if lowp else None,
+                                "lr_mult": k, "decay": decay})
+            opt_bytes += (28.0 + (2.0 if lowp else 0.0)) * n
+    opt_step = [0]
+
+    def adamw_step():
+        opt_step[0] += 1
+        binding.noble_adamw_step(opt_tensors, lr=3e-4, weight_decay=0.01, step=opt_step[0])
+
+    for _ in range(args.warmup):
+        adamw_step()
+    ms_adamw = timed(adamw_step, args.steps) / args.steps
+    binding.noble_get_device_status(None)
+    adamw = {"ms_per_step": ms_adamw, "bytes_per_step": opt_bytes,
+             "achieved_gbs": opt_bytes / (ms_adamw * 1e-3) / 1e9, "peak_gbs": pk["hbm"],
+             "frac": opt_bytes / (ms_adamw * 1e-3) / 1e9 / pk["hbm"],
+             "params": sum(t["param"].numel() for t in opt_tensors),
+             "note": "not part of the fwd+bwd step; lr 3e-4, betas (0.9, 0.98), weight decay 0.01"}
+    del opt_tensors
+
     per_layer = None
     if args.per_layer:
         per_layer = {}
@@ -513,6 +551,7 @@ def main():
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "per_layer": per_layer,
             "gpu_launches": launches,
             "profiled_ms_per_step": ms_profiled / args.steps,
+            "optimizer_step": adamw,
             "kernel_breakdown": {k: {"ms_per_step": v["ms"] / args.steps,
                                      "launches_per_step": v["launches"] / args.steps}
                                  for k, v in sorted(prof.items(), key=lambda kv: -kv[1]["ms"])},
