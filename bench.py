@@ -198,6 +198,8 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--profile-run", action="store_true",
                     help="fwd+bwd of the selected layers only, for ncu; prints no bench line")
+    ap.add_argument("--profile-optimizer", action="store_true",
+                    help="with --profile-run: also one optimizer step over the layers' parameters")
     ap.add_argument("--layers", default="", help="comma-separated layer names (default: all)")
     ap.add_argument("--config", type=int, default=CONFIG_INDEX,
                     help="workload: configuration 0-4 (default 3, the headline)")
@@ -272,9 +274,35 @@ def main():
             ms = float(t.item())
         return ms
 
+    # optimizer step over the layers' parameters (fused AdamW with NOBLE's
+    # per-group learning rates; fp32 masters and moments, bf16 operand copies
+    # of W, W_down and W_up): HBM-bound, reported against the copy bandwidth
+    def optimizer_tensors():
+        opt_tensors, opt_bytes = [], 0.0
+        for layer, d, b in zip(layers, dev_inputs, bufs):
+            mult = binding.noble_linear_lr_multipliers(b.desc) if layer.r > 0 else [1.0] * 5
+            groups = [("W", "dW", mult[0], True, True), ("bias", "dbias", mult[0], False, False)]
+            if layer.r > 0:
+                groups += [("W_down", "dW_down", mult[0], True, True), ("W_up", "dW_up", mult[1], True, True),
+                           ("M", "dM", mult[2], True, False), ("omega1", "domega1", mult[3], False, False),
+                           ("omega2", "domega2", mult[3], False, False), ("phi1", "dphi1", mult[4], False, False),
+                           ("phi2", "dphi2", mult[4], False, False)]
+            for name, gname, k, decay, lowp in groups:
+                g = b.grads[gname].reshape(-1)
+                n = g.numel()
+                opt_tensors.append({"param": d[name].float().reshape(-1).clone(), "grad": g,
+                                    "exp_avg": torch.zeros(n, device="cuda"), "exp_avg_sq": torch.zeros(n, device="cuda"),
+                                    "param_bf16": torch.empty(n, dtype=torch.bfloat16, device="cuda") if lowp else None,
+                                    "lr_mult": k, "decay": decay})
+                opt_bytes += (28.0 + (2.0 if lowp else 0.0)) * n
+        return opt_tensors, opt_bytes
+
     if args.profile_run:
         for _ in range(args.warmup + args.steps):
             step(bufs)
+        if args.profile_optimizer:
+            ts, _ = optimizer_tensors()
+            binding.noble_adamw_step(ts, lr=3e-4, weight_decay=0.01, step=1)
         torch.cuda.synchronize()
         binding.noble_get_device_status(None)
         print("profile run done", flush=True)
@@ -445,27 +473,8 @@ def main():
                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h, "ms_per_step": ms_e2e,
                "copies": "pinned host buffers, copy streams overlapping compute"}
 
-    # optimizer step over the layers' parameters (fused AdamW with NOBLE's
-    # per-group learning rates; fp32 masters and moments, bf16 operand copies
-    # of W, W_down and W_up): HBM-bound, reported against the copy bandwidth
     adamw = None
-    opt_tensors, opt_bytes = [], 0.0
-    for layer, d, b in zip(layers, dev_inputs, bufs):
-        mult = binding.noble_linear_lr_multipliers(b.desc) if layer.r > 0 else [1.0] * 5
-        groups = [("W", "dW", mult[0], True, True), ("bias", "dbias", mult[0], False, False)]
-        if layer.r > 0:
-            groups += [("W_down", "dW_down", mult[0], True, True), ("W_up", "dW_up", mult[1], True, True),
-                       ("M", "dM", mult[2], True, False), ("omega1", "domega1", mult[3], False, False),
-                       ("omega2", "domega2", mult[3], False, False), ("phi1", "dphi1", mult[4], False, False),
-                       ("phi2", "dphi2", mult[4], False, False)]
-        for name, gname, k, decay, lowp in groups:
-            g = b.grads[gname].reshape(-1)
-            n = g.numel()
-            opt_tensors.append({"param": d[name].float().reshape(-1).clone(), "grad": g,
-                                "exp_avg": torch.zeros(n, device="cuda"), "exp_avg_sq": torch.zeros(n, device="cuda"),
-                                "param_bf16": torch.empty(n, dtype=torch.bfloat16, device="cuda") if lowp else None,
-                                "lr_mult": k, "decay": decay})
-            opt_bytes += (28.0 + (2.0 if lowp else 0.0)) * n
+    opt_tensors, opt_bytes = optimizer_tensors()
     opt_step = [0]
 
     def adamw_step():
