@@ -183,6 +183,25 @@ def run_reference(args, rank):
     print(json.dumps(line), flush=True)
 
 
+# ------------------------------------------------------------------ ranks
+def max_over_ranks(ms: float, dist, device: str = "cuda") -> float:
+    """The job's time for a timed region: the slowest rank's (each rank's
+    region ends at its own last event).  ``dist`` is torch.distributed or
+    None for one process."""
+    if dist is None:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(world: int, flops_per_rank_step: float, ms_per_step: float) -> float:
+    """Whole-job TFLOP/s: every rank processes its own batch of the same
+    shape (weak scaling, replicas), so the work is world times one rank's."""
+    return world * flops_per_rank_step / (ms_per_step * 1e-3) / 1e12
+
+
 # ------------------------------------------------------------------ GPU arm
 def main():
     ap = argparse.ArgumentParser()
@@ -267,12 +286,7 @@ def main():
             fn()
         e1.record(stream)
         torch.cuda.synchronize()
-        ms = e0.elapsed_time(e1)
-        if dist is not None:
-            t = torch.tensor([ms], device="cuda")
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            ms = float(t.item())
-        return ms
+        return max_over_ranks(e0.elapsed_time(e1), dist)
 
     # optimizer step over the layers' parameters (fused AdamW with NOBLE's
     # per-group learning rates; fp32 masters and moments, bf16 operand copies
@@ -361,7 +375,7 @@ def main():
     binding.noble_get_device_status(None)
 
     ms_step = ms / args.steps
-    value = world * flops_step / (ms_step * 1e-3) / 1e12
+    value = job_throughput(world, flops_step, ms_step)
     pk = peaks()
 
     # dominant kernel: largest share of summed kernel time (profiled run)
@@ -459,12 +473,7 @@ def main():
             stream.wait_stream(d2h_s)
             e1.record(stream)
             torch.cuda.synchronize()
-            ms = e0.elapsed_time(e1)
-            if dist is not None:
-                t = torch.tensor([ms], device="cuda")
-                dist.all_reduce(t, op=dist.ReduceOp.MAX)
-                ms = float(t.item())
-            return ms
+            return max_over_ranks(e0.elapsed_time(e1), dist)
 
         for _ in range(2):
             e2e_step()
