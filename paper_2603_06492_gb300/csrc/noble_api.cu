@@ -561,64 +561,6 @@ struct ProbSpec {
 
 template <int BN_MAX> struct PStagesFor { static constexpr int value = BN_MAX >= 256 ? 4 : 6; };
 
-template <int BN_MAX, bool A_MN, bool B_MN, class Epi>
-noble_status tc_group(cudaStream_t st, const char *name, int n, const ProbSpec *specs,
-                      const typename Epi::Params *eps)
-{
-    constexpr int STAGES = PStagesFor<BN_MAX>::value;
-    using SM = tc::PSmem<BN_MAX, STAGES>;
-    if (n < 1 || n > tc::kMaxProblems) return fail(NOBLE_ERR_INVALID_ARG, "%s: %d problems", name, n);
-    tc::GroupMaps maps;
-    tc::GroupArgs<typename Epi::Params> g{};
-    int tiles = 0;
-    double flops = 0, bytes = 0;
-    int np = 0;
-    for (int i = 0; i < n; ++i) {
-        const ProbSpec &P = specs[i];
-        if (P.M == 0 || P.N == 0) continue;
-        if (P.bn % 32 || P.bn > BN_MAX || (B_MN && P.bn % 64))
-            return fail(NOBLE_ERR_INVALID_ARG, "%s: tile width %d", name, P.bn);
-        auto mk = [&](CUtensorMap *m, const void *p, bool mn, int64_t mnrows, int64_t K, uint32_t box_rows) {
-            return mn ? make_map(m, p, K, mnrows, 64) : make_map(m, p, mnrows, K, box_rows);
-        };
-        NOBLE_TRY(mk(&maps.m[np][0], P.s0.A, A_MN, P.M, P.s0.K, tc::kBM));
-        NOBLE_TRY(mk(&maps.m[np][1], P.s0.B, B_MN, P.N, P.s0.K, (uint32_t)P.bn));
-        if (P.s1) {
-            NOBLE_TRY(mk(&maps.m[np][2], P.s1->A, A_MN, P.M, P.s1->K, tc::kBM));
-            NOBLE_TRY(mk(&maps.m[np][3], P.s1->B, B_MN, P.N, P.s1->K, (uint32_t)P.bn));
-        } else {
-            maps.m[np][2] = maps.m[np][0];
-            maps.m[np][3] = maps.m[np][1];
-        }
-        auto &q = g.p[np];
-        q.M = P.M;
-        q.N = P.N;
-        q.kb0 = (int)ceil_div(P.s0.K, tc::kBK);
-        q.kb1 = P.s1 ? (int)ceil_div(P.s1->K, tc::kBK) : 0;
-        q.bn = P.bn;
-        q.tiles_m = (int)ceil_div(P.M, tc::kBM);
-        q.tiles_n = (int)ceil_div(P.N, P.bn);
-        q.nsplit = P.nsplit;
-        q.kb_per_split = P.kb_per_split;
-        q.tile_begin = tiles;
-        q.ep = eps[i];
-        tiles += q.tiles_m * q.tiles_n * q.nsplit;
-        const double K = (double)P.s0.K + (P.s1 ? (double)P.s1->K : 0.0);
-        flops += 2.0 * P.M * P.N * K;
-        bytes += 2.0 * (P.M + P.N) * K;
-        ++np;
-    }
-    if (np == 0) return NOBLE_OK;
-    g.nproblems = np;
-    g.total_tiles = tiles;
-    g.status = status_ptr();
-    auto kern = tc::gemm_persistent<BN_MAX, A_MN, B_MN, STAGES, Epi>;
-    if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kDynamic) != cudaSuccess)
-        return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
-    const int grid = tiles < num_sms() ? tiles : num_sms();
-    const KernelInfo ki{name, kBoundTensor, flops, bytes};
-    return run(st, ki, [&] { kern<<<grid, tc::kThreads, SM::kDynamic, st>>>(maps, g); });
-}
 
 
 
@@ -1381,8 +1323,8 @@ noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, 
     const int64_t split_stride = nsplit > 1 ? M * N : 0;
     const tc::EpiStore<float>::Params pf{(float *)C, N, bias, split_stride};
     const tc::EpiStore<bf16>::Params pb{(bf16 *)C, N, bias, split_stride};
-    // N tiles of 128 and 256 run on CTA pairs (the product path's kernel), 64 on
-    // the single-CTA persistent kernel, narrower ones on the one-tile kernel
+    // N tiles of 128 and 256 run on CTA pairs (the product path's kernel),
+    // narrower ones on the single-CTA one-tile kernel
     if ((bn == 128 || bn == 256) && !(a_mn && !b_mn)) {
         const ProbSpec P{M, N, s0, s1, bn, nsplit, kb_per_split};
         // MN-major operands take the 4-D layout when their extents allow it
