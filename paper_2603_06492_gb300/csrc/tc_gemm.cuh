@@ -166,7 +166,8 @@ struct EpiStore {
             ptx::fence_proxy_async_smem();
             __syncwarp();
             if (lane == 0) {
-                ptx::tma_store_3d(map, stg, (int)(n0 + c), (int)(m0 + quarter * 32), z);
+                ptx::tma_store_3d_hint(map, stg, (int)(n0 + c), (int)(m0 + quarter * 32), z,
+                                       ptx::l2_policy_evict_first());
                 ptx::bulk_commit_group();
             }
         }
