@@ -31,7 +31,8 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from paper_2603_06492_gb300.inputs import CONFIGS, layer_seed, make_layer_inputs  # noqa: E402
+from paper_2603_06492_gb300.inputs import (CONFIGS, PAPER_WORKLOAD_SEED, PAPER_WORKLOADS,  # noqa: E402
+                                           layer_seed, make_layer_inputs)
 
 CONFIG_INDEX = 3
 WORKLOADS = {
@@ -40,6 +41,9 @@ WORKLOADS = {
     2: "250M-scale FFN up + down, T=8192, d=1024, r=64, CosNet, fwd+bwd",
     3: "1.5B-scale FFN up/down + QKV, T=16384, d=2048, r=128, CosNet, fwd+bwd",
     4: "ViT-Base-shaped QKV + FFN up/down, T=50432, d=768, r in {16..256}, CosNet, fwd+bwd",
+    "geglu-base": "paper Base model GeGLU FFN (gate, up 1024->2752, down 2752->1024), T=8192, r=64, CosNet, fwd+bwd",
+    "geglu-large": "paper Large model GeGLU FFN (gate, up 2048->5504, down 5504->2048), T=16384, r=128, CosNet, "
+                   "fwd+bwd",
 }
 
 # DRAM bytes per launch of each tensor-core kernel class on the 1.5B-scale
@@ -49,7 +53,7 @@ WORKLOADS = {
 # DRAM bytes (read + write) per launch from one ncu capture of the current
 # kernels (profiles/traffic_config3_ffn_qkv_fwd_bwd.md), mean over the three
 # layers of config 3.
-TRAFFIC_PER_LAUNCH = {3: {"tc_wgrad": 869.9e6, "tc_main_up_fwd": 520.0e6, "tc_dx": 578.8e6}}
+TRAFFIC_PER_LAUNCH = {3: {"tc_wgrad": 869.7e6, "tc_main_up_fwd": 489.5e6, "tc_dx": 553.5e6}}
 METRIC = "NOBLE linear fwd+bwd TFLOP/s"
 
 
@@ -154,11 +158,19 @@ def host_cores():
     return int(n) if n else len(os.sched_getaffinity(0))
 
 
+def select_workload(args):
+    """(key, seed key, layers) of the workload the flags name: a numbered
+    configuration, or one of the paper's GeGLU FFN shapes (--workload)."""
+    if args.workload:
+        return args.workload, PAPER_WORKLOAD_SEED[args.workload], PAPER_WORKLOADS[args.workload]
+    return args.config, args.config, CONFIGS[args.config]
+
+
 def run_reference(args, rank):
     """--impl reference: the oracle as it stands, on host cores, rank 0 only."""
     if rank != 0:
         return
-    layers = CONFIGS[args.config]
+    cfg, _, layers = select_workload(args)
     import oracle
     oracle.build()
     for _ in range(args.warmup):
@@ -175,7 +187,7 @@ def run_reference(args, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOADS[args.config], "config_index": args.config, "sample": sample},
+            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "sample": sample},
             "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": host_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
@@ -222,6 +234,8 @@ def main():
     ap.add_argument("--layers", default="", help="comma-separated layer names (default: all)")
     ap.add_argument("--config", type=int, default=CONFIG_INDEX,
                     help="workload: configuration 0-4 (default 3, the headline)")
+    ap.add_argument("--workload", default="", choices=["", "geglu-base", "geglu-large"],
+                    help="the paper's GeGLU FFN shapes instead of a numbered configuration")
     ap.add_argument("--sigma", default="cosnet", choices=["cosnet", "cos1", "identity"],
                     help="bottleneck activation (cos1, identity: the variants of the ablation)")
     ap.add_argument("--per-layer", action="store_true",
@@ -250,15 +264,15 @@ def main():
     binding.load()
     assert args.profile_run or args.warmup >= 3, "at least 3 warm-up steps"
 
-    cfg = args.config
-    layers = CONFIGS[cfg]
+    cfg, seed_cfg, all_layers = select_workload(args)
+    layers = all_layers
     if args.layers:
         keep = set(args.layers.split(","))
         layers = [l for l in layers if l.name in keep]
     dev_inputs, bufs, plain_bufs = [], [], []
     for layer in layers:
-        li = [l.name for l in CONFIGS[cfg]].index(layer.name)
-        inp = make_layer_inputs(layer, layer_seed(cfg, li))
+        li = [l.name for l in all_layers].index(layer.name)
+        inp = make_layer_inputs(layer, layer_seed(seed_cfg, li))
         dev_inputs.append(binding.params_to_device(inp, layer.dtype))
         del inp
         sig_flags = {"cosnet": 0, "cos1": binding.NOBLE_FLAG_SIGMA_COS1,

@@ -139,6 +139,27 @@ def to_paper_orientation(inp: dict) -> dict:
     return out
 
 
+def geglu_hidden(d: int) -> int:
+    """GeGLU FFN hidden width of the paper's language models: 8/3 d rounded up
+    to a multiple of 64 (Section 4.1)."""
+    return -(-8 * d // (3 * 64)) * 64
+
+
+# The paper's own FFN shapes (GeGLU: gate and up projections d -> hidden,
+# down projection hidden -> d, NOBLE on all three), as extra workloads next
+# to the numbered configurations: the Base model (d = 1024, T = 8192 tokens
+# per GPU, r = 64) and the Large model (d = 2048, T = 16384, r = 128).
+PAPER_WORKLOADS = {
+    "geglu-base": [Layer("gate", 8192, 1024, geglu_hidden(1024), 64, "bf16"),
+                   Layer("up", 8192, 1024, geglu_hidden(1024), 64, "bf16"),
+                   Layer("down", 8192, geglu_hidden(1024), 1024, 64, "bf16")],
+    "geglu-large": [Layer("gate", 16384, 2048, geglu_hidden(2048), 128, "bf16"),
+                    Layer("up", 16384, 2048, geglu_hidden(2048), 128, "bf16"),
+                    Layer("down", 16384, geglu_hidden(2048), 2048, 128, "bf16")],
+}
+PAPER_WORKLOAD_SEED = {"geglu-base": 10, "geglu-large": 11}
+
+
 def layer_seed(config: int, layer_index: int) -> int:
     """Seed of layer ``layer_index`` of configuration ``config`` (config 0 -> 0)."""
     return config * 1000 + layer_index

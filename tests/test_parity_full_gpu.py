@@ -11,7 +11,8 @@ import numpy as np
 import pytest
 
 import oracle
-from paper_2603_06492_gb300.inputs import CONFIGS, layer_seed, make_layer_inputs, to_paper_orientation
+from paper_2603_06492_gb300.inputs import (CONFIGS, PAPER_WORKLOAD_SEED, PAPER_WORKLOADS, layer_seed,
+                                           make_layer_inputs, to_paper_orientation)
 from tests.gpu_helpers import TOL, rel_err, run_gpu
 
 pytestmark = pytest.mark.gpu
@@ -32,10 +33,23 @@ def lib():
 @pytest.mark.parametrize("cfg,li", CASES, ids=lambda v: str(v))
 def test_full_size_sampled(cfg, li):
     layer = CONFIGS[cfg][li]
-    inp = make_layer_inputs(layer, layer_seed(cfg, li))
+    check_full_size(layer, layer_seed(cfg, li), 100 + cfg * 31 + li, f"config {cfg}")
+
+
+@pytest.mark.parametrize("li", [0, 2], ids=["gate_2048x5504", "down_5504x2048"])
+def test_paper_geglu_shapes_sampled(li):
+    # the paper's Large-model GeGLU FFN projections: a hidden width (5504) that
+    # leaves a half-filled last 256-wide tile
+    w = "geglu-large"
+    layer = PAPER_WORKLOADS[w][li]
+    check_full_size(layer, layer_seed(PAPER_WORKLOAD_SEED[w], li), 700 + li, w)
+
+
+def check_full_size(layer, seed, rng_seed, ctx):
+    inp = make_layer_inputs(layer, seed)
     got = run_gpu(layer, inp)
     p = to_paper_orientation(inp)
-    rng = np.random.default_rng(100 + cfg * 31 + li)
+    rng = np.random.default_rng(rng_seed)
     tol = TOL[layer.dtype]
 
     rows = np.sort(rng.choice(layer.T, 48, replace=False))
@@ -66,4 +80,4 @@ def test_full_size_sampled(cfg, li):
     for k in ("dM", "domega1", "dphi1", "domega2", "dphi2"):
         errs[k] = rel_err(got[k], g[k])
     bad = {k: e for k, e in errs.items() if not e <= tol}
-    assert not bad, f"config {cfg} {layer.name}: {bad} (all {errs})"
+    assert not bad, f"{ctx} {layer.name}: {bad} (all {errs})"
