@@ -238,6 +238,8 @@ def main():
                     help="the paper's GeGLU FFN shapes instead of a numbered configuration")
     ap.add_argument("--sigma", default="cosnet", choices=["cosnet", "cos1", "identity"],
                     help="bottleneck activation (cos1, identity: the variants of the ablation)")
+    ap.add_argument("--fused-branch", action="store_true",
+                    help="run the bottleneck inside the output GEMMs (NOBLE_FLAG_FUSED_BRANCH)")
     ap.add_argument("--per-layer", action="store_true",
                     help="also time every layer alone (NOBLE and plain) and report each")
     args = ap.parse_args()
@@ -277,6 +279,8 @@ def main():
         del inp
         sig_flags = {"cosnet": 0, "cos1": binding.NOBLE_FLAG_SIGMA_COS1,
                      "identity": binding.NOBLE_FLAG_SIGMA_IDENTITY}[args.sigma]
+        if args.fused_branch:
+            sig_flags |= binding.NOBLE_FLAG_FUSED_BRANCH
         bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype,
                                                flags=sig_flags))
         plain_bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, 0, layer.dtype))

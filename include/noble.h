@@ -85,7 +85,8 @@ typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
                                    Limitations section): on the
                                    tensor-core path h and b are not written
                                    and `saved` holds only c, the second K
-                                   segment of the output GEMM.  The backward
+                                   segment of the output GEMM (and the ready
+                                   flags of a fused launch).  The backward
                                    entry points reject such a descriptor
                                    (NOBLE_ERR_INVALID_ARG).  The CUDA-core
                                    paths (fp32, SIMT_ONLY) use the full saved
@@ -101,6 +102,18 @@ typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
                                     not used (may be NULL) and their
                                     gradients are written as 0.  Not together
                                     with NOBLE_FLAG_SIGMA_COS1. */
+#define NOBLE_FLAG_FUSED_BRANCH 16u /* tensor-core path, CosNet bottleneck,
+                                    r in {64, 128}: run the r-wide GEMM and
+                                    the CosNet (forward h = x W_down^T and
+                                    Eq. 2; backward dc = dy W_up and its chain
+                                    rule) as tiles of the output GEMM launch
+                                    (y, dx) instead of kernels of their own;
+                                    the backward then sums dbias as dy^T 1 in
+                                    the weight-gradient launch.  Same results
+                                    up to summation order.  Off by default:
+                                    slower than the separate kernels at the
+                                    measured shapes.  Other shapes and
+                                    variants always run separately. */
 
 typedef struct {
     int64_t T;      /* tokens (rows of x)                          */
@@ -114,7 +127,10 @@ typedef struct {
 /*
  * Bytes of the saved-activation buffer that noble_linear_fwd writes and
  * noble_linear_bwd reads (per token: h and b in fp32, c in the operand dtype;
- * only c with NOBLE_FLAG_INFERENCE on the tensor-core path).  0 when r == 0.
+ * only c with NOBLE_FLAG_INFERENCE on the tensor-core path), plus, when the
+ * forward runs the bottleneck inside the output GEMM (NOBLE_FLAG_FUSED_BRANCH
+ * on the tensor-core path, CosNet, r in {64, 128}), one 32-bit ready flag per
+ * 128 tokens that the forward resets itself.  0 when r == 0.
  * Returns 0 for an invalid descriptor as well; the entry points then report
  * why.
  */

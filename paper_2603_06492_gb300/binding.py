@@ -22,6 +22,7 @@ HEADER = os.path.join(os.path.dirname(HERE), "include", "noble.h")
 NOBLE_BF16, NOBLE_FP32 = 0, 1
 NOBLE_FLAG_SIMT_ONLY, NOBLE_FLAG_INFERENCE = 1, 2
 NOBLE_FLAG_SIGMA_COS1, NOBLE_FLAG_SIGMA_IDENTITY = 4, 8
+NOBLE_FLAG_FUSED_BRANCH = 16
 STATUS = {0: "NOBLE_OK", 1: "NOBLE_ERR_INVALID_ARG", 2: "NOBLE_ERR_MISALIGNED",
           3: "NOBLE_ERR_UNSUPPORTED", 4: "NOBLE_ERR_BUFFER_TOO_SMALL", 5: "NOBLE_ERR_CUDA",
           6: "NOBLE_ERR_TIMEOUT", 7: "NOBLE_ERR_NO_DEVICE"}

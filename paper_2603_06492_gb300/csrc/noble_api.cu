@@ -75,6 +75,7 @@ constexpr uint32_t kFlagSimtOnly = NOBLE_FLAG_SIMT_ONLY;
 constexpr uint32_t kFlagInference = NOBLE_FLAG_INFERENCE;
 constexpr uint32_t kFlagSigmaCos1 = NOBLE_FLAG_SIGMA_COS1;
 constexpr uint32_t kFlagSigmaIdentity = NOBLE_FLAG_SIGMA_IDENTITY;
+constexpr uint32_t kFlagFusedBranch = NOBLE_FLAG_FUSED_BRANCH;
 
 // Bottleneck activation selected by the descriptor: 0 CosNet (Eq. 2), 1 single
 // cosine, 2 identity (the variants of the ablation, Section 4.4).
@@ -100,7 +101,7 @@ noble_status validate_desc(const noble_linear_desc *d)
         return fail(NOBLE_ERR_UNSUPPORTED, "r=%lld not in {0,16,32,64,128,256}", (long long)d->r);
     if (d->dtype != NOBLE_BF16 && d->dtype != NOBLE_FP32)
         return fail(NOBLE_ERR_UNSUPPORTED, "dtype %d not supported", (int)d->dtype);
-    if (d->flags & ~(kFlagSimtOnly | kFlagInference | kFlagSigmaCos1 | kFlagSigmaIdentity))
+    if (d->flags & ~(kFlagSimtOnly | kFlagInference | kFlagSigmaCos1 | kFlagSigmaIdentity | kFlagFusedBranch))
         return fail(NOBLE_ERR_UNSUPPORTED, "unknown flags 0x%x", d->flags);
     if ((d->flags & kFlagSigmaCos1) && (d->flags & kFlagSigmaIdentity))
         return fail(NOBLE_ERR_INVALID_ARG, "NOBLE_FLAG_SIGMA_COS1 and NOBLE_FLAG_SIGMA_IDENTITY together");
@@ -140,10 +141,22 @@ size_t esize(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 ? 2 : 4
 // True when the bf16 tensor-core path runs (the default for bf16 operands).
 bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->flags & kFlagSimtOnly); }
 
+// Tensor-core launches that run the bottleneck inside the output GEMM
+// (tc_pair.cuh, FUSE), on request: the CosNet with r in {64, 128}.  The
+// backward's MN-major operands also need d_in a multiple of 64 (4-D TMA layout).
+bool fuse_fwd(const noble_linear_desc *d)
+{
+    return use_tc(d) && sigma_mode(d) == 0 && (d->r == 64 || d->r == 128) && d->T > 0 &&
+           (d->flags & kFlagFusedBranch);
+}
+bool fuse_bwd(const noble_linear_desc *d) { return fuse_fwd(d) && d->d_in % 64 == 0; }
+// ready flags of a fused launch: one per 128-row block of whole row pairs
+size_t fuse_flag_bytes(const noble_linear_desc *d) { return (size_t)(2 * ((d->T + 255) / 256)) * 4; }
+
 // Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r];
 // only c for an inference forward on the tensor-core path.
 struct SavedLayout {
-    size_t h, b, c, total;
+    size_t h, b, c, flags, total;
     bool only_c;
 };
 SavedLayout saved_layout(const noble_linear_desc *d)
@@ -155,12 +168,16 @@ SavedLayout saved_layout(const noble_linear_desc *d)
         L.only_c = true;
         L.c = 0;
         L.total = align_up(tr * esize(d), 256);
-        return L;
+    } else {
+        L.h = 0;
+        L.b = align_up(L.h + tr * 4, 256);
+        L.c = align_up(L.b + tr * 4, 256);
+        L.total = align_up(L.c + tr * esize(d), 256);
     }
-    L.h = 0;
-    L.b = align_up(L.h + tr * 4, 256);
-    L.c = align_up(L.b + tr * 4, 256);
-    L.total = align_up(L.c + tr * esize(d), 256);
+    if (fuse_fwd(d)) {
+        L.flags = L.total;
+        L.total = align_up(L.flags + fuse_flag_bytes(d), 256);
+    }
     return L;
 }
 
@@ -200,10 +217,11 @@ void wgrad_shapes(const noble_linear_desc *d, int64_t (&mn)[5][2])
 //   CUDA-core path: dh (dtype), dc, a, db (fp32) [T][r]; M^T fp32; per-block
 //     partials of the CosNet sums, of dM and of dbias.
 //   tensor-core path: dh, a, db (bf16) [T][r]; per-CTA CosNet and dbias
-//     partials; without a branch an all-ones
-//     [T][64] bf16 operand (dbias = dy^T 1).
+//     partials; without a branch, or with the bottleneck fused into the dx
+//     launch, an all-ones [T][64] bf16 operand (dbias = dy^T 1); the fused
+//     launch's CosNet partials per 32 tokens and its ready flags.
 struct WorkLayout {
-    size_t dh, dc, a, db, mt, ones, cos_part, dm_part, bias_part, wsplit[5], total;
+    size_t dh, dc, a, db, mt, ones, cos_part, dm_part, bias_part, flags, wsplit[5], total;
     int split;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
 };
@@ -218,13 +236,21 @@ WorkLayout work_layout(const noble_linear_desc *d)
     if (use_tc(d)) {
         L.a = take(tr * 2);
         L.db = take(tr * 2);
-        L.ones = r ? 0 : take((size_t)T * kOnesCols * 2);  // dbias = dy^T 1 without a branch
-        // one partial per CTA of the CosNet kernel, whose grid is a whole number
-        // of CTA pairs (a padding CTA contributes exact zeros)
-        L.n_cos_blocks = r ? 2 * ceil_div(ceil_div(T, 128), 2) : 0;
-        L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
-        // with a branch, dbias is summed from the dy tiles of the CosNet kernel
-        L.bias_part = take((size_t)L.n_cos_blocks * d->d_out * 4);
+        const bool fused = fuse_bwd(d);
+        L.ones = (r && !fused) ? 0 : take((size_t)T * kOnesCols * 2);  // dbias = dy^T 1
+        if (fused) {
+            // one partial per 32 tokens (an epilogue warp's rows)
+            L.n_cos_blocks = ceil_div(T, 32);
+            L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
+            L.flags = take(fuse_flag_bytes(d));
+        } else {
+            // one partial per CTA of the CosNet kernel, whose grid is a whole
+            // number of CTA pairs (a padding CTA contributes exact zeros)
+            L.n_cos_blocks = r ? 2 * ceil_div(ceil_div(T, 128), 2) : 0;
+            L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
+            // with a branch, dbias is summed from the dy tiles of the CosNet kernel
+            L.bias_part = take((size_t)L.n_cos_blocks * d->d_out * 4);
+        }
         L.split = wgrad_split(d);
         if (L.split > 1) {
             int64_t mn[5][2];
@@ -557,6 +583,7 @@ struct ProbSpec {
     int bn;           // N tile (multiple of 32; of 64 when B is MN-major)
     int nsplit = 1;
     int kb_per_split = 0;
+    bool bneck = false;  // fused bottleneck tiles: the kernel's own epilogue, no C
 };
 
 template <int BN_MAX> struct PStagesFor { static constexpr int value = BN_MAX >= 256 ? 4 : 6; };
@@ -620,9 +647,9 @@ noble_status pair_schedule(GA &g, int clusters)
 
 // Grouped GEMM on CTA pairs (tc_pair.cuh): every problem's tile width must be
 // 128 or 256.  Tiles are 256 rows (a pair of 128-row halves).
-template <bool A_MN, bool B_MN, class Epi, bool MN4 = false>
+template <bool A_MN, bool B_MN, class Epi, bool MN4 = false, int FUSE = tc::pair::kFuseNone>
 noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbSpec *specs,
-                           const typename Epi::Params *eps)
+                           const typename Epi::Params *eps, const tc::pair::FuseArgs *fa = nullptr)
 {
     constexpr int STAGES = 6;
     using SM = tc::pair::PairSmem<STAGES>;
@@ -666,8 +693,9 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
             using OutT = typename Epi::out_type;
             constexpr int64_t es = sizeof(OutT);
             const auto &e = eps[i];
-            const bool ok = !e.col0 && reinterpret_cast<uintptr_t>(e.C) % 16 == 0 && (e.ldc * es) % 16 == 0 &&
-                            P.N % 4 == 0 && (P.nsplit == 1 || (e.split_stride * es) % 16 == 0);
+            const bool ok = !P.bneck && !e.col0 && reinterpret_cast<uintptr_t>(e.C) % 16 == 0 &&
+                            (e.ldc * es) % 16 == 0 && P.N % 4 == 0 &&
+                            (P.nsplit == 1 || (e.split_stride * es) % 16 == 0);
             q.ep.tma = ok ? 1 : 0;
             if (ok)
                 NOBLE_TRY(make_store_map(&maps.m[np][4], e.C, es == 4, P.M, P.N, e.ldc, P.nsplit, e.split_stride));
@@ -682,7 +710,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
     g.nproblems = np;
     g.total_tiles = tiles;
     g.status = status_ptr();
-    auto kern = tc::pair::gemm_pair<A_MN, B_MN, STAGES, Epi, MN4>;
+    auto kern = tc::pair::gemm_pair<A_MN, B_MN, STAGES, Epi, MN4, FUSE>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SM::kDynamic) != cudaSuccess)
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
     // as many pairs as can be resident at once
@@ -709,9 +737,11 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         if (dev >= 0 && dev < 64) max_clusters_cache[dev] = max_clusters;
     }
     const int clusters = tiles < max_clusters ? tiles : max_clusters;
-    NOBLE_TRY(pair_schedule(g, clusters));
+    // a fused launch walks its own dependency order (tc_pair.cuh: fused_tile)
+    if (FUSE == tc::pair::kFuseNone) NOBLE_TRY(pair_schedule(g, clusters));
+    const tc::pair::FuseArgs fargs = fa ? *fa : tc::pair::FuseArgs{};
     const KernelInfo ki{name, kBoundTensor, flops, bytes};
-    return run(st, ki, [&] { kern<<<2 * clusters, tc::pair::kPairThreads, SM::kDynamic, st>>>(maps, g); });
+    return run(st, ki, [&] { kern<<<2 * clusters, tc::pair::kPairThreads, SM::kDynamic, st>>>(maps, g, fargs); });
 }
 
 // Runtime r -> compile-time N tile for the r-wide products.
@@ -859,6 +889,23 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     const SavedLayout SL = saved_layout(d);
     float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
     bf16 *c = (bf16 *)(saved + SL.c);
+    if (fuse_fwd(d)) {
+        // one launch: bottleneck tiles (h, CosNet, c) and output tiles
+        uint32_t *flags = (uint32_t *)(saved + SL.flags);
+        if (cudaMemsetAsync(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
+            return fail(NOBLE_ERR_CUDA, "flags: %s", cudaGetErrorString(cudaGetLastError()));
+        tc::pair::FuseArgs fa{};
+        fa.T = T, fa.r = (int)r;
+        fa.om1 = om1, fa.ph1 = ph1, fa.om2 = om2, fa.ph2 = ph2, fa.M = M;
+        fa.h_out = SL.only_c ? nullptr : h, fa.b_out = SL.only_c ? nullptr : b, fa.c_out = c;
+        fa.flags = flags;
+        const TcSeg up{c, W_up, r};
+        ProbSpec P[2] = {ProbSpec{T, r, TcSeg{x, W_down, di}, nullptr, 128}, ProbSpec{T, dout, main, &up, 256}};
+        P[0].bneck = true;
+        const tc::EpiStore<bf16>::Params E[2] = {{nullptr, 0, nullptr, 0}, py};
+        return tc_pair_group<false, false, tc::EpiStore<bf16>, false, tc::pair::kFuseFwd>(st, "tc_main_up_fwd", 2, P,
+                                                                                           E, &fa);
+    }
     tc::CosnetArgs a{};
     a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2, a.M = M;
     a.h_out = SL.only_c ? nullptr : h, a.b_out = SL.only_c ? nullptr : b, a.c_out = c;
@@ -886,9 +933,36 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     const WorkLayout WL = work_layout(d);
     bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
     bf16 *ones = (bf16 *)(ws + WL.ones);
-    const bool ones_dbias = dbias && r == 0;
+    const bool fused = fuse_bwd(d);
+    const bool ones_dbias = dbias && (r == 0 || fused);
     if (ones_dbias) NOBLE_TRY(fill_ones(st, T * kOnesCols, ones));
-    if (r > 0) {
+    // domega1, dphi1, domega2, dphi2 (and dbias) from per-CTA or per-32-token partials
+    auto reduce_cosnet = [&](const float *cpart, const float *bpart) {
+        SplitJobs J{};
+        float *outs[4] = {dom1, dph1, dom2, dph2};
+        J.nparts = (int)WL.n_cos_blocks;
+        J.begin[0] = 0;
+        for (int q = 0; q < 4; ++q) {
+            J.part[q] = cpart + q * r;
+            J.out[q] = outs[q];
+            J.n[q] = r;
+            J.stride[q] = 4 * r;
+            J.begin[q + 1] = J.begin[q] + r;
+        }
+        J.njobs = 4;
+        if (bpart) {
+            J.part[4] = bpart;
+            J.out[4] = dbias;
+            J.n[4] = dout;
+            J.stride[4] = dout;
+            J.begin[5] = J.begin[4] + dout;
+            J.njobs = 5;
+        }
+        const int64_t total = J.begin[J.njobs];
+        const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
+        return run(st, kr, [&] { reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J); });
+    };
+    if (r > 0 && !fused) {
         float *cpart = (float *)(ws + WL.cos_part);
         tc::CosnetArgs ca{};
         ca.om1 = om1, ca.ph1 = ph1, ca.om2 = om2, ca.ph2 = ph2, ca.M = M;
@@ -905,33 +979,29 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             default: return cosnet_launch<R, true, tc::kSigCosnet>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
             }
         }));
-        // domega1, dphi1, domega2, dphi2 (and dbias) from the per-CTA partials
-        SplitJobs J{};
-        float *outs[4] = {dom1, dph1, dom2, dph2};
-        J.nparts = (int)WL.n_cos_blocks;
-        J.begin[0] = 0;
-        for (int q = 0; q < 4; ++q) {
-            J.part[q] = cpart + q * r;
-            J.out[q] = outs[q];
-            J.n[q] = r;
-            J.stride[q] = 4 * r;
-            J.begin[q + 1] = J.begin[q] + r;
-        }
-        J.njobs = 4;
-        if (dbias) {
-            J.part[4] = bpart;
-            J.out[4] = dbias;
-            J.n[4] = dout;
-            J.stride[4] = dout;
-            J.begin[5] = J.begin[4] + dout;
-            J.njobs = 5;
-        }
-        const int64_t total = J.begin[J.njobs];
-        const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
-        NOBLE_TRY(run(st, kr, [&] { reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J); }));
+        NOBLE_TRY(reduce_cosnet(cpart, dbias ? bpart : nullptr));
     }
     // dx = [dy | dh] [W ; W_down]
-    {
+    if (fused) {
+        // one launch: bottleneck tiles (dc, CosNet chain rule, dh) and dx tiles
+        uint32_t *flags = (uint32_t *)(ws + WL.flags);
+        if (cudaMemsetAsync(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
+            return fail(NOBLE_ERR_CUDA, "flags: %s", cudaGetErrorString(cudaGetLastError()));
+        float *cpart = (float *)(ws + WL.cos_part);
+        tc::pair::FuseArgs fa{};
+        fa.T = T, fa.r = (int)r;
+        fa.om1 = om1, fa.ph1 = ph1, fa.om2 = om2, fa.ph2 = ph2, fa.M = M;
+        fa.h_in = (const float *)(saved + SL.h), fa.b_in = (const float *)(saved + SL.b);
+        fa.dh_out = dh, fa.a_out = a, fa.db_out = db, fa.part = cpart, fa.flags = flags;
+        const tc::EpiStore<bf16>::Params E[2] = {{nullptr, 0, nullptr, 0}, {dx, di, nullptr, 0}};
+        const TcSeg sdx2{dh, W_down, r};
+        ProbSpec P[2] = {ProbSpec{T, r, TcSeg{dy, W_up, dout}, nullptr, 128},
+                         ProbSpec{T, di, TcSeg{dy, W, dout}, &sdx2, 256}};
+        P[0].bneck = true;
+        NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>, true, tc::pair::kFuseBwd>(st, "tc_dx", 2, P, E,
+                                                                                           &fa)));
+        NOBLE_TRY(reduce_cosnet(cpart, nullptr));
+    } else {
         const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
         const TcSeg sdx2{dh, W_down, r};
         const ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};

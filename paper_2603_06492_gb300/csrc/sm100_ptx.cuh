@@ -247,6 +247,60 @@ __device__ __forceinline__ void tmem_ld_32x32b_x16(uint32_t taddr, float (&v)[16
     for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
+// 32 TMEM lanes x 16 consecutive 32-bit columns from registers (thread i of
+// the warp writes lane warp_quarter*32 + i); returns once the writes are done.
+__device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_t (&v)[16])
+{
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]),
+        "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+        : "memory");
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// ------------------------------------------------------------- flags in global memory
+// A ready flag set by one CTA after its stores and polled by another CTA
+// before reading those stores through TMA (the async proxy).
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p)
+{
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release_gpu(uint32_t *p, uint32_t v)
+{
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+// Orders this thread's generic-proxy shared-memory writes before async-proxy
+// reads of them by any CTA of the cluster (an MMA of the CTA pair).
+__device__ __forceinline__ void fence_proxy_async_smem_cluster()
+{
+    asm volatile("fence.proxy.async.shared::cluster;" ::: "memory");
+}
+// Orders this thread's generic-proxy global accesses with its async-proxy ones.
+__device__ __forceinline__ void fence_proxy_async_global() { asm volatile("fence.proxy.async.global;" ::: "memory"); }
+
+// Wait until *flag is non-zero, for at most about kWaitLimitNs (then as
+// mbar_wait: status flagged, false returned).  On success the writes that
+// preceded the flag's release are visible to this thread's later TMA reads.
+__device__ __forceinline__ bool flag_wait(const uint32_t *flag, uint32_t *status)
+{
+    if (ld_acquire_gpu(flag) == 0) {
+        const uint64_t t0 = globaltimer_ns();
+        while (ld_acquire_gpu(flag) == 0) {
+            if (globaltimer_ns() - t0 > kWaitLimitNs) {
+                raise_status(status, kStatusTimeout);
+                return false;
+            }
+            __nanosleep(64);
+        }
+    }
+    fence_proxy_async_global();
+    return true;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi)
 {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);

@@ -19,9 +19,33 @@
 //     alternate 32-column chunks): reads its own accumulator rows and
 //     arrives on the LEADER's `tempty` (16 arrivals: 8 warps x 2 CTAs).
 // All waits are bounded as in the single-CTA kernels.
+//
+// Fused bottleneck (FUSE = kFuseFwd / kFuseBwd, on request through
+// NOBLE_FLAG_FUSED_BRANCH; the separate kernels of tc_cosnet.cuh are the
+// default because they are faster at the measured shapes): problem 0 of the launch is
+// the r-wide GEMM of the low-rank branch, h = x W_down^T (forward) or
+// dc = dy W_up (backward), one 256 x r tile per row pair, and problem 1 the
+// output GEMM whose second K segment reads c = CosNet(h) (forward, Eq. 1-2)
+// or dh (backward) of the same rows.  A bottleneck tile's epilogue runs the
+// CosNet of Eq. 2 (or its chain rule) on the accumulator:
+//   phase 1   a = cos(omega1 h + phi1)      | du2 = -sin(omega2 b + phi2) dc,
+//                                           |   db = omega2 du2
+//             as bf16 high and low parts written back into TMEM columns [0, r)
+//   product   b = a M  (or da = db M^T), a second pair MMA with A in TMEM and
+//             the mixing matrix (bf16 high/low, this CTA's half of its
+//             columns) in the epilogue staging buffer, into columns
+//             [128, 128 + r) of the same accumulator
+//   phase 2   c = cos(omega2 b + phi2)      | du1 = -sin(omega1 h + phi1) da,
+//                                           |   dh = omega1 du1, a = cos(u1)
+// then stores c (dh) for its 128 rows and releases a flag per 128-row block.
+// The producer of an output tile polls that flag (bounded) before loading
+// its second segment.  Tiles run in the order of fused_tile, which puts
+// every bottleneck tile before the output tiles that wait for it, so with all
+// clusters resident every wait ends.
 #pragma once
 
 #include "tc_persistent.cuh"
+#include "tc_cosnet.cuh"
 
 namespace noble {
 namespace tc {
@@ -155,6 +179,65 @@ __device__ __forceinline__ PairTile locate_pair(const GroupArgs<EpiParams> &g, i
     return r;
 }
 
+constexpr int kFuseNone = 0, kFuseFwd = 1, kFuseBwd = 2;
+constexpr uint32_t kR2Col = 128;  // TMEM column of the bottleneck's second accumulator
+
+struct FuseArgs {
+    int64_t T;
+    int r;                       // 64 or 128
+    const float *om1, *ph1, *om2, *ph2;
+    const float *M;              // fp32 [r][r], b_j = sum_i a_i M[i][j]
+    float *h_out, *b_out;        // forward: saved h, b (NULL: not saved)
+    __nv_bfloat16 *c_out;        // forward: c
+    const float *h_in, *b_in;    // backward: saved h, b
+    __nv_bfloat16 *dh_out, *a_out, *db_out;
+    float *part;                 // backward: [ceil(T / 32)][4][r] column sums per 32 tokens
+    uint32_t *flags;             // [2 * row pairs], zero at launch
+};
+
+// Fused tile order: the bottleneck tiles of row-pair group 0, then for each
+// group g the bottleneck tiles of group g + 1 followed by the output tiles of
+// group g (groups of 8 row pairs as in locate_pair).
+template <class EpiParams>
+__device__ __forceinline__ int fused_tile(const GroupArgs<EpiParams> &g, int p)
+{
+    const Problem<EpiParams> &C = g.p[0], &O = g.p[1];
+    const int pairs = (C.tiles_m + 1) / 2;
+    const int ng = (pairs + 7) / 8;
+    const int tn = O.tiles_n;
+    const int c0 = min(8, pairs);
+    if (p < c0) return C.tile_begin + p;
+    p -= c0;
+    // block gi = [C(gi + 1)] [O(gi)]; blocks below ng - 2 are all 8 + 8 tn long
+    const int full = 8 + 8 * tn;
+    int gi = 0;
+    if (ng > 2) {
+        gi = min(p / full, ng - 2);
+        p -= gi * full;
+    }
+#pragma unroll 1
+    for (; gi < ng; ++gi) {
+        const int cn = gi + 1 < ng ? min(8, pairs - 8 * (gi + 1)) : 0;
+        const int on = min(8, pairs - 8 * gi) * tn;
+        if (p < cn) return C.tile_begin + 8 * (gi + 1) + p;
+        p -= cn;
+        if (p < on) return O.tile_begin + 8 * gi * tn + p;
+        p -= on;
+    }
+    return -1;
+}
+
+__device__ __forceinline__ void mma2_bf16_ta(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc, uint32_t idesc,
+                                             uint32_t accumulate)
+{
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], [%1], %2, %3, p;\n\t}\n" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 // Tile of the given slot (see GroupArgs::sched); -1 when the slot is empty.
 template <class EpiParams>
 __device__ __forceinline__ int slot_tile(const GroupArgs<EpiParams> &g, int slot)
@@ -167,6 +250,245 @@ __device__ __forceinline__ int slot_tile(const GroupArgs<EpiParams> &g, int slot
 // Warps 0 (TMA), 1 (MMA, TMEM owner) and eight epilogue warps.
 constexpr int kPairThreads = 320;
 
+// ---------------------------------------------------------------- fused bottleneck
+// The mixing matrix as the B operand of the second product: this CTA's half of
+// its rows n (output columns of b or da), n in [rank r/2, (rank + 1) r/2), all
+// K = r, as bf16 high and low parts (x = x_hi + x_lo), K-major with the
+// 128-byte swizzle in k-blocks of 64.  Forward B[n][k] = M[k][n]
+// (b_j = sum_i a_i M[i][j]); backward B[n][k] = M[n][k] (da_i = sum_j db_j M[i][j]).
+// Epilogue thread et (0..255) converts the groups gi = et + 256 it of eight
+// consecutive k of one row n.
+template <int FUSE>
+__device__ __forceinline__ void mix_load(const FuseArgs &fa, uint32_t rank, int et, float (&mr)[4][8])
+{
+    const int r = fa.r, hr = r / 2, ngroups = hr * (r / 8);
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+        const int gi = et + 256 * it;
+        if (gi >= ngroups) continue;
+        const int n = (int)rank * hr + gi % hr, k = 8 * (gi / hr);
+        if constexpr (FUSE == kFuseBwd) {
+            const float4 *src = reinterpret_cast<const float4 *>(fa.M + (int64_t)n * r + k);
+            const float4 u = __ldg(src), w = __ldg(src + 1);
+            mr[it][0] = u.x, mr[it][1] = u.y, mr[it][2] = u.z, mr[it][3] = u.w;
+            mr[it][4] = w.x, mr[it][5] = w.y, mr[it][6] = w.z, mr[it][7] = w.w;
+        } else {
+#pragma unroll
+            for (int q = 0; q < 8; ++q) mr[it][q] = __ldg(fa.M + (int64_t)(k + q) * r + n);
+        }
+    }
+}
+
+__device__ __forceinline__ uint32_t mix_part_bytes(int r) { return (uint32_t)(r / 64) * (uint32_t)(r / 2) * 128u; }
+
+__device__ __forceinline__ void mix_store(int r, uint8_t *dst, int et, const float (&mr)[4][8])
+{
+    const int hr = r / 2, ngroups = hr * (r / 8);
+    const uint32_t part = mix_part_bytes(r);
+#pragma unroll
+    for (int it = 0; it < 4; ++it) {
+        const int gi = et + 256 * it;
+        if (gi >= ngroups) continue;
+        const int nl = gi % hr, k = 8 * (gi / hr);
+        uint4 hi, lo;
+        uint32_t *ph = &hi.x, *pl = &lo.x;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const __nv_bfloat162 h2 = __floats2bfloat162_rn(mr[it][2 * q], mr[it][2 * q + 1]);
+            const float2 hf = __bfloat1622float2(h2);
+            const __nv_bfloat162 l2 = __floats2bfloat162_rn(mr[it][2 * q] - hf.x, mr[it][2 * q + 1] - hf.y);
+            ph[q] = *reinterpret_cast<const uint32_t *>(&h2);
+            pl[q] = *reinterpret_cast<const uint32_t *>(&l2);
+        }
+        const uint32_t off = (uint32_t)(k / 64) * hr * 128u + (uint32_t)nl * 128u +
+                             ((((uint32_t)(k % 64) >> 3) ^ ((uint32_t)nl & 7u)) << 4);
+        *reinterpret_cast<uint4 *>(dst + off) = hi;
+        *reinterpret_cast<uint4 *>(dst + part + off) = lo;
+    }
+}
+
+// x = hi + lo in bf16 for two values: packed high parts and packed low parts.
+__device__ __forceinline__ void split_hi_lo(float x0, float x1, uint32_t &hi, uint32_t &lo)
+{
+    const __nv_bfloat162 h2 = __floats2bfloat162_rn(x0, x1);
+    const float2 hf = __bfloat1622float2(h2);
+    const __nv_bfloat162 l2 = __floats2bfloat162_rn(x0 - hf.x, x1 - hf.y);
+    hi = *reinterpret_cast<const uint32_t *>(&h2);
+    lo = *reinterpret_cast<const uint32_t *>(&l2);
+}
+
+// Epilogue of a bottleneck tile (see the header), run by all eight epilogue
+// warps of a CTA on its 128 rows; `acc` is the tile's TMEM accumulator.  A
+// thread owns one row and the 32-column chunks c = 32 half + 64 i < r.
+// Returns false, uniformly over the eight warps, after a timed-out wait.
+template <int FUSE>
+__device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *stg, uint32_t acc, int warp, int lane, int64_t m0,
+                                    uint32_t rank, uint32_t a_ready_leader, uint32_t b_full, uint32_t parity,
+                                    uint32_t *status)
+{
+    const int r = fa.r;
+    const int quarter = warp % 4, half = (warp - 2) / 4;
+    const int64_t t0 = m0 + quarter * 32;  // the warp's first row
+    const bool live = t0 + lane < fa.T;
+    const uint32_t lane_addr = acc + ((uint32_t)(quarter * 32) << 16);
+    const int et = (warp - 2) * 32 + lane;
+    float *part = FUSE == kFuseBwd ? fa.part + (t0 / 32) * 4 * (int64_t)r : nullptr;
+    // ---- phase 1: first accumulator (h or dc).  The row operand of the
+    // second product (a or db) replaces each 32-column chunk it came from:
+    // bf16 high parts of its 32 values in the chunk's first 16 columns, low
+    // parts in the last 16 (two values per 32-bit column, lower k in the low
+    // half), so each warp overwrites only columns it has read itself.
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const int c = 32 * half + 64 * i;
+        if (c >= r) continue;
+        float v[32];
+        ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
+        uint32_t ohi[16], olo[16];
+        if constexpr (FUSE == kFuseFwd) {
+            if (fa.h_out) {
+                uint32_t w[8][4];
+#pragma unroll
+                for (int g = 0; g < 8; ++g)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) w[g][q] = __float_as_uint(v[4 * g + q]);
+                store_segments<8>(w, fa.h_out + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+            }
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int k = c + 2 * e;
+                const float a0 = cos_reduced(fmaf(__ldg(fa.om1 + k), v[2 * e], __ldg(fa.ph1 + k)));
+                const float a1 = cos_reduced(fmaf(__ldg(fa.om1 + k + 1), v[2 * e + 1], __ldg(fa.ph1 + k + 1)));
+                split_hi_lo(a0, a1, ohi[e], olo[e]);
+            }
+        } else {
+            // v = dc; with b of this row: du2 = -sin(omega2 b + phi2) dc (kept
+            // in v), db = omega2 du2
+            float bv[32];
+            {
+                uint32_t w[8][4];
+                load_segments<8>(w, fa.b_in + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+#pragma unroll
+                for (int g = 0; g < 8; ++g)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) bv[4 * g + q] = __uint_as_float(w[g][q]);
+            }
+            uint32_t wdb[4][4];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int k = c + 2 * e;
+                const float w0 = __ldg(fa.om2 + k), w1 = __ldg(fa.om2 + k + 1);
+                const float d0 = live ? -sin_reduced(fmaf(w0, bv[2 * e], __ldg(fa.ph2 + k))) * v[2 * e] : 0.f;
+                const float d1 = live ? -sin_reduced(fmaf(w1, bv[2 * e + 1], __ldg(fa.ph2 + k + 1))) * v[2 * e + 1] : 0.f;
+                v[2 * e] = d0;
+                v[2 * e + 1] = d1;
+                split_hi_lo(w0 * d0, w1 * d1, ohi[e], olo[e]);
+                wdb[e / 4][e % 4] = ohi[e];
+            }
+            store_segments<4>(wdb, fa.db_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) bv[e] *= v[e];  // du2 b
+            const float s2 = warp_colsum32(bv);
+            const float s3 = warp_colsum32(v);
+            if (t0 < fa.T) {
+                part[2 * r + c + lane] = s2;
+                part[3 * r + c + lane] = s3;
+            }
+        }
+        ptx::tmem_st_32x32b_x16(lane_addr + c, ohi);
+        ptx::tmem_st_32x32b_x16(lane_addr + c + 16, olo);
+    }
+    // ---- the mixing matrix goes into the staging buffer once every warp's
+    // TMA stores have left it
+    {
+        float mr[4][8];
+        mix_load<FUSE>(fa, rank, et, mr);
+        if (lane == 0) ptx::bulk_wait_read_all();
+        __syncwarp();
+        ptx::tc_fence_before();
+        ptx::named_barrier_sync(1, 256);
+        ptx::tc_fence_after();
+        mix_store(r, stg, et, mr);
+    }
+    ptx::fence_proxy_async_smem_cluster();  // generic writes, read by the leader's MMA (async proxy)
+    ptx::tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive_cluster(a_ready_leader);
+    bool ok = ptx::mbar_wait(b_full, parity, status);
+    ok = ptx::named_barrier_and(1, 256, __all_sync(0xffffffffu, ok));
+    if (!ok) return false;
+    ptx::tc_fence_after();
+    // ---- phase 2: second accumulator (b or da)
+#pragma unroll
+    for (int i = 0; i < 2; ++i) {
+        const int c = 32 * half + 64 * i;
+        if (c >= r) continue;
+        float v[32];
+        ptx::tmem_ld_32x32b_x32(lane_addr + kR2Col + c, v);
+        if constexpr (FUSE == kFuseFwd) {
+            // v = b: c = cos(omega2 b + phi2)
+            uint32_t wc[4][4];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const int k = c + 2 * e;
+                const float c0 = cos_reduced(fmaf(__ldg(fa.om2 + k), v[2 * e], __ldg(fa.ph2 + k)));
+                const float c1 = cos_reduced(fmaf(__ldg(fa.om2 + k + 1), v[2 * e + 1], __ldg(fa.ph2 + k + 1)));
+                wc[e / 4][e % 4] = ptx::pack_bf16x2(c0, c1);
+            }
+            if (fa.b_out) {
+                uint32_t w[8][4];
+#pragma unroll
+                for (int g = 0; g < 8; ++g)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) w[g][q] = __float_as_uint(v[4 * g + q]);
+                store_segments<8>(w, fa.b_out + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+            }
+            store_segments<4>(wc, fa.c_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
+        } else {
+            // v = da; with h of this row: du1 = -sin(u1) da, dh = omega1 du1, a = cos(u1)
+            float hv[32];
+            {
+                uint32_t w[8][4];
+                load_segments<8>(w, fa.h_in + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+#pragma unroll
+                for (int g = 0; g < 8; ++g)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) hv[4 * g + q] = __uint_as_float(w[g][q]);
+            }
+            // du1 kept in v
+            uint32_t wdh[4][4], wa[4][4];
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                float dh2[2], av2[2];
+#pragma unroll
+                for (int u = 0; u < 2; ++u) {
+                    const int k = c + 2 * e + u;
+                    const float w1 = __ldg(fa.om1 + k);
+                    float s1, c1;
+                    sincos_reduced(fmaf(w1, hv[2 * e + u], __ldg(fa.ph1 + k)), &s1, &c1);
+                    const float du1 = live ? -s1 * v[2 * e + u] : 0.f;
+                    v[2 * e + u] = du1;
+                    dh2[u] = w1 * du1;
+                    av2[u] = c1;
+                }
+                wdh[e / 4][e % 4] = ptx::pack_bf16x2(dh2[0], dh2[1]);
+                wa[e / 4][e % 4] = ptx::pack_bf16x2(av2[0], av2[1]);
+            }
+            store_segments<4>(wdh, fa.dh_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
+            store_segments<4>(wa, fa.a_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
+#pragma unroll
+            for (int e = 0; e < 32; ++e) hv[e] *= v[e];  // du1 h
+            const float s0 = warp_colsum32(hv);
+            const float s1 = warp_colsum32(v);
+            if (t0 < fa.T) {
+                part[c + lane] = s0;
+                part[r + c + lane] = s1;
+            }
+        }
+    }
+    return true;
+}
+
 template <int STAGES>
 struct PairSmem {
     static constexpr uint32_t kA = kBM * kBK * 2;         // 128 rows of A
@@ -175,7 +497,8 @@ struct PairSmem {
     static constexpr uint32_t kStgOff = STAGES * kStage;  // epilogue staging, 4 KB per epilogue warp
     static constexpr uint32_t kStgBytes = 8 * 4096;
     static constexpr uint32_t kBarOff = kStgOff + kStgBytes;
-    static constexpr uint32_t kNumBars = 2 * STAGES + 5;  // full, empty, tfull[2], tempty[2], mma_done
+    static constexpr uint32_t kNumBars = 2 * STAGES + 7;  // full, empty, tfull[2], tempty[2], mma_done,
+                                                          // a_ready, b_full (fused bottleneck)
     static constexpr uint32_t kBytes = kBarOff + 8 * kNumBars + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
@@ -185,9 +508,12 @@ struct PairSmem {
 //   [8-row K group][64-wide MN chunk][8 rows][128 B]
 // (chunk stride 1 KB, group stride nchunks KB) instead of two or more 2-D
 // boxes giving [MN chunk][64 K rows][128 B] (chunk stride 8 KB, group 1 KB).
-template <bool A_MN, bool B_MN, int STAGES, class Epi, bool MN4 = false>
+// FUSE: kFuseNone, or a fused bottleneck launch (problem 0 bottleneck tiles
+// of N = r <= 128 with bn = 128, problem 1 output tiles, see the header).
+template <bool A_MN, bool B_MN, int STAGES, class Epi, bool MN4 = false, int FUSE = kFuseNone>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
-gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupArgs<typename Epi::Params> g)
+gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupArgs<typename Epi::Params> g,
+          const __grid_constant__ FuseArgs fa)
 {
     using S = PairSmem<STAGES>;
     constexpr uint32_t kAccCols = 256;
@@ -203,6 +529,9 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
     auto tfull_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + b); };
     auto tempty_bar = [&](int b) { return bar0 + 8u * (2 * STAGES + 2 + b); };
     const uint32_t mma_done = bar0 + 8u * (2 * STAGES + 4);
+    const uint32_t a_ready = bar0 + 8u * (2 * STAGES + 5);  // fused: row operand in TMEM, matrix in smem
+    const uint32_t b_full = bar0 + 8u * (2 * STAGES + 6);   // fused: second product complete
+    auto tile_of = [&](int slot) { return FUSE != kFuseNone ? fused_tile(g, slot) : slot_tile(g, slot); };
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + S::kBarOff + 8 * S::kNumBars);
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -224,6 +553,8 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             ptx::mbar_init(tempty_bar(b), 16);  // 8 epilogue warps in each CTA of the pair
         }
         ptx::mbar_init(mma_done, 1);
+        ptx::mbar_init(a_ready, 16);  // 8 epilogue warps in each CTA of the pair
+        ptx::mbar_init(b_full, 1);
         ptx::fence_barrier_init();
     }
     if (warp == 1) {
@@ -243,7 +574,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             bool ok = true;
             const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
             for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
-                const int t = slot_tile(g, slot);
+                const int t = tile_of(slot);
                 if (t < 0) continue;
                 const PairTile tr = locate_pair(g, t, rank);
                 const auto &P = g.p[tr.prob];
@@ -255,6 +586,14 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     if (!ptx::mbar_wait(empty_bar(s), ph ^ 1, g.status)) {
                         ok = false;
                         break;
+                    }
+                    if constexpr (FUSE != kFuseNone) {
+                        // the second segment of an output tile reads c (dh) of
+                        // this CTA's 128 rows, stored by a bottleneck tile
+                        if (tr.prob == 1 && kb == P.kb0 && !ptx::flag_wait(fa.flags + tr.m0 / kBM, g.status)) {
+                            ok = false;
+                            break;
+                        }
                     }
                     const uint32_t fb = map_to_rank(full_bar(s), 0);
                     if (leader) ptx::mbar_arrive_expect_tx(full_bar(s), 2 * cta_bytes);
@@ -304,8 +643,9 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             constexpr uint32_t kStepA = A_MN ? (MN4 ? 4096 / 16 : 2048 / 16) : 32 / 16;
             constexpr uint32_t kStageUnits = S::kStage / 16;
             const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
+            uint32_t nc = 0;  // bottleneck tiles so far
             for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
-                const int t = slot_tile(g, slot);
+                const int t = tile_of(slot);
                 if (t < 0) continue;
                 const PairTile tr = locate_pair(g, t, 0);
                 const auto &P = g.p[tr.prob];
@@ -363,6 +703,33 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     }
                 }
                 mma2_commit_mc(tfull_bar(b), 0x3);
+                if constexpr (FUSE != kFuseNone) {
+                    if (ok && tr.prob == 0) {
+                        // second product of the bottleneck tile: b | da (cols
+                        // kR2Col..) = (a | db in TMEM cols [0, r): per 32-column
+                        // chunk 16 columns of bf16 high parts, then 16 of low
+                        // parts) x (matrix hi/lo in the staging buffers of both
+                        // CTAs), as hi*hi + lo*hi + hi*lo
+                        if (!ptx::mbar_wait(a_ready, nc & 1, g.status)) break;
+                        ptx::tc_fence_after();
+                        const int r = fa.r;
+                        const uint32_t acc = tmem + b * kAccCols;
+                        const uint32_t idesc2 = ptx::idesc_bf16(2 * kBM, r, false, false);
+                        const uint32_t mhi = sbase + S::kStgOff, mlo = mhi + mix_part_bytes(r);
+                        for (int kk = 0; kk < r / 16; ++kk) {
+                            const uint32_t off = (uint32_t)(kk / 4) * (uint32_t)(r / 2) * 128u + (uint32_t)(kk % 4) * 32u;
+                            const uint64_t dmh = ptx::smem_desc_sw128(mhi + off, 16, 1024);
+                            const uint64_t dml = ptx::smem_desc_sw128(mlo + off, 16, 1024);
+                            const uint32_t ahi = acc + (uint32_t)(kk / 2) * 32u + (uint32_t)(kk % 2) * 8u;
+                            const uint32_t alo = ahi + 16u;
+                            mma2_bf16_ta(acc + kR2Col, ahi, dmh, idesc2, kk > 0 ? 1u : 0u);
+                            mma2_bf16_ta(acc + kR2Col, alo, dmh, idesc2, 1u);
+                            mma2_bf16_ta(acc + kR2Col, ahi, dml, idesc2, 1u);
+                        }
+                        mma2_commit_mc(b_full, 0x3);
+                        ++nc;
+                    }
+                }
                 ++j;
             }
             mma2_commit_mc(mma_done, 0x1);
@@ -377,18 +744,43 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         const uint32_t stg = sbase + S::kStgOff + (uint32_t)(warp - 2) * 4096u;
         uint8_t *stg_ptr = smem + S::kStgOff + (warp - 2) * 4096;
         int j = 0;
+        uint32_t nc = 0;  // bottleneck tiles so far
+        const uint32_t leader_a_ready = map_to_rank(a_ready, 0);
         const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
         for (int slot = cluster; slot < nslots; slot += nclusters) {
-            const int t = slot_tile(g, slot);
+            const int t = tile_of(slot);
             if (t < 0) continue;
             const PairTile tr = locate_pair(g, t, rank);
             const auto &P = g.p[tr.prob];
             const int b = j & 1;
             const uint32_t use = (uint32_t)(j >> 1);
+            const bool bneck = FUSE != kFuseNone && tr.prob == 0;
             bool ok = ptx::mbar_wait(tfull_bar(b), use & 1, g.status);
             ok = __all_sync(0xffffffffu, ok);
+            // fused launches use named barriers below: leave together or not at all
+            if constexpr (FUSE != kFuseNone) ok = ptx::named_barrier_and(1, 256, ok);
             if (!ok) break;
             ptx::tc_fence_after();
+            if constexpr (FUSE != kFuseNone) {
+                if (bneck) {
+                    if (!bottleneck_epilogue<FUSE>(fa, smem + S::kStgOff, tmem + b * kAccCols, warp, lane, tr.m0,
+                                                   rank, leader_a_ready, b_full, nc & 1, g.status))
+                        break;
+                    ptx::tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive_cluster(b ? leader_tempty1 : leader_tempty0);
+                    // every warp's stores of this CTA's rows are issued: publish them
+                    ptx::named_barrier_sync(1, 256);
+                    if (warp == 2 && lane == 0) {
+                        __threadfence();
+                        ptx::fence_proxy_async_global();
+                        ptx::st_release_gpu(fa.flags + tr.m0 / kBM, 1u);
+                    }
+                    ++nc;
+                    ++j;
+                    continue;
+                }
+            }
             if (P.ep.tma)
                 Epi::run_tma(P.ep, &maps.m[tr.prob][4], stg_ptr, stg, tmem + b * kAccCols, P.bn, quarter, lane, tr.m0,
                              tr.n0, P.N, tr.z, half);

@@ -29,11 +29,11 @@ def rel_err(got, ref) -> float:
     return float(err / scale) if scale > 0 else float(err)
 
 
-def run_gpu(layer: Layer, inp: dict, with_dbias=True, repeat=1):
+def run_gpu(layer: Layer, inp: dict, with_dbias=True, repeat=1, flags=0):
     """fwd + bwd through the C ABI; returns numpy fp64 outputs (library layout)."""
     import torch
     dev = binding.params_to_device(inp, layer.dtype)
-    buf = binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype)
+    buf = binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype, flags=flags)
     for _ in range(repeat):
         binding.forward(buf, dev["x"], dev)
         binding.backward(buf, dev["x"], dev["dy"], dev, with_dbias=with_dbias)

@@ -53,6 +53,38 @@ def test_small_shapes(dtype, shape, init):
     assert_close(got, ref, dtype, ctx=f"{shape} {dtype} {init}")
 
 
+# The bottleneck fused into the output GEMMs (NOBLE_FLAG_FUSED_BRANCH, the
+# CosNet with r in {64, 128}) and the separate kernels: both against the
+# oracle, on shapes with several groups of 8 row pairs, a ragged last group
+# and ragged column tiles (the fused tile order and its ready flags).
+FUSED = [
+    (5000, 256, 520, 128),
+    (5000, 192, 264, 64),
+    (2049, 512, 1000, 128),
+    (300, 136, 264, 64),   # d_in % 64 != 0: fused forward, separate backward
+]
+
+
+@pytest.mark.parametrize("shape", FUSED, ids=lambda s: "x".join(map(str, s)))
+@pytest.mark.parametrize("separate", [False, True], ids=["fused", "separate"])
+def test_fused_bottleneck(shape, separate):
+    layer = Layer("fused", *shape, "bf16")
+    inp = make_layer_inputs(layer, 4321 + sum(shape), init="strong_branch")
+    flags = 0 if separate else binding.NOBLE_FLAG_FUSED_BRANCH
+    got, ref = run_gpu(layer, inp, flags=flags), run_oracle(layer, inp)
+    assert_close(got, ref, "bf16", ctx=f"{shape} {'separate' if separate else 'fused'}")
+
+
+def test_fused_matches_separate():
+    # same arithmetic up to summation order: far tighter than the oracle bound
+    layer = Layer("fused", 3000, 256, 520, 128, "bf16")
+    inp = make_layer_inputs(layer, 99)
+    a = run_gpu(layer, inp, flags=binding.NOBLE_FLAG_FUSED_BRANCH)
+    b = run_gpu(layer, inp)
+    for k in a:
+        assert rel_err(a[k], b[k]) <= 2e-3, (k, rel_err(a[k], b[k]))
+
+
 @pytest.mark.parametrize("dtype", ["fp32", "bf16"])
 def test_paper_init(dtype):
     layer = Layer("paper_init", 257, 192, 264, 64, dtype)
@@ -125,6 +157,15 @@ def test_deterministic(dtype):
     layer = Layer("det", 300, 200, 264, 64, dtype)
     inp = make_layer_inputs(layer, 3)
     a, b = run_gpu(layer, inp), run_gpu(layer, inp, repeat=2)
+    for k in a:
+        assert np.array_equal(a[k], b[k]), k
+
+
+def test_deterministic_fused():
+    layer = Layer("det", 2049, 256, 520, 128, "bf16")
+    inp = make_layer_inputs(layer, 5)
+    f = binding.NOBLE_FLAG_FUSED_BRANCH
+    a, b = run_gpu(layer, inp, flags=f), run_gpu(layer, inp, repeat=3, flags=f)
     for k in a:
         assert np.array_equal(a[k], b[k]), k
 
