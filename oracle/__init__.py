@@ -24,6 +24,11 @@ import threading
 import numpy as np
 
 COSNET, IDENTITY, COS1 = 0, 1, 2
+# the other activations of the ablation (Section 4.4, Table 5): one layer
+# sigma(h) = f(h), or two layers sigma(h) = f(f(h) M), without frequency/phase
+TANH1, TANH2, LEAKY1, LEAKY2, GELU1, GELU2 = 3, 4, 5, 6, 7, 8
+MODES = {"cosnet": COSNET, "identity": IDENTITY, "cos1": COS1, "tanh1": TANH1, "tanh2": TANH2,
+         "leaky1": LEAKY1, "leaky2": LEAKY2, "gelu1": GELU1, "gelu2": GELU2}
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
 _SRC = os.path.join(_HERE, "noble_oracle.c")

@@ -21,12 +21,19 @@
  *     u2 = omega2 * b + phi2
  *     c  = cos(u2)    = sigma(h)
  *
- * Two further sigma modes pin the oracle and are the reference for the GPU's
+ * Further sigma modes pin the oracle and are the reference for the GPU's
  * bottleneck variants of the same name:
  *   ORACLE_IDENTITY: sigma(h) = h, where the branch collapses to
  *                    x (W + W_down W_up)   (the LoRA remark in Section 1 and 3.1)
  *   ORACLE_COS1:     sigma(h) = cos(omega1 * h + phi1), the single-cosine
  *                    activation of the ablation in Section 4.4 (Table 5).
+ *   ORACLE_{TANH,LEAKY,GELU}{1,2}: the other activations f of that ablation,
+ *                    one layer, sigma(h) = f(h), or two layers around the
+ *                    mixing matrix, sigma(h) = f(f(h) M).  The paper gives
+ *                    frequencies and phases to the cosine only, so these
+ *                    have none.  LeakyReLU: f(u) = u for u > 0, 0.01 u
+ *                    otherwise (the usual default slope; the paper gives
+ *                    none).  GELU: the exact form 0.5 u (1 + erf(u / sqrt 2)).
  *
  * The backward pass is the chain rule applied to the definitions above; the
  * paper trains with autograd and never writes it out.  For a scalar loss
@@ -44,6 +51,10 @@
  *     dx      = dy W^T + dh W_down^T
  *     dW      = x^T dy     dbias = sum_t dy
  *     dW_up   = c^T dy     dW_down = x^T dh
+ *
+ * With another activation f (no frequency or phase) the same chain reads
+ * du2 = f'(b) dc, db = du2, du1 = f'(h) da, dh = du1 (two layers) or
+ * dh = f'(h) dc (one layer).
  *
  * Every sum runs over its index in ascending order.  Rows (tokens) are
  * independent in the forward pass, so the only parallelism is over tokens for
@@ -64,21 +75,69 @@
 #define ORACLE_COSNET 0
 #define ORACLE_IDENTITY 1
 #define ORACLE_COS1 2
+#define ORACLE_TANH1 3
+#define ORACLE_TANH2 4
+#define ORACLE_LEAKY1 5
+#define ORACLE_LEAKY2 6
+#define ORACLE_GELU1 7
+#define ORACLE_GELU2 8
+
+#define ACT_COS 0
+#define ACT_ID 1
+#define ACT_TANH 2
+#define ACT_LEAKY 3
+#define ACT_GELU 4
+
+static int mode_act(int mode)
+{
+    switch (mode) {
+    case ORACLE_IDENTITY: return ACT_ID;
+    case ORACLE_TANH1: case ORACLE_TANH2: return ACT_TANH;
+    case ORACLE_LEAKY1: case ORACLE_LEAKY2: return ACT_LEAKY;
+    case ORACLE_GELU1: case ORACLE_GELU2: return ACT_GELU;
+    default: return ACT_COS;
+    }
+}
+
+/* 2 when sigma has the mixing matrix M (two activation layers), else 1 */
+static int mode_layers(int mode)
+{
+    return (mode == ORACLE_COSNET || mode == ORACLE_TANH2 || mode == ORACLE_LEAKY2 ||
+            mode == ORACLE_GELU2) ? 2 : 1;
+}
+
+/* activation without frequency or phase, and its derivative */
+static double act_f(int act, double u)
+{
+    switch (act) {
+    case ACT_TANH: return tanh(u);
+    case ACT_LEAKY: return u > 0.0 ? u : 0.01 * u;
+    case ACT_GELU: return 0.5 * u * (1.0 + erf(u / sqrt(2.0)));
+    default: return u;
+    }
+}
+static double act_df(int act, double u)
+{
+    switch (act) {
+    case ACT_TANH: { double t = tanh(u); return 1.0 - t * t; }
+    case ACT_LEAKY: return u > 0.0 ? 1.0 : 0.01;
+    case ACT_GELU:
+        return 0.5 * (1.0 + erf(u / sqrt(2.0))) + u * exp(-0.5 * u * u) / sqrt(2.0 * acos(-1.0));
+    default: return 1.0;
+    }
+}
 
 /* sigma for one token, Eq. 2 / Eqs. 5-7.  Writes a, b, c (each [r]).  In the
- * identity and single-cosine modes b is set equal to a (there is no M).      */
+ * one-layer modes b is set equal to a (there is no M).                       */
 static void sigma_token(int mode, int64_t r, const double *h,
                         const double *om1, const double *ph1, const double *M,
                         const double *om2, const double *ph2,
                         double *a, double *b, double *c)
 {
     int64_t i, j;
-    if (mode == ORACLE_IDENTITY) {
-        for (i = 0; i < r; ++i) { a[i] = h[i]; b[i] = h[i]; c[i] = h[i]; }
-        return;
-    }
-    for (i = 0; i < r; ++i) a[i] = cos(om1[i] * h[i] + ph1[i]);
-    if (mode == ORACLE_COS1) {
+    const int act = mode_act(mode);
+    for (i = 0; i < r; ++i) a[i] = act == ACT_COS ? cos(om1[i] * h[i] + ph1[i]) : act_f(act, h[i]);
+    if (mode_layers(mode) == 1) {
         for (i = 0; i < r; ++i) { b[i] = a[i]; c[i] = a[i]; }
         return;
     }
@@ -87,7 +146,7 @@ static void sigma_token(int mode, int64_t r, const double *h,
         for (i = 0; i < r; ++i) s += a[i] * M[i * r + j];
         b[j] = s;
     }
-    for (j = 0; j < r; ++j) c[j] = cos(om2[j] * b[j] + ph2[j]);
+    for (j = 0; j < r; ++j) c[j] = act == ACT_COS ? cos(om2[j] * b[j] + ph2[j]) : act_f(act, b[j]);
 }
 
 /*
@@ -145,8 +204,8 @@ void oracle_fwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
  *   dM [r][r], dom1/dph1/dom2/dph2 [r], dW_up [r][d_out].
  * Optional intermediates for sampled checks (each may be NULL), all [T][r]:
  *   c_out (= sigma(h)), a_out, db_out, dh_out.
- * In the identity and single-cosine modes the gradients of parameters that the
- * mode does not use are written as zero.
+ * In the modes other than CosNet the gradients of parameters that the mode
+ * does not use are written as zero.
  */
 void oracle_bwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
                 const double *x, const double *W, const double *W_down,
@@ -169,6 +228,7 @@ void oracle_bwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
     double *DB = (double *)calloc(n, sizeof(double));
     double *DH = (double *)calloc(n, sizeof(double));
     int64_t t, i, j, k, o;
+    const int act = mode_act(mode);
 
     if (r > 0) {
 #pragma omp parallel for schedule(static) private(i, j, k, o)
@@ -188,16 +248,31 @@ void oracle_bwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
                 h[k] = s;
             }
             sigma_token(mode, r, h, om1, ph1, M, om2, ph2, a, b, c);
-            for (k = 0; k < r; ++k) u1[k] = om1 ? om1[k] * h[k] + ph1[k] : 0.0;
+            for (k = 0; k < r; ++k) u1[k] = (om1 && act == ACT_COS) ? om1[k] * h[k] + ph1[k] : 0.0;
             /* dc = dy W_up^T */
             for (k = 0; k < r; ++k) {
                 double s = 0.0;
                 for (o = 0; o < d_out; ++o) s += dyt[o] * W_up[k * d_out + o];
                 dc[k] = s;
             }
-            if (mode == ORACLE_IDENTITY) {
-                /* sigma(h) = h: dh = dc */
-                for (k = 0; k < r; ++k) dh[k] = dc[k];
+            if (act != ACT_COS && mode_layers(mode) == 1) {
+                /* sigma(h) = f(h): dh = f'(h) dc (identity: dh = dc) */
+                for (k = 0; k < r; ++k) dh[k] = act_df(act, h[k]) * dc[k];
+            } else if (act != ACT_COS) {
+                /* sigma(h) = f(f(h) M) */
+                for (j = 0; j < r; ++j) {
+                    du2[j] = act_df(act, b[j]) * dc[j];
+                    db[j] = du2[j];
+                }
+                for (i = 0; i < r; ++i) {
+                    double s = 0.0;
+                    for (j = 0; j < r; ++j) s += db[j] * M[i * r + j];
+                    da[i] = s;
+                }
+                for (i = 0; i < r; ++i) {
+                    du1[i] = act_df(act, h[i]) * da[i];
+                    dh[i] = du1[i];
+                }
             } else if (mode == ORACLE_COS1) {
                 /* c = cos(u1): du1 = -sin(u1) dc, dh = omega1 du1 */
                 for (k = 0; k < r; ++k) {
@@ -282,7 +357,7 @@ void oracle_bwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
     /* dM = a^T db (zero when the mode has no M) */
     if (dM && r > 0) {
         for (i = 0; i < r * r; ++i) dM[i] = 0.0;
-        if (mode == ORACLE_COSNET)
+        if (mode_layers(mode) == 2)
             for (t = 0; t < T; ++t)
                 for (i = 0; i < r; ++i)
                     for (j = 0; j < r; ++j)
@@ -292,7 +367,7 @@ void oracle_bwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
     if (r > 0) {
         for (k = 0; k < r; ++k) {
             double so1 = 0.0, sp1 = 0.0, so2 = 0.0, sp2 = 0.0;
-            if (mode != ORACLE_IDENTITY) {
+            if (act == ACT_COS) {
                 for (t = 0; t < T; ++t) {
                     so1 += DU1[t * r + k] * H[t * r + k];
                     sp1 += DU1[t * r + k];
