@@ -236,8 +236,9 @@ def main():
                     help="workload: configuration 0-4 (default 3, the headline)")
     ap.add_argument("--workload", default="", choices=["", "geglu-base", "geglu-large"],
                     help="the paper's GeGLU FFN shapes instead of a numbered configuration")
-    ap.add_argument("--sigma", default="cosnet", choices=["cosnet", "cos1", "identity"],
-                    help="bottleneck activation (cos1, identity: the variants of the ablation)")
+    ap.add_argument("--sigma", default="cosnet",
+                    choices=["cosnet", "cos1", "identity", "tanh1", "tanh2", "leaky1", "leaky2", "gelu1", "gelu2"],
+                    help="bottleneck activation (the others: variants of the ablation, Section 4.4)")
     ap.add_argument("--fused-branch", action="store_true",
                     help="run the bottleneck inside the output GEMMs (NOBLE_FLAG_FUSED_BRANCH)")
     ap.add_argument("--per-layer", action="store_true",
@@ -277,8 +278,7 @@ def main():
         inp = make_layer_inputs(layer, layer_seed(seed_cfg, li))
         dev_inputs.append(binding.params_to_device(inp, layer.dtype))
         del inp
-        sig_flags = {"cosnet": 0, "cos1": binding.NOBLE_FLAG_SIGMA_COS1,
-                     "identity": binding.NOBLE_FLAG_SIGMA_IDENTITY}[args.sigma]
+        sig_flags = binding.SIGMA_FLAGS[args.sigma]
         if args.fused_branch:
             sig_flags |= binding.NOBLE_FLAG_FUSED_BRANCH
         bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype,

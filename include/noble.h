@@ -102,6 +102,21 @@ typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
                                     not used (may be NULL) and their
                                     gradients are written as 0.  Not together
                                     with NOBLE_FLAG_SIGMA_COS1. */
+/* The other activations f of the ablation (Section 4.4, Table 5), a 2-bit
+ * field: sigma(h) = f(f(h) M) (two layers around the mixing matrix), or with
+ * NOBLE_FLAG_SIGMA_SINGLE sigma(h) = f(h).  tanh; LeakyReLU f(u) = u for
+ * u > 0, 0.01 u otherwise (the paper gives no slope; 0.01 is the common
+ * default); GELU in its exact form u/2 (1 + erf(u / sqrt 2)).  The paper
+ * gives frequencies and phases to the cosine only: omega1, phi1, omega2, phi2
+ * are not used (may be NULL) and their gradients are written as 0; dM is
+ * written as 0 for one layer.  Not together with NOBLE_FLAG_SIGMA_IDENTITY. */
+#define NOBLE_FLAG_ACT_TANH 32u
+#define NOBLE_FLAG_ACT_LEAKYRELU 64u
+#define NOBLE_FLAG_ACT_GELU 96u
+#define NOBLE_FLAG_ACT_MASK 96u
+/* one activation layer, no mixing matrix: with the cosine (no ACT bits) the
+ * same as NOBLE_FLAG_SIGMA_COS1 */
+#define NOBLE_FLAG_SIGMA_SINGLE NOBLE_FLAG_SIGMA_COS1
 #define NOBLE_FLAG_FUSED_BRANCH 16u /* tensor-core path, CosNet bottleneck,
                                     r in {64, 128}: run the r-wide GEMM and
                                     the CosNet (forward h = x W_down^T and

@@ -23,6 +23,19 @@ NOBLE_BF16, NOBLE_FP32 = 0, 1
 NOBLE_FLAG_SIMT_ONLY, NOBLE_FLAG_INFERENCE = 1, 2
 NOBLE_FLAG_SIGMA_COS1, NOBLE_FLAG_SIGMA_IDENTITY = 4, 8
 NOBLE_FLAG_FUSED_BRANCH = 16
+NOBLE_FLAG_ACT_TANH, NOBLE_FLAG_ACT_LEAKYRELU, NOBLE_FLAG_ACT_GELU = 32, 64, 96
+NOBLE_FLAG_SIGMA_SINGLE = NOBLE_FLAG_SIGMA_COS1
+# bottleneck variants by name (Section 4.4, Table 5): flags of the descriptor
+SIGMA_FLAGS = {"cosnet": 0, "cos1": NOBLE_FLAG_SIGMA_COS1, "identity": NOBLE_FLAG_SIGMA_IDENTITY,
+               "tanh1": NOBLE_FLAG_ACT_TANH | NOBLE_FLAG_SIGMA_SINGLE, "tanh2": NOBLE_FLAG_ACT_TANH,
+               "leaky1": NOBLE_FLAG_ACT_LEAKYRELU | NOBLE_FLAG_SIGMA_SINGLE, "leaky2": NOBLE_FLAG_ACT_LEAKYRELU,
+               "gelu1": NOBLE_FLAG_ACT_GELU | NOBLE_FLAG_SIGMA_SINGLE, "gelu2": NOBLE_FLAG_ACT_GELU}
+# parameters a variant does not read (may be passed as None)
+SIGMA_UNUSED = {"cosnet": (), "cos1": ("M", "omega2", "phi2"),
+                "identity": ("omega1", "phi1", "M", "omega2", "phi2")}
+for _n in ("tanh", "leaky", "gelu"):
+    SIGMA_UNUSED[_n + "1"] = ("omega1", "phi1", "M", "omega2", "phi2")
+    SIGMA_UNUSED[_n + "2"] = ("omega1", "phi1", "omega2", "phi2")
 STATUS = {0: "NOBLE_OK", 1: "NOBLE_ERR_INVALID_ARG", 2: "NOBLE_ERR_MISALIGNED",
           3: "NOBLE_ERR_UNSUPPORTED", 4: "NOBLE_ERR_BUFFER_TOO_SMALL", 5: "NOBLE_ERR_CUDA",
           6: "NOBLE_ERR_TIMEOUT", 7: "NOBLE_ERR_NO_DEVICE"}

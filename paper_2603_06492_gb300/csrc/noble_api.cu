@@ -76,12 +76,26 @@ constexpr uint32_t kFlagInference = NOBLE_FLAG_INFERENCE;
 constexpr uint32_t kFlagSigmaCos1 = NOBLE_FLAG_SIGMA_COS1;
 constexpr uint32_t kFlagSigmaIdentity = NOBLE_FLAG_SIGMA_IDENTITY;
 constexpr uint32_t kFlagFusedBranch = NOBLE_FLAG_FUSED_BRANCH;
+constexpr uint32_t kFlagActMask = NOBLE_FLAG_ACT_MASK;
 
-// Bottleneck activation selected by the descriptor: 0 CosNet (Eq. 2), 1 single
-// cosine, 2 identity (the variants of the ablation, Section 4.4).
-int sigma_mode(const noble_linear_desc *d)
+// Bottleneck activation selected by the descriptor: CosNet (Eq. 2), or a
+// variant of the ablation (Section 4.4, Table 5): single cosine, identity, or
+// another activation with one or two layers (activations.cuh).
+struct Sigma {
+    int sig;  // tc::kSig*, the CosNet kernels' template parameter
+    int act;  // act::k*: the activation of the kSigAct* variants
+    bool two_layers() const { return tc::sig_two_layers(sig); }
+    bool first_phase() const { return sig == tc::kSigCosnet || sig == tc::kSigCos1; }  // omega1, phi1
+    bool second_phase() const { return sig == tc::kSigCosnet; }                         // omega2, phi2
+};
+Sigma sigma_of(const noble_linear_desc *d)
 {
-    return (d->flags & kFlagSigmaCos1) ? 1 : (d->flags & kFlagSigmaIdentity) ? 2 : 0;
+    if (d->flags & kFlagSigmaIdentity) return {tc::kSigIdentity, act::kIdentity};
+    const uint32_t a = d->flags & kFlagActMask;
+    const bool one = (d->flags & kFlagSigmaCos1) != 0;
+    if (a == 0) return {one ? tc::kSigCos1 : tc::kSigCosnet, act::kCos};
+    const int f = a == NOBLE_FLAG_ACT_TANH ? act::kTanh : a == NOBLE_FLAG_ACT_LEAKYRELU ? act::kLeaky : act::kGelu;
+    return {one ? tc::kSigAct1 : tc::kSigAct2, f};
 }
 
 bool rank_supported(int64_t r) { return r == 0 || r == 16 || r == 32 || r == 64 || r == 128 || r == 256; }
@@ -101,10 +115,13 @@ noble_status validate_desc(const noble_linear_desc *d)
         return fail(NOBLE_ERR_UNSUPPORTED, "r=%lld not in {0,16,32,64,128,256}", (long long)d->r);
     if (d->dtype != NOBLE_BF16 && d->dtype != NOBLE_FP32)
         return fail(NOBLE_ERR_UNSUPPORTED, "dtype %d not supported", (int)d->dtype);
-    if (d->flags & ~(kFlagSimtOnly | kFlagInference | kFlagSigmaCos1 | kFlagSigmaIdentity | kFlagFusedBranch))
+    if (d->flags &
+        ~(kFlagSimtOnly | kFlagInference | kFlagSigmaCos1 | kFlagSigmaIdentity | kFlagFusedBranch | kFlagActMask))
         return fail(NOBLE_ERR_UNSUPPORTED, "unknown flags 0x%x", d->flags);
     if ((d->flags & kFlagSigmaCos1) && (d->flags & kFlagSigmaIdentity))
         return fail(NOBLE_ERR_INVALID_ARG, "NOBLE_FLAG_SIGMA_COS1 and NOBLE_FLAG_SIGMA_IDENTITY together");
+    if ((d->flags & kFlagActMask) && (d->flags & kFlagSigmaIdentity))
+        return fail(NOBLE_ERR_INVALID_ARG, "NOBLE_FLAG_ACT_* and NOBLE_FLAG_SIGMA_IDENTITY together");
     return NOBLE_OK;
 }
 
@@ -146,7 +163,7 @@ bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->
 // backward's MN-major operands also need d_in a multiple of 64 (4-D TMA layout).
 bool fuse_fwd(const noble_linear_desc *d)
 {
-    return use_tc(d) && sigma_mode(d) == 0 && (d->r == 64 || d->r == 128) && d->T > 0 &&
+    return use_tc(d) && sigma_of(d).sig == tc::kSigCosnet && (d->r == 64 || d->r == 128) && d->T > 0 &&
            (d->flags & kFlagFusedBranch);
 }
 bool fuse_bwd(const noble_linear_desc *d) { return fuse_fwd(d) && d->d_in % 64 == 0; }
@@ -315,18 +332,18 @@ noble_status fwd_simt(const noble_linear_desc *d, const TIn *x, const TIn *W, co
         simt::Seg down{{x, di, 1}, {W_down, di, 1}, di};
         NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, down, nullptr, nullptr, h, r)));
         const int tpb = cosnet_tokens_per_block(r);
-        const int sig = sigma_mode(d);
-        if (sig == 0) {
+        const Sigma sg = sigma_of(d);
+        if (sg.two_layers()) {
             const KernelInfo ki{"simt_cosnet_fwd", kBoundAlu, 2.0 * T * r * r, 0.0};
             NOBLE_TRY(run(st, ki, [&] {
                 simt::cosnet_fwd_rows<TIn><<<(unsigned)ceil_div(T, tpb), 256, tpb * r * sizeof(float), st>>>(
-                    T, (int)r, tpb, h, om1, ph1, M, om2, ph2, b, c);
+                    T, (int)r, sg.act, tpb, h, om1, ph1, M, om2, ph2, b, c);
             }));
         } else {
             const KernelInfo ki{"simt_sigma_fwd", kBoundHbm, 0.0, (4.0 + sizeof(TIn)) * T * r};
             NOBLE_TRY(run(st, ki, [&] {
                 simt::sigma_fwd_rows<TIn><<<(unsigned)std::min<int64_t>(ceil_div(T * r, 256), 4096), 256, 0, st>>>(
-                    T * r, (int)r, sig, h, om1, ph1, c);
+                    T * r, (int)r, sg.act, h, om1, ph1, c);
             }));
         }
         simt::Seg up{{c, r, 1}, {W_up, r, 1}, r};
@@ -352,8 +369,8 @@ noble_status bwd_simt(const noble_linear_desc *d, const TIn *dy, const TIn *x, c
         float *dc = (float *)(ws + WL.dc), *a = (float *)(ws + WL.a), *db = (float *)(ws + WL.db);
         float *Mt = (float *)(ws + WL.mt), *cpart = (float *)(ws + WL.cos_part);
         float *dmpart = (float *)(ws + WL.dm_part);
-        const int sig = sigma_mode(d);
-        if (sig == 0) {
+        const Sigma sg = sigma_of(d);
+        if (sg.two_layers()) {
             const KernelInfo kt{"transpose_M", kBoundHbm, 0.0, 8.0 * r * r};
             NOBLE_TRY(run(st, kt, [&] {
                 simt::transpose_square<<<(unsigned)ceil_div(r * r, 256), 256, 0, st>>>((int)r, M, Mt);
@@ -363,21 +380,21 @@ noble_status bwd_simt(const noble_linear_desc *d, const TIn *dy, const TIn *x, c
         simt::Seg sdc{{dy, dout, 1}, {W_up, 1, r}, dout};
         NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, sdc, nullptr, nullptr, dc, r)));
         const int tpb = cosnet_tokens_per_block(r);
-        if (sig == 0) {
+        if (sg.two_layers()) {
             const KernelInfo kc{"simt_cosnet_bwd", kBoundAlu, 2.0 * T * r * r, 0.0};
             NOBLE_TRY(run(st, kc, [&] {
                 simt::cosnet_bwd_rows<TIn><<<(unsigned)WL.n_cos_blocks, 256, 5 * tpb * r * sizeof(float), st>>>(
-                    T, (int)r, tpb, h, b, dc, om1, ph1, Mt, om2, ph2, dh, a, db, cpart);
+                    T, (int)r, sg.act, tpb, h, b, dc, om1, ph1, Mt, om2, ph2, dh, a, db, cpart);
             }));
         } else {
             const KernelInfo kc{"simt_sigma_bwd", kBoundHbm, 0.0, (12.0 + sizeof(TIn)) * T * r};
             NOBLE_TRY(run(st, kc, [&] {
-                simt::sigma_bwd_rows<TIn><<<(unsigned)WL.n_cos_blocks, 256, 0, st>>>(T, (int)r, sig, tpb, h, dc,
-                                                                                    om1, ph1, dh, cpart);
+                simt::sigma_bwd_rows<TIn><<<(unsigned)WL.n_cos_blocks, 256, 0, st>>>(T, (int)r, sg.act, tpb, h,
+                                                                                    dc, om1, ph1, dh, cpart);
             }));
         }
         NOBLE_TRY(reduce(st, WL.n_cos_blocks, 4 * r, r, cpart, dom1, dph1, dom2, dph2));
-        if (sig == 0) {
+        if (sg.two_layers()) {
             // dM = a^T db, fixed token chunks
             simt::Seg sdm{{a, 1, r}, {db, 1, r}, T};
             NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
@@ -909,12 +926,17 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     tc::CosnetArgs a{};
     a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2, a.M = M;
     a.h_out = SL.only_c ? nullptr : h, a.b_out = SL.only_c ? nullptr : b, a.c_out = c;
+    const Sigma sg = sigma_of(d);
+    a.act = sg.act;
     NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
         constexpr int R = decltype(bn)::value;
-        switch (sigma_mode(d)) {
-        case 1: return cosnet_launch<R, false, tc::kSigCos1>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
-        case 2: return cosnet_launch<R, false, tc::kSigIdentity>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
-        default: return cosnet_launch<R, false, tc::kSigCosnet>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
+        const char *nm = "tc_down_cosnet_fwd";
+        switch (sg.sig) {
+        case tc::kSigCos1: return cosnet_launch<R, false, tc::kSigCos1>(st, nm, T, x, di, W_down, a);
+        case tc::kSigIdentity: return cosnet_launch<R, false, tc::kSigIdentity>(st, nm, T, x, di, W_down, a);
+        case tc::kSigAct1: return cosnet_launch<R, false, tc::kSigAct1>(st, nm, T, x, di, W_down, a);
+        case tc::kSigAct2: return cosnet_launch<R, false, tc::kSigAct2>(st, nm, T, x, di, W_down, a);
+        default: return cosnet_launch<R, false, tc::kSigCosnet>(st, nm, T, x, di, W_down, a);
         }
     }));
     const TcSeg up{c, W_up, r};
@@ -935,6 +957,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     bf16 *ones = (bf16 *)(ws + WL.ones);
     const bool fused = fuse_bwd(d);
     const bool ones_dbias = dbias && (r == 0 || fused);
+    const Sigma sg = sigma_of(d);
     if (ones_dbias) NOBLE_TRY(fill_ones(st, T * kOnesCols, ones));
     // domega1, dphi1, domega2, dphi2 (and dbias) from per-CTA or per-32-token partials
     auto reduce_cosnet = [&](const float *cpart, const float *bpart) {
@@ -971,12 +994,16 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         float *bpart = (float *)(ws + WL.bias_part);
         ca.bias_part = dbias ? bpart : nullptr;
         ca.kdim = dout;
+        ca.act = sg.act;
         NOBLE_TRY(with_rank_tile(r, [&](auto bn) {
             constexpr int R = decltype(bn)::value;
-            switch (sigma_mode(d)) {
-            case 1: return cosnet_launch<R, true, tc::kSigCos1>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
-            case 2: return cosnet_launch<R, true, tc::kSigIdentity>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
-            default: return cosnet_launch<R, true, tc::kSigCosnet>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
+            const char *nm = "tc_dc_cosnet_bwd";
+            switch (sg.sig) {
+            case tc::kSigCos1: return cosnet_launch<R, true, tc::kSigCos1>(st, nm, T, dy, dout, W_up, ca);
+            case tc::kSigIdentity: return cosnet_launch<R, true, tc::kSigIdentity>(st, nm, T, dy, dout, W_up, ca);
+            case tc::kSigAct1: return cosnet_launch<R, true, tc::kSigAct1>(st, nm, T, dy, dout, W_up, ca);
+            case tc::kSigAct2: return cosnet_launch<R, true, tc::kSigAct2>(st, nm, T, dy, dout, W_up, ca);
+            default: return cosnet_launch<R, true, tc::kSigCosnet>(st, nm, T, dy, dout, W_up, ca);
             }
         }));
         NOBLE_TRY(reduce_cosnet(cpart, dbias ? bpart : nullptr));
@@ -1034,7 +1061,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         if (r > 0) {
             add(1, ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256}, dW_down, di, false);
             add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false);
-            if (sigma_mode(d) == 0)
+            if (sg.two_layers())
                 add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);
             else if (cudaMemsetAsync(dM, 0, (size_t)r * r * 4, st) != cudaSuccess)
                 return fail(NOBLE_ERR_CUDA, "dM: %s", cudaGetErrorString(cudaGetLastError()));
@@ -1132,13 +1159,13 @@ noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, cons
     NOBLE_TRY(check_ptr(bias, "bias", true));
     NOBLE_TRY(check_ptr(y, "y", empty));
     // parameters the bottleneck variant does not use may be NULL
-    const int sig = sigma_mode(desc);
+    const Sigma sg = sigma_of(desc);
     NOBLE_TRY(check_ptr(W_down, "W_down", !br));
-    NOBLE_TRY(check_ptr(omega1, "omega1", !br || sig == 2));
-    NOBLE_TRY(check_ptr(phi1, "phi1", !br || sig == 2));
-    NOBLE_TRY(check_ptr(M, "M", !br || sig != 0));
-    NOBLE_TRY(check_ptr(omega2, "omega2", !br || sig != 0));
-    NOBLE_TRY(check_ptr(phi2, "phi2", !br || sig != 0));
+    NOBLE_TRY(check_ptr(omega1, "omega1", !br || !sg.first_phase()));
+    NOBLE_TRY(check_ptr(phi1, "phi1", !br || !sg.first_phase()));
+    NOBLE_TRY(check_ptr(M, "M", !br || !sg.two_layers()));
+    NOBLE_TRY(check_ptr(omega2, "omega2", !br || !sg.second_phase()));
+    NOBLE_TRY(check_ptr(phi2, "phi2", !br || !sg.second_phase()));
     NOBLE_TRY(check_ptr(W_up, "W_up", !br));
     NOBLE_TRY(check_ptr(saved, "saved", !br || empty));
     if (saved_bytes < saved_layout(desc).total)
@@ -1180,10 +1207,13 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, con
                             "dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2", "dW_up"};
     const void *bptr[] = {W_down, omega1, phi1, M, omega2, phi2, W_up, saved,
                           dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up};
-    const int sig = sigma_mode(desc);
+    const Sigma sg = sigma_of(desc);
     // inputs the bottleneck variant does not use may be NULL; every gradient
     // output is written (zeros for unused parameters)
-    auto unused = [&](int i) { return (sig == 2 && i >= 1 && i <= 5) || (sig == 1 && i >= 3 && i <= 5); };
+    auto unused = [&](int i) {
+        return ((i == 1 || i == 2) && !sg.first_phase()) || (i == 3 && !sg.two_layers()) ||
+               ((i == 4 || i == 5) && !sg.second_phase());
+    };
     for (int i = 0; i < 15; ++i) NOBLE_TRY(check_ptr(bptr[i], bnames[i], !br || (empty && i == 7) || unused(i)));
     if (saved_bytes < saved_layout(desc).total)
         return fail(NOBLE_ERR_BUFFER_TOO_SMALL, "saved_bytes=%zu < %zu", saved_bytes, saved_layout(desc).total);

@@ -6,7 +6,7 @@
 // so results are deterministic.
 #pragma once
 
-#include "common.cuh"
+#include "activations.cuh"
 
 namespace noble {
 namespace simt {
@@ -104,9 +104,11 @@ gemm_kernel(int64_t M, int64_t N, Seg s0, Seg s1, int nseg, const float *bias, T
 // CosNet forward on rows (Eq. 2): from h [T][r] (fp32) computes
 //   a = cos(omega1 h + phi1), b = a M, c = cos(omega2 b + phi2)
 // and writes b (fp32) and c (TOut), each [T][r].  Block: tokens_per_block rows.
+// With act != act::kCos the two-layer variant of the ablation (Section 4.4):
+// a = f(h), b = a M, c = f(b) (activations.cuh).
 template <typename TOut>
 __global__ void __launch_bounds__(256)
-cosnet_fwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const float *om1,
+cosnet_fwd_rows(int64_t T, int r, int act, int tokens_per_block, const float *h, const float *om1,
                 const float *ph1, const float *M, const float *om2, const float *ph2,
                 float *b_out, TOut *c_out)
 {
@@ -116,7 +118,10 @@ cosnet_fwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const fl
     for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
         const int tt = idx / r, i = idx % r;
         const int64_t t = t0 + tt;
-        a_s[idx] = t < T ? cosf(fmaf(om1[i], h[t * r + i], ph1[i])) : 0.f;
+        if (t >= T)
+            a_s[idx] = 0.f;
+        else
+            a_s[idx] = act == act::kCos ? cosf(fmaf(om1[i], h[t * r + i], ph1[i])) : act::f(act, h[t * r + i]);
     }
     __syncthreads();
     for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
@@ -126,31 +131,31 @@ cosnet_fwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const fl
         float s = 0.f;
         for (int i = 0; i < r; ++i) s = fmaf(a_s[tt * r + i], M[i * r + j], s);
         b_out[t * r + j] = s;
-        Elem<TOut>::store(c_out + t * r + j, cosf(fmaf(om2[j], s, ph2[j])));
+        Elem<TOut>::store(c_out + t * r + j, act == act::kCos ? cosf(fmaf(om2[j], s, ph2[j])) : act::f(act, s));
     }
 }
 
-// Single-cosine (mode 1) or identity (mode 2) bottleneck on rows, the
-// variants of the ablation (Section 4.4): c = cos(omega1 h + phi1) or c = h,
-// elementwise over h [T][r] (n = T r elements).
+// One-layer bottleneck on rows, the variants of the ablation (Section 4.4):
+// c = cos(omega1 h + phi1) (act::kCos) or c = f(h) (identity, tanh,
+// LeakyReLU, GELU; activations.cuh), elementwise over h [T][r] (n = T r).
 template <typename TOut>
 __global__ void __launch_bounds__(256)
-sigma_fwd_rows(int64_t n, int r, int mode, const float *h, const float *om1, const float *ph1, TOut *c_out)
+sigma_fwd_rows(int64_t n, int r, int act, const float *h, const float *om1, const float *ph1, TOut *c_out)
 {
     for (int64_t idx = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; idx < n; idx += (int64_t)gridDim.x * blockDim.x) {
         const int i = (int)(idx % r);
         const float v = h[idx];
-        Elem<TOut>::store(c_out + idx, mode == 1 ? cosf(fmaf(om1[i], v, ph1[i])) : v);
+        Elem<TOut>::store(c_out + idx, act == act::kCos ? cosf(fmaf(om1[i], v, ph1[i])) : act::f(act, v));
     }
 }
 
-// Backward of sigma_fwd_rows: mode 1: du1 = -sin(omega1 h + phi1) dc,
-// dh = omega1 du1; mode 2: dh = dc.  Per-block column sums over the block's
-// tokens in ascending order: part[blk][0:r] = sum du1*h, [r:2r] = sum du1,
-// [2r:4r] = 0 (no second layer).
+// Backward of sigma_fwd_rows: cosine: du1 = -sin(omega1 h + phi1) dc,
+// dh = omega1 du1; otherwise dh = f'(h) dc.  Per-block column sums over the
+// block's tokens in ascending order: part[blk][0:r] = sum du1*h,
+// [r:2r] = sum du1 (zero without a phase), [2r:4r] = 0 (no second layer).
 template <typename TOut>
 __global__ void __launch_bounds__(256)
-sigma_bwd_rows(int64_t T, int r, int mode, int tokens_per_block, const float *h, const float *dc,
+sigma_bwd_rows(int64_t T, int r, int act, int tokens_per_block, const float *h, const float *dc,
                const float *om1, const float *ph1, TOut *dh_out, float *part)
 {
     const int64_t t0 = (int64_t)blockIdx.x * tokens_per_block;
@@ -160,14 +165,14 @@ sigma_bwd_rows(int64_t T, int r, int mode, int tokens_per_block, const float *h,
         float so = 0.f, sp = 0.f;
         for (int64_t t = t0; t < t1; ++t) {
             const float d = dc[t * r + j];
-            if (mode == 1) {
-                const float hv = h[t * r + j];
+            const float hv = h[t * r + j];
+            if (act == act::kCos) {
                 const float du1 = -sinf(fmaf(om1[j], hv, ph1[j])) * d;
                 Elem<TOut>::store(dh_out + t * r + j, om1[j] * du1);
                 so += du1 * hv;
                 sp += du1;
             } else {
-                Elem<TOut>::store(dh_out + t * r + j, d);
+                Elem<TOut>::store(dh_out + t * r + j, act::df(act, hv) * d);
             }
         }
         pb[j] = so;
@@ -184,13 +189,16 @@ sigma_bwd_rows(int64_t T, int r, int mode, int tokens_per_block, const float *h,
 // writing dh (TOut), a and db (fp32) [T][r], and per-block column sums
 //   part[blk][0:r] = sum du1*h, [r:2r] = sum du1, [2r:3r] = sum du2*b,
 //   [3r:4r] = sum du2      (tokens of the block in ascending order).
+// With act != act::kCos (two-layer variant f(f(h) M)): db = f'(b) dc,
+// du1 = f'(h) da, dh = du1, a = f(h), and the sums are zero.
 template <typename TOut>
 __global__ void __launch_bounds__(256)
-cosnet_bwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const float *b,
+cosnet_bwd_rows(int64_t T, int r, int act, int tokens_per_block, const float *h, const float *b,
                 const float *dc, const float *om1, const float *ph1, const float *Mt,
                 const float *om2, const float *ph2, TOut *dh_out, float *a_out, float *db_out,
                 float *part)
 {
+    const bool cosine = act == act::kCos;
     extern __shared__ float sm[];
     const int n = tokens_per_block * r;
     float *db_s = sm, *du2_s = sm + n, *p2_s = sm + 2 * n, *du1_s = sm + 3 * n, *p1_s = sm + 4 * n;
@@ -201,12 +209,12 @@ cosnet_bwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const fl
         float du2 = 0.f, bv = 0.f;
         if (t < T) {
             bv = b[t * r + j];
-            du2 = -sinf(fmaf(om2[j], bv, ph2[j])) * dc[t * r + j];
+            du2 = (cosine ? -sinf(fmaf(om2[j], bv, ph2[j])) : act::df(act, bv)) * dc[t * r + j];
         }
-        const float dbv = om2[j] * du2;
+        const float dbv = cosine ? om2[j] * du2 : du2;
         db_s[idx] = dbv;
-        du2_s[idx] = du2;
-        p2_s[idx] = du2 * bv;
+        du2_s[idx] = cosine ? du2 : 0.f;
+        p2_s[idx] = cosine ? du2 * bv : 0.f;
         if (t < T) db_out[t * r + j] = dbv;
     }
     __syncthreads();
@@ -218,12 +226,17 @@ cosnet_bwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const fl
             float da = 0.f;
             for (int j = 0; j < r; ++j) da = fmaf(db_s[tt * r + j], Mt[j * r + i], da);
             hv = h[t * r + i];
-            const float u1 = fmaf(om1[i], hv, ph1[i]);
-            float s1, c1;
-            sincosf(u1, &s1, &c1);
-            du1 = -s1 * da;
-            a_out[t * r + i] = c1;
-            Elem<TOut>::store(dh_out + t * r + i, om1[i] * du1);
+            if (cosine) {
+                const float u1 = fmaf(om1[i], hv, ph1[i]);
+                float s1, c1;
+                sincosf(u1, &s1, &c1);
+                du1 = -s1 * da;
+                a_out[t * r + i] = c1;
+                Elem<TOut>::store(dh_out + t * r + i, om1[i] * du1);
+            } else {
+                a_out[t * r + i] = act::f(act, hv);
+                Elem<TOut>::store(dh_out + t * r + i, act::df(act, hv) * da);
+            }
         }
         du1_s[idx] = du1;
         p1_s[idx] = du1 * hv;

@@ -27,6 +27,7 @@
 // tokens of the frequency and phase gradients do not average away.
 #pragma once
 
+#include "activations.cuh"
 #include "tc_gemm.cuh"
 
 namespace noble {
@@ -48,6 +49,7 @@ struct CosnetArgs {
     // [gridDim.x][kdim], accumulated from the dy tiles of the main loop
     float *bias_part;
     int64_t kdim;
+    int act;             // kSigAct1 / kSigAct2: the activation (act::kTanh, kLeaky, kGelu)
     uint32_t *status;
 };
 
@@ -261,12 +263,17 @@ __device__ __forceinline__ uint32_t cta_rank_in_cluster()
     return r;
 }
 
-// Bottleneck activation of the kernel: the CosNet of Eq. 2 (default), or two
+// Bottleneck activation of the kernel: the CosNet of Eq. 2 (default), or the
 // variants of the ablation in Section 4.4 (Table 5): a single cosine
-// sigma(h) = cos(omega1 h + phi1), and the identity sigma(h) = h (the linear
-// collapse of Sections 1 and 3.1).  The variants have no mixing matrix, so
-// their epilogue ends after the first accumulator.
-constexpr int kSigCosnet = 0, kSigCos1 = 1, kSigIdentity = 2;
+// sigma(h) = cos(omega1 h + phi1); the identity sigma(h) = h (the linear
+// collapse of Sections 1 and 3.1); another activation f (activations.cuh,
+// chosen at run time by CosnetArgs::act), one layer sigma(h) = f(h) or two
+// layers sigma(h) = f(f(h) M).  The one-layer variants have no mixing matrix,
+// so their epilogue ends after the first accumulator; the two-layer ones run
+// the CosNet epilogue with f in place of the cosines and no frequencies or
+// phases (their partial sums are written as zeros).
+constexpr int kSigCosnet = 0, kSigCos1 = 1, kSigIdentity = 2, kSigAct1 = 3, kSigAct2 = 4;
+__host__ __device__ constexpr bool sig_two_layers(int sig) { return sig == kSigCosnet || sig == kSigAct2; }
 
 template <int R, bool BWD, int SIG = kSigCosnet>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kCosnetThreads, 1)
@@ -453,7 +460,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
         };
         // the first pass's part of M is read while the main loop runs
-        if constexpr (SIG == kSigCosnet) m_load(0);
+        if constexpr (sig_two_layers(SIG)) m_load(0);
         if constexpr (BWD) {
             // the tile's saved h and b rows are read after the main loop: bring
             // them into L2 meanwhile
@@ -518,9 +525,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ok = ptx::named_barrier_and(3, 256, ok);  // uniform over the epilogue warps
         if (ok) {
             // the ring is free once the main accumulator is complete
-            if constexpr (SIG == kSigCosnet) m_store(0);
+            if constexpr (sig_two_layers(SIG)) m_store(0);
             ptx::tc_fence_after();
-            if constexpr (SIG != kSigCosnet) {
+            if constexpr (!sig_two_layers(SIG)) {
                 // single-cosine or identity bottleneck: c (forward) or dh
                 // (backward) straight from the first accumulator
 #pragma unroll 1
@@ -553,7 +560,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                             for (int i = 0; i < 8; ++i) {
                                 const int k = c + 8 * g + i;
-                                cc[i] = SIG == kSigCos1 ? cos_reduced(fmaf(om1[k], v[8 * g + i], ph1[k])) : v[8 * g + i];
+                                cc[i] = SIG == kSigCos1   ? cos_reduced(fmaf(om1[k], v[8 * g + i], ph1[k]))
+                                        : SIG == kSigAct1 ? act::f(args.act, v[8 * g + i])
+                                                          : v[8 * g + i];
                             }
 #pragma unroll
                             for (int q = 0; q < 4; ++q) wc[g][q] = ptx::pack_bf16x2(cc[2 * q], cc[2 * q + 1]);
@@ -561,11 +570,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         store_segments<W / 8>(wc, args.c_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                     } else {
                         // v = dc; single cosine: du1 = -sin(omega1 h + phi1) dc,
-                        // dh = omega1 du1; identity: dh = dc
+                        // dh = omega1 du1; one-layer f: dh = f'(h) dc; identity: dh = dc
                         float hv[32];
 #pragma unroll
                         for (int i = 0; i < 32; ++i) hv[i] = 0.f;
-                        if constexpr (SIG == kSigCos1) {
+                        if constexpr (SIG == kSigCos1 || SIG == kSigAct1) {
                             uint32_t w[W / 4][4];
                             load_segments<W / 4>(w, args.h_in + t0 * R + c, (int64_t)R * 4, t0, args.T);
 #pragma unroll
@@ -587,6 +596,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                                 if constexpr (SIG == kSigCos1) {
                                     du1 = live ? -sin_reduced(fmaf(om1[k], hv[j], ph1[k])) * v[j] : 0.f;
                                     dh[i] = om1[k] * du1;
+                                } else if constexpr (SIG == kSigAct1) {
+                                    dh[i] = live ? act::df(args.act, hv[j]) * v[j] : 0.f;
                                 } else {
                                     dh[i] = live ? v[j] : 0.f;
                                 }
@@ -637,7 +648,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const int k = c + 8 * g + i;
-                            o[i] = cos_reduced(fmaf(om1[k], v[8 * g + i], ph1[k]));
+                            o[i] = SIG == kSigAct2 ? act::f(args.act, v[8 * g + i])
+                                                   : cos_reduced(fmaf(om1[k], v[8 * g + i], ph1[k]));
                         }
                         store_hi_lo(tile, row, c + 8 * g, o);
                     }
@@ -664,10 +676,17 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const int k = c + 8 * g + i, j = 8 * g + i;
-                            const float du2 = live ? -sin_reduced(fmaf(om2[k], bv[j], ph2[k])) * v[j] : 0.f;
-                            o[i] = om2[k] * du2;
-                            q2[j] = du2 * bv[j];
-                            q3[j] = du2;
+                            if constexpr (SIG == kSigAct2) {
+                                // f(b): db = f'(b) dc, no frequency or phase
+                                o[i] = live ? act::df(args.act, bv[j]) * v[j] : 0.f;
+                                q2[j] = 0.f;
+                                q3[j] = 0.f;
+                            } else {
+                                const float du2 = live ? -sin_reduced(fmaf(om2[k], bv[j], ph2[k])) * v[j] : 0.f;
+                                o[i] = om2[k] * du2;
+                                q2[j] = du2 * bv[j];
+                                q3[j] = du2;
+                            }
                         }
                         const uint4 q = store_hi_lo(tile, row, c + 8 * g, o);
                         wdb[g][0] = q.x, wdb[g][1] = q.y, wdb[g][2] = q.z, wdb[g][3] = q.w;
@@ -724,13 +743,13 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             if (threadIdx.x == 64) ptx::mma_commit(mma2_done);
             const bool done = ptx::mbar_wait(mma2_done, 0, args.status);
             ok = ptx::named_barrier_and(3, 256, ok && done);
-            }  // SIG == kSigCosnet
+            }  // two layers
         }
         if (ok) {
             ptx::tc_fence_after();
             // ---- phase 2: second accumulator
 #pragma unroll 1
-            for (int c = 32 * half; SIG == kSigCosnet && c < R; c += 64) {
+            for (int c = 32 * half; sig_two_layers(SIG) && c < R; c += 64) {
                 float v[32];
                 if constexpr (R >= 32) {
                     ptx::tmem_ld_32x32b_x32(acc2 + c, v);
@@ -748,7 +767,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     for (int g = 0; g < W / 8; ++g) {
                         float cc[8];
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) cc[i] = cos_reduced(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
+                        for (int i = 0; i < 8; ++i)
+                            cc[i] = SIG == kSigAct2 ? act::f(args.act, v[8 * g + i])
+                                                    : cos_reduced(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
 #pragma unroll
                         for (int q = 0; q < 4; ++q) wc[g][q] = ptx::pack_bf16x2(cc[2 * q], cc[2 * q + 1]);
                     }
@@ -784,13 +805,21 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                         for (int i = 0; i < 8; ++i) {
                             const int k = c + 8 * g + i, j = 8 * g + i;
-                            float s1, c1;
-                            sincos_reduced(fmaf(om1[k], hv[j], ph1[k]), &s1, &c1);
-                            const float du1 = live ? -s1 * v[j] : 0.f;
-                            dh[i] = om1[k] * du1;
-                            av[i] = c1;
-                            q0[j] = du1 * hv[j];
-                            q1[j] = du1;
+                            if constexpr (SIG == kSigAct2) {
+                                // f(h): dh = f'(h) da, a = f(h)
+                                dh[i] = live ? act::df(args.act, hv[j]) * v[j] : 0.f;
+                                av[i] = act::f(args.act, hv[j]);
+                                q0[j] = 0.f;
+                                q1[j] = 0.f;
+                            } else {
+                                float s1, c1;
+                                sincos_reduced(fmaf(om1[k], hv[j], ph1[k]), &s1, &c1);
+                                const float du1 = live ? -s1 * v[j] : 0.f;
+                                dh[i] = om1[k] * du1;
+                                av[i] = c1;
+                                q0[j] = du1 * hv[j];
+                                q1[j] = du1;
+                            }
                         }
 #pragma unroll
                         for (int q = 0; q < 4; ++q) {

@@ -170,3 +170,27 @@ def test_adamw_arguments_validated(lib):
     with pytest.raises(binding.NobleError) as e:
         binding.noble_adamw_step([t], lr=1e-3, beta2=1.0)
     assert e.value.status == 1
+
+
+def test_activation_flags(lib):
+    # ACT_* with the identity is rejected; the other combinations validate and
+    # reach the device check (no GPU here), with the pointers a variant does
+    # not read passed as NULL
+    import torch
+    bad = binding.make_desc(256, 128, 128, 16, "bf16",
+                            binding.NOBLE_FLAG_ACT_GELU | binding.NOBLE_FLAG_SIGMA_IDENTITY)
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(bad)
+    assert e.value.status == 1
+    if torch.cuda.is_available():
+        pytest.skip("device present")
+    for name, flags in binding.SIGMA_FLAGS.items():
+        d = binding.make_desc(256, 128, 128, 16, "bf16", flags)
+        unused = {k: None for k in binding.SIGMA_UNUSED[name]}
+        with pytest.raises(binding.NobleError) as e:
+            _fwd(d, **unused)
+        assert e.value.status == 7, name
+    # a two-layer variant needs M
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(binding.make_desc(256, 128, 128, 16, "bf16", binding.NOBLE_FLAG_ACT_TANH), M=None)
+    assert e.value.status == 1
