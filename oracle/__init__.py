@@ -60,6 +60,10 @@ def _load():
             lib.oracle_fwd.restype = None
             lib.oracle_bwd.argtypes = [ctypes.c_int, i64, i64, i64, i64] + [p] * 24
             lib.oracle_bwd.restype = None
+            lib.oracle_fwd3.argtypes = [i64, i64, i64, i64] + [p] * 18
+            lib.oracle_fwd3.restype = None
+            lib.oracle_bwd3.argtypes = [i64, i64, i64, i64] + [p] * 26
+            lib.oracle_bwd3.restype = None
             lib.oracle_outer_elems.argtypes = [i64, p, i64, p, i64, i64, p, p, p]
             lib.oracle_outer_elems.restype = None
             _lib = lib
@@ -136,6 +140,46 @@ def bwd(x, W, W_down, omega1, phi1, M, omega2, phi2, W_up, dy, mode=COSNET,
     if want_intermediates:
         res.update(inter)
     return res
+
+
+# the three-layer cosine (Section 4.4, Table 5), with M2 [r,r], omega3, phi3 [r]
+PARAMS3 = ("W_down", "omega1", "phi1", "M", "omega2", "phi2", "M2", "omega3", "phi3", "W_up")
+GRAD_NAMES3 = ("dx", "dW", "dbias", "dW_down", "dM", "domega1", "dphi1", "domega2", "dphi2",
+               "dM2", "domega3", "dphi3", "dW_up")
+
+
+def fwd3(x, W, bias, p, want_intermediates=False):
+    """Forward with the three-layer cosine; ``p`` maps the names of PARAMS3
+    (paper orientation) to arrays.  Returns y, or (y, h, b, b2, c)."""
+    lib = _load()
+    x, W, bias = _c(x), _c(W), _c(bias)
+    T, d_in = x.shape
+    d_out = W.shape[1]
+    r = np.asarray(p["W_down"]).shape[1]
+    q = [_c(p[k]) for k in PARAMS3]
+    y = np.empty((T, d_out))
+    inter = [np.empty((T, r)) if want_intermediates else None for _ in range(4)]
+    lib.oracle_fwd3(T, d_in, d_out, r, _ptr(x), _ptr(W), _ptr(bias), *[_ptr(a) for a in q], _ptr(y),
+                    *[_ptr(a) for a in inter])
+    return (y, *inter) if want_intermediates else y
+
+
+def bwd3(x, W, p, dy):
+    """Backward of ``L = sum(y * dy)`` with the three-layer cosine; returns a
+    dict over GRAD_NAMES3, each in the orientation of its parameter."""
+    lib = _load()
+    x, W, dy = _c(x), _c(W), _c(dy)
+    T, d_in = x.shape
+    d_out = W.shape[1]
+    r = np.asarray(p["W_down"]).shape[1]
+    q = [_c(p[k]) for k in PARAMS3]
+    shapes = {"dx": (T, d_in), "dW": (d_in, d_out), "dbias": (d_out,), "dW_down": (d_in, r),
+              "dM": (r, r), "domega1": (r,), "dphi1": (r,), "domega2": (r,), "dphi2": (r,),
+              "dM2": (r, r), "domega3": (r,), "dphi3": (r,), "dW_up": (r, d_out)}
+    out = {k: np.empty(shapes[k]) for k in GRAD_NAMES3}
+    lib.oracle_bwd3(T, d_in, d_out, r, _ptr(x), _ptr(W), *[_ptr(a) for a in q], _ptr(dy),
+                    *[_ptr(out[k]) for k in GRAD_NAMES3])
+    return out
 
 
 def outer_elems(P, Q, rows, cols):

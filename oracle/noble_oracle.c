@@ -394,6 +394,212 @@ void oracle_bwd(int mode, int64_t T, int64_t d_in, int64_t d_out, int64_t r,
 }
 
 /*
+ * Three-layer cosine bottleneck, the deepest row of the ablation in
+ * Section 4.4 (Table 5): CosNet with a second mixing matrix and a third
+ * cosine,
+ *     a  = cos(omega1 h + phi1),  b  = a M,
+ *     a2 = cos(omega2 b + phi2),  b2 = a2 M2,
+ *     c  = cos(omega3 b2 + phi3),  y = x W + bias + c W_up,
+ * M2 [r][r] with b2_j = sum_i a2_i M2[i][j], omega3 and phi3 [r].  The
+ * backward continues the chain rule of oracle_bwd one layer further:
+ *     du3 = -sin(u3) dc,  domega3 = sum_t du3 b2,  dphi3 = sum_t du3,
+ *     db2 = omega3 du3,   dM2 = sum_t a2^T db2,   da2 = db2 M2^T,
+ *     du2 = -sin(u2) da2, domega2 = sum_t du2 b,   dphi2 = sum_t du2,
+ *     db  = omega2 du2,   dM = sum_t a^T db,       da = db M^T,
+ *     du1 = -sin(u1) da,  domega1 = sum_t du1 h,   dphi1 = sum_t du1,
+ *     dh  = omega1 du1,   and dx, dW, dbias, dW_up, dW_down as in oracle_bwd.
+ * Kept apart from oracle_fwd / oracle_bwd (extra parameters); sums run in
+ * ascending order.  Any output pointer may be NULL.
+ */
+static void cos3_token(int64_t r, const double *h, const double *om1, const double *ph1,
+                       const double *M, const double *om2, const double *ph2, const double *M2,
+                       const double *om3, const double *ph3, double *a, double *b, double *a2,
+                       double *b2, double *c)
+{
+    int64_t i, j;
+    for (i = 0; i < r; ++i) a[i] = cos(om1[i] * h[i] + ph1[i]);
+    for (j = 0; j < r; ++j) {
+        double s = 0.0;
+        for (i = 0; i < r; ++i) s += a[i] * M[i * r + j];
+        b[j] = s;
+    }
+    for (i = 0; i < r; ++i) a2[i] = cos(om2[i] * b[i] + ph2[i]);
+    for (j = 0; j < r; ++j) {
+        double s = 0.0;
+        for (i = 0; i < r; ++i) s += a2[i] * M2[i * r + j];
+        b2[j] = s;
+    }
+    for (j = 0; j < r; ++j) c[j] = cos(om3[j] * b2[j] + ph3[j]);
+}
+
+void oracle_fwd3(int64_t T, int64_t d_in, int64_t d_out, int64_t r, const double *x, const double *W,
+                 const double *bias, const double *W_down, const double *om1, const double *ph1,
+                 const double *M, const double *om2, const double *ph2, const double *M2,
+                 const double *om3, const double *ph3, const double *W_up, double *y, double *h_out,
+                 double *b_out, double *b2_out, double *c_out)
+{
+    int64_t t;
+#pragma omp parallel for schedule(static)
+    for (t = 0; t < T; ++t) {
+        const double *xt = x + t * d_in;
+        double *h = (double *)malloc(sizeof(double) * 6 * r);
+        double *a = h + r, *b = a + r, *a2 = b + r, *b2 = a2 + r, *c = b2 + r;
+        int64_t i, k, o;
+        for (k = 0; k < r; ++k) {
+            double s = 0.0;
+            for (i = 0; i < d_in; ++i) s += xt[i] * W_down[i * r + k];
+            h[k] = s;
+        }
+        cos3_token(r, h, om1, ph1, M, om2, ph2, M2, om3, ph3, a, b, a2, b2, c);
+        if (h_out) memcpy(h_out + t * r, h, sizeof(double) * r);
+        if (b_out) memcpy(b_out + t * r, b, sizeof(double) * r);
+        if (b2_out) memcpy(b2_out + t * r, b2, sizeof(double) * r);
+        if (c_out) memcpy(c_out + t * r, c, sizeof(double) * r);
+        for (o = 0; o < d_out; ++o) {
+            double s = 0.0, br = 0.0;
+            for (i = 0; i < d_in; ++i) s += xt[i] * W[i * d_out + o];
+            if (bias) s = s + bias[o];
+            for (k = 0; k < r; ++k) br += c[k] * W_up[k * d_out + o];
+            y[t * d_out + o] = s + br;
+        }
+        free(h);
+    }
+}
+
+void oracle_bwd3(int64_t T, int64_t d_in, int64_t d_out, int64_t r, const double *x, const double *W,
+                 const double *W_down, const double *om1, const double *ph1, const double *M,
+                 const double *om2, const double *ph2, const double *M2, const double *om3,
+                 const double *ph3, const double *W_up, const double *dy, double *dx, double *dW,
+                 double *dbias, double *dW_down, double *dM, double *dom1, double *dph1, double *dom2,
+                 double *dph2, double *dM2, double *dom3, double *dph3, double *dW_up)
+{
+    const size_t n = (size_t)T * (size_t)r;
+    /* per-token intermediates [T][r] */
+    double *H = (double *)calloc(n, sizeof(double)), *A = (double *)calloc(n, sizeof(double));
+    double *B = (double *)calloc(n, sizeof(double)), *A2 = (double *)calloc(n, sizeof(double));
+    double *B2 = (double *)calloc(n, sizeof(double)), *C = (double *)calloc(n, sizeof(double));
+    double *DU1 = (double *)calloc(n, sizeof(double)), *DU2 = (double *)calloc(n, sizeof(double));
+    double *DU3 = (double *)calloc(n, sizeof(double)), *DB = (double *)calloc(n, sizeof(double));
+    double *DB2 = (double *)calloc(n, sizeof(double)), *DH = (double *)calloc(n, sizeof(double));
+    int64_t t, i, j, k, o;
+#pragma omp parallel for schedule(static) private(i, j, k, o)
+    for (t = 0; t < T; ++t) {
+        const double *xt = x + t * d_in, *dyt = dy + t * d_out;
+        double *h = H + t * r, *a = A + t * r, *b = B + t * r, *a2 = A2 + t * r, *b2 = B2 + t * r;
+        double *c = C + t * r, *du1 = DU1 + t * r, *du2 = DU2 + t * r, *du3 = DU3 + t * r;
+        double *db = DB + t * r, *db2 = DB2 + t * r, *dh = DH + t * r;
+        double *dc = (double *)malloc(sizeof(double) * 3 * r);
+        double *da2 = dc + r, *da = da2 + r;
+        for (k = 0; k < r; ++k) {
+            double s = 0.0;
+            for (i = 0; i < d_in; ++i) s += xt[i] * W_down[i * r + k];
+            h[k] = s;
+        }
+        cos3_token(r, h, om1, ph1, M, om2, ph2, M2, om3, ph3, a, b, a2, b2, c);
+        for (k = 0; k < r; ++k) {
+            double s = 0.0;
+            for (o = 0; o < d_out; ++o) s += dyt[o] * W_up[k * d_out + o];
+            dc[k] = s;
+        }
+        for (j = 0; j < r; ++j) {
+            du3[j] = -sin(om3[j] * b2[j] + ph3[j]) * dc[j];
+            db2[j] = om3[j] * du3[j];
+        }
+        for (i = 0; i < r; ++i) {
+            double s = 0.0;
+            for (j = 0; j < r; ++j) s += db2[j] * M2[i * r + j];
+            da2[i] = s;
+        }
+        for (j = 0; j < r; ++j) {
+            du2[j] = -sin(om2[j] * b[j] + ph2[j]) * da2[j];
+            db[j] = om2[j] * du2[j];
+        }
+        for (i = 0; i < r; ++i) {
+            double s = 0.0;
+            for (j = 0; j < r; ++j) s += db[j] * M[i * r + j];
+            da[i] = s;
+        }
+        for (i = 0; i < r; ++i) {
+            du1[i] = -sin(om1[i] * h[i] + ph1[i]) * da[i];
+            dh[i] = om1[i] * du1[i];
+        }
+        free(dc);
+    }
+    if (dx) {
+#pragma omp parallel for schedule(static) private(i, k, o)
+        for (t = 0; t < T; ++t)
+            for (i = 0; i < d_in; ++i) {
+                double s = 0.0, sb = 0.0;
+                for (o = 0; o < d_out; ++o) s += dy[t * d_out + o] * W[i * d_out + o];
+                for (k = 0; k < r; ++k) sb += DH[t * r + k] * W_down[i * r + k];
+                dx[t * d_in + i] = s + sb;
+            }
+    }
+    if (dW) {
+#pragma omp parallel for schedule(static) private(t, o)
+        for (i = 0; i < d_in; ++i) {
+            double *row = dW + i * d_out;
+            for (o = 0; o < d_out; ++o) row[o] = 0.0;
+            for (t = 0; t < T; ++t)
+                for (o = 0; o < d_out; ++o) row[o] += x[t * d_in + i] * dy[t * d_out + o];
+        }
+    }
+    if (dbias) {
+        for (o = 0; o < d_out; ++o) dbias[o] = 0.0;
+        for (t = 0; t < T; ++t)
+            for (o = 0; o < d_out; ++o) dbias[o] += dy[t * d_out + o];
+    }
+    if (dW_up) {
+#pragma omp parallel for schedule(static) private(t, o)
+        for (k = 0; k < r; ++k) {
+            double *row = dW_up + k * d_out;
+            for (o = 0; o < d_out; ++o) row[o] = 0.0;
+            for (t = 0; t < T; ++t)
+                for (o = 0; o < d_out; ++o) row[o] += C[t * r + k] * dy[t * d_out + o];
+        }
+    }
+    if (dW_down) {
+#pragma omp parallel for schedule(static) private(t, k)
+        for (i = 0; i < d_in; ++i) {
+            double *row = dW_down + i * r;
+            for (k = 0; k < r; ++k) row[k] = 0.0;
+            for (t = 0; t < T; ++t)
+                for (k = 0; k < r; ++k) row[k] += x[t * d_in + i] * DH[t * r + k];
+        }
+    }
+    /* dM = a^T db, dM2 = a2^T db2 */
+    for (i = 0; i < r * r; ++i) {
+        if (dM) dM[i] = 0.0;
+        if (dM2) dM2[i] = 0.0;
+    }
+    for (t = 0; t < T; ++t)
+        for (i = 0; i < r; ++i)
+            for (j = 0; j < r; ++j) {
+                if (dM) dM[i * r + j] += A[t * r + i] * DB[t * r + j];
+                if (dM2) dM2[i * r + j] += A2[t * r + i] * DB2[t * r + j];
+            }
+    for (k = 0; k < r; ++k) {
+        double s[6] = {0.0, 0.0, 0.0, 0.0, 0.0, 0.0};
+        for (t = 0; t < T; ++t) {
+            s[0] += DU1[t * r + k] * H[t * r + k];
+            s[1] += DU1[t * r + k];
+            s[2] += DU2[t * r + k] * B[t * r + k];
+            s[3] += DU2[t * r + k];
+            s[4] += DU3[t * r + k] * B2[t * r + k];
+            s[5] += DU3[t * r + k];
+        }
+        if (dom1) dom1[k] = s[0];
+        if (dph1) dph1[k] = s[1];
+        if (dom2) dom2[k] = s[2];
+        if (dph2) dph2[k] = s[3];
+        if (dom3) dom3[k] = s[4];
+        if (dph3) dph3[k] = s[5];
+    }
+    free(H); free(A); free(B); free(A2); free(B2); free(C);
+    free(DU1); free(DU2); free(DU3); free(DB); free(DB2); free(DH);
+}
+
+/*
  * Selected elements of a token-summed outer product:
  *     out[p] = sum_t P[t][rows[p]] * Q[t][cols[p]]     (ascending t)
  * P is [T][p_ld], Q is [T][q_ld].  This is the definition of one element of a
