@@ -210,14 +210,16 @@ def test_pins_catch_planted_mistakes(tmp_path):
     import subprocess
     src = open(os.path.join(os.path.dirname(oracle.__file__), "noble_oracle.c")).read()
     mistakes = {
-        "transposed M": ("s += a[i] * M[i * r + j];", "s += a[i] * M[j * r + i];"),
+        "transposed M": ("s += a[i] * M[i * r + j];\n        b[j] = s;\n    }\n    for (j = 0; j < r; ++j) c[j]",
+                         "s += a[i] * M[j * r + i];\n        b[j] = s;\n    }\n    for (j = 0; j < r; ++j) c[j]"),
         "phase sign": ("cos(om2[j] * b[j] + ph2[j])", "cos(om2[j] * b[j] - ph2[j])"),
         "dropped sin sign": ("du1[i] = -sin(u1[i]) * da[i];", "du1[i] = sin(u1[i]) * da[i];"),
         "da uses M not M^T": ("s += db[j] * M[i * r + j];\n                    da[i] = s;\n                }\n"
                               "                for (i = 0; i < r; ++i) {\n                    du1[i] = -sin",
                               "s += db[j] * M[j * r + i];\n                    da[i] = s;\n                }\n"
                               "                for (i = 0; i < r; ++i) {\n                    du1[i] = -sin"),
-        "dropped dh term": ("dx[t * d_in + i] = s + sb;", "dx[t * d_in + i] = s;"),
+        "dropped dh term": ("dx[t * d_in + i] = s + sb;\n            }\n        }\n",
+                            "dx[t * d_in + i] = s;\n            }\n        }\n"),
     }
     p, e = _golden()
     for name, (old, new) in mistakes.items():
