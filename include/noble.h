@@ -117,6 +117,14 @@ typedef enum { NOBLE_BF16 = 0, NOBLE_FP32 = 1 } noble_dtype;
 /* one activation layer, no mixing matrix: with the cosine (no ACT bits) the
  * same as NOBLE_FLAG_SIGMA_COS1 */
 #define NOBLE_FLAG_SIGMA_SINGLE NOBLE_FLAG_SIGMA_COS1
+/* The three-layer cosine of the ablation (Section 4.4, Table 5): CosNet with a
+ * second mixing matrix and a third cosine,
+ *     a2 = cos(omega2 b + phi2), b2 = a2 M2, c = cos(omega3 b2 + phi3),
+ * b2_j = sum_i a2_i M2[i][j].  It has parameters the other variants lack, so
+ * only noble_linear_fwd_cos3 / noble_linear_bwd_cos3 accept it (and they
+ * accept nothing else); saved holds h, b, b2 (fp32) and c.  Not together with
+ * another NOBLE_FLAG_SIGMA_* or NOBLE_FLAG_ACT_* bit. */
+#define NOBLE_FLAG_SIGMA_COS3 128u
 #define NOBLE_FLAG_FUSED_BRANCH 16u /* tensor-core path, CosNet bottleneck,
                                     r in {64, 128}: run the r-wide GEMM and
                                     the CosNet (forward h = x W_down^T and
@@ -274,6 +282,51 @@ noble_status noble_linear_lr_multipliers(const noble_linear_desc *desc, float ga
  *    results; the caller must order them, e.g. on a single stream.
  */
 #define NOBLE_NOALLOC_SCRATCH_BYTES (64u << 20)
+/*
+ * Three-layer cosine bottleneck (NOBLE_FLAG_SIGMA_COS3): the extra parameters
+ * M2 [r][r], omega3, phi3 [r] (fp32, device) and their gradients.  All are
+ * required (not NULL) when r > 0.
+ */
+typedef struct {
+    const float *M2;
+    const float *omega3;
+    const float *phi3;
+} noble_cos3_params;
+typedef struct {
+    float *dM2;
+    float *domega3;
+    float *dphi3;
+} noble_cos3_grads;
+
+/* noble_linear_fwd for a NOBLE_FLAG_SIGMA_COS3 descriptor; the other
+ * arguments as there.  Errors as noble_linear_fwd, and NOBLE_ERR_INVALID_ARG
+ * for a descriptor without the flag. */
+noble_status noble_linear_fwd_cos3(const noble_linear_desc *desc, const void *x,
+                                   const void *W, const float *bias,
+                                   const void *W_down, const float *omega1,
+                                   const float *phi1, const float *M,
+                                   const float *omega2, const float *phi2,
+                                   const noble_cos3_params *p3, const void *W_up,
+                                   void *y, void *saved, size_t saved_bytes,
+                                   noble_stream stream);
+
+/* noble_linear_bwd for a NOBLE_FLAG_SIGMA_COS3 descriptor, also writing
+ * g3->dM2 = sum_t a2^T db2, g3->domega3, g3->dphi3 (overwritten).  The
+ * workspace size is noble_linear_bwd_workspace_bytes of the same descriptor. */
+noble_status noble_linear_bwd_cos3(const noble_linear_desc *desc, const void *dy,
+                                   const void *x, const void *W,
+                                   const void *W_down, const float *omega1,
+                                   const float *phi1, const float *M,
+                                   const float *omega2, const float *phi2,
+                                   const noble_cos3_params *p3, const void *W_up,
+                                   const void *saved, size_t saved_bytes, void *dx,
+                                   float *dW, float *dbias, float *dW_down,
+                                   float *dM, float *domega1, float *dphi1,
+                                   float *domega2, float *dphi2,
+                                   const noble_cos3_grads *g3, float *dW_up,
+                                   void *workspace, size_t workspace_bytes,
+                                   noble_stream stream);
+
 noble_status noble_linear_bwd_noalloc(const noble_linear_desc *desc,
                                       const void *dy, const void *x,
                                       const void *W, const void *W_down,

@@ -25,6 +25,7 @@ NOBLE_FLAG_SIGMA_COS1, NOBLE_FLAG_SIGMA_IDENTITY = 4, 8
 NOBLE_FLAG_FUSED_BRANCH = 16
 NOBLE_FLAG_ACT_TANH, NOBLE_FLAG_ACT_LEAKYRELU, NOBLE_FLAG_ACT_GELU = 32, 64, 96
 NOBLE_FLAG_SIGMA_SINGLE = NOBLE_FLAG_SIGMA_COS1
+NOBLE_FLAG_SIGMA_COS3 = 128
 # bottleneck variants by name (Section 4.4, Table 5): flags of the descriptor
 SIGMA_FLAGS = {"cosnet": 0, "cos1": NOBLE_FLAG_SIGMA_COS1, "identity": NOBLE_FLAG_SIGMA_IDENTITY,
                "tanh1": NOBLE_FLAG_ACT_TANH | NOBLE_FLAG_SIGMA_SINGLE, "tanh2": NOBLE_FLAG_ACT_TANH,
@@ -63,6 +64,14 @@ class AdamwHparams(ctypes.Structure):
                 ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("step", ctypes.c_int64)]
 
 
+class Cos3Params(ctypes.Structure):
+    _fields_ = [("M2", ctypes.c_void_p), ("omega3", ctypes.c_void_p), ("phi3", ctypes.c_void_p)]
+
+
+class Cos3Grads(ctypes.Structure):
+    _fields_ = [("dM2", ctypes.c_void_p), ("domega3", ctypes.c_void_p), ("dphi3", ctypes.c_void_p)]
+
+
 def make_desc(T, d_in, d_out, r, dtype, flags=0) -> Desc:
     if isinstance(dtype, str):
         dtype = {"bf16": NOBLE_BF16, "fp32": NOBLE_FP32}[dtype]
@@ -99,6 +108,11 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.noble_linear_fwd.restype = ctypes.c_int
         lib.noble_linear_bwd.argtypes = [D] + [P] * 11 + [S] + [P] * 11 + [S, P]
         lib.noble_linear_bwd.restype = ctypes.c_int
+        C3P, C3G = ctypes.POINTER(Cos3Params), ctypes.POINTER(Cos3Grads)
+        lib.noble_linear_fwd_cos3.argtypes = [D] + [P] * 9 + [C3P] + [P] * 3 + [S, P]
+        lib.noble_linear_fwd_cos3.restype = ctypes.c_int
+        lib.noble_linear_bwd_cos3.argtypes = [D] + [P] * 9 + [C3P] + [P] * 2 + [S] + [P] * 9 + [C3G] + [P] * 2 + [S, P]
+        lib.noble_linear_bwd_cos3.restype = ctypes.c_int
         lib.noble_linear_bwd_noalloc.argtypes = [D] + [P] * 11 + [S] + [P] * 10 + [P]
         lib.noble_linear_bwd_noalloc.restype = ctypes.c_int
         lib.noble_get_device_status.argtypes = [P]
@@ -170,6 +184,27 @@ def noble_linear_bwd(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up
                                    _p(saved), saved_bytes, _p(dx), _p(dW), _p(dbias), _p(dW_down),
                                    _p(dM), _p(domega1), _p(dphi1), _p(domega2), _p(dphi2),
                                    _p(dW_up), _p(workspace), workspace_bytes, stream))
+
+
+def noble_linear_fwd_cos3(desc, x, W, bias, W_down, omega1, phi1, M, omega2, phi2, M2, omega3, phi3, W_up,
+                          y, saved, saved_bytes, stream):
+    p3 = Cos3Params(_p(M2), _p(omega3), _p(phi3))
+    _check(load().noble_linear_fwd_cos3(ctypes.byref(desc), _p(x), _p(W), _p(bias), _p(W_down),
+                                        _p(omega1), _p(phi1), _p(M), _p(omega2), _p(phi2),
+                                        ctypes.byref(p3), _p(W_up), _p(y), _p(saved), saved_bytes, stream))
+
+
+def noble_linear_bwd_cos3(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, M2, omega3, phi3, W_up,
+                          saved, saved_bytes, dx, dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2,
+                          dM2, domega3, dphi3, dW_up, workspace, workspace_bytes, stream):
+    p3 = Cos3Params(_p(M2), _p(omega3), _p(phi3))
+    g3 = Cos3Grads(_p(dM2), _p(domega3), _p(dphi3))
+    _check(load().noble_linear_bwd_cos3(ctypes.byref(desc), _p(dy), _p(x), _p(W), _p(W_down),
+                                        _p(omega1), _p(phi1), _p(M), _p(omega2), _p(phi2),
+                                        ctypes.byref(p3), _p(W_up), _p(saved), saved_bytes, _p(dx),
+                                        _p(dW), _p(dbias), _p(dW_down), _p(dM), _p(domega1), _p(dphi1),
+                                        _p(domega2), _p(dphi2), ctypes.byref(g3), _p(dW_up),
+                                        _p(workspace), workspace_bytes, stream))
 
 
 def noble_test_gemm_bf16(M, N, K0, K1, a_mn, b_mn, bn, A0, B0, A1, B1, bias, C, c_fp32,
@@ -280,11 +315,21 @@ class NobleLinearBuffers:
                                    "domega2": torch.empty(r, **f32),
                                    "dphi2": torch.empty(r, **f32),
                                    "dW_up": torch.empty((d_out, r), **f32)})
+                if flags & NOBLE_FLAG_SIGMA_COS3:
+                    self.grads.update({"dM2": torch.empty((r, r), **f32),
+                                       "domega3": torch.empty(r, **f32),
+                                       "dphi3": torch.empty(r, **f32)})
 
 
 def forward(buf: NobleLinearBuffers, x, params: dict, stream=None):
     """y = NOBLE(x) into ``buf.y``; saves activations in ``buf.saved``."""
     p = params
+    if buf.desc.flags & NOBLE_FLAG_SIGMA_COS3:
+        noble_linear_fwd_cos3(buf.desc, x, p["W"], p.get("bias"), p.get("W_down"), p.get("omega1"),
+                              p.get("phi1"), p.get("M"), p.get("omega2"), p.get("phi2"), p.get("M2"),
+                              p.get("omega3"), p.get("phi3"), p.get("W_up"), buf.y, buf.saved,
+                              buf.saved_bytes, _stream_handle(stream))
+        return buf.y
     noble_linear_fwd(buf.desc, x, p["W"], p.get("bias"), p.get("W_down"), p.get("omega1"),
                      p.get("phi1"), p.get("M"), p.get("omega2"), p.get("phi2"), p.get("W_up"),
                      buf.y, buf.saved, buf.saved_bytes, _stream_handle(stream))
@@ -294,6 +339,15 @@ def forward(buf: NobleLinearBuffers, x, params: dict, stream=None):
 def backward(buf: NobleLinearBuffers, x, dy, params: dict, stream=None, with_dbias=True):
     """dx into ``buf.dx`` and parameter gradients into ``buf.grads``."""
     p, g = params, buf.grads
+    if buf.desc.flags & NOBLE_FLAG_SIGMA_COS3:
+        noble_linear_bwd_cos3(buf.desc, dy, x, p["W"], p.get("W_down"), p.get("omega1"), p.get("phi1"),
+                              p.get("M"), p.get("omega2"), p.get("phi2"), p.get("M2"), p.get("omega3"),
+                              p.get("phi3"), p.get("W_up"), buf.saved, buf.saved_bytes, buf.dx, g["dW"],
+                              g["dbias"] if with_dbias else None, g.get("dW_down"), g.get("dM"),
+                              g.get("domega1"), g.get("dphi1"), g.get("domega2"), g.get("dphi2"),
+                              g.get("dM2"), g.get("domega3"), g.get("dphi3"), g.get("dW_up"),
+                              buf.workspace, buf.workspace_bytes, _stream_handle(stream))
+        return buf.dx, g
     noble_linear_bwd(buf.desc, dy, x, p["W"], p.get("W_down"), p.get("omega1"), p.get("phi1"),
                      p.get("M"), p.get("omega2"), p.get("phi2"), p.get("W_up"), buf.saved,
                      buf.saved_bytes, buf.dx, g["dW"], g["dbias"] if with_dbias else None,

@@ -77,6 +77,16 @@ constexpr uint32_t kFlagSigmaCos1 = NOBLE_FLAG_SIGMA_COS1;
 constexpr uint32_t kFlagSigmaIdentity = NOBLE_FLAG_SIGMA_IDENTITY;
 constexpr uint32_t kFlagFusedBranch = NOBLE_FLAG_FUSED_BRANCH;
 constexpr uint32_t kFlagActMask = NOBLE_FLAG_ACT_MASK;
+constexpr uint32_t kFlagSigmaCos3 = NOBLE_FLAG_SIGMA_COS3;
+
+// Three-layer cosine (NOBLE_FLAG_SIGMA_COS3): its extra parameters and
+// gradients, threaded through the forward and backward paths (NULL: not a
+// three-layer descriptor).
+struct Cos3 {
+    const float *M2, *om3, *ph3;
+    float *dM2, *dom3, *dph3;
+};
+bool is_cos3(const noble_linear_desc *d) { return (d->flags & kFlagSigmaCos3) != 0 && d->r > 0; }
 
 // Bottleneck activation selected by the descriptor: CosNet (Eq. 2), or a
 // variant of the ablation (Section 4.4, Table 5): single cosine, identity, or
@@ -116,8 +126,11 @@ noble_status validate_desc(const noble_linear_desc *d)
     if (d->dtype != NOBLE_BF16 && d->dtype != NOBLE_FP32)
         return fail(NOBLE_ERR_UNSUPPORTED, "dtype %d not supported", (int)d->dtype);
     if (d->flags &
-        ~(kFlagSimtOnly | kFlagInference | kFlagSigmaCos1 | kFlagSigmaIdentity | kFlagFusedBranch | kFlagActMask))
+        ~(kFlagSimtOnly | kFlagInference | kFlagSigmaCos1 | kFlagSigmaIdentity | kFlagFusedBranch | kFlagActMask |
+          kFlagSigmaCos3))
         return fail(NOBLE_ERR_UNSUPPORTED, "unknown flags 0x%x", d->flags);
+    if ((d->flags & kFlagSigmaCos3) && (d->flags & (kFlagSigmaCos1 | kFlagSigmaIdentity | kFlagActMask)))
+        return fail(NOBLE_ERR_INVALID_ARG, "NOBLE_FLAG_SIGMA_COS3 with another bottleneck flag");
     if ((d->flags & kFlagSigmaCos1) && (d->flags & kFlagSigmaIdentity))
         return fail(NOBLE_ERR_INVALID_ARG, "NOBLE_FLAG_SIGMA_COS1 and NOBLE_FLAG_SIGMA_IDENTITY together");
     if ((d->flags & kFlagActMask) && (d->flags & kFlagSigmaIdentity))
@@ -163,7 +176,7 @@ bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->
 // backward's MN-major operands also need d_in a multiple of 64 (4-D TMA layout).
 bool fuse_fwd(const noble_linear_desc *d)
 {
-    return use_tc(d) && sigma_of(d).sig == tc::kSigCosnet && (d->r == 64 || d->r == 128) && d->T > 0 &&
+    return use_tc(d) && sigma_of(d).sig == tc::kSigCosnet && !is_cos3(d) && (d->r == 64 || d->r == 128) && d->T > 0 &&
            (d->flags & kFlagFusedBranch);
 }
 bool fuse_bwd(const noble_linear_desc *d) { return fuse_fwd(d) && d->d_in % 64 == 0; }
@@ -173,7 +186,7 @@ size_t fuse_flag_bytes(const noble_linear_desc *d) { return (size_t)(2 * ((d->T 
 // Saved-activation buffer: h, b (fp32) and c (operand dtype), each [T][r];
 // only c for an inference forward on the tensor-core path.
 struct SavedLayout {
-    size_t h, b, c, flags, total;
+    size_t h, b, b2, c, flags, total;
     bool only_c;
 };
 SavedLayout saved_layout(const noble_linear_desc *d)
@@ -181,6 +194,15 @@ SavedLayout saved_layout(const noble_linear_desc *d)
     SavedLayout L{};
     if (d->r == 0 || d->T == 0) return L;
     const size_t tr = (size_t)d->T * (size_t)d->r;
+    if (is_cos3(d)) {
+        // three-layer cosine: h, b, b2 (fp32) and c, also for inference
+        L.h = 0;
+        L.b = align_up(tr * 4, 256);
+        L.b2 = align_up(L.b + tr * 4, 256);
+        L.c = align_up(L.b2 + tr * 4, 256);
+        L.total = align_up(L.c + tr * esize(d), 256);
+        return L;
+    }
     if ((d->flags & kFlagInference) && use_tc(d)) {
         L.only_c = true;
         L.c = 0;
@@ -202,6 +224,7 @@ constexpr int64_t kDmChunk = 1024;     // tokens per dM partial (CUDA-core path)
 constexpr int64_t kBiasChunk = 128;    // tokens per dbias partial (CUDA-core path)
 constexpr int64_t kOnesCols = 64;      // width of the all-ones operand that yields dbias
 int cosnet_tokens_per_block(int64_t r) { return (int)(2048 / r); }
+int cos3_tokens_per_block(int64_t r) { return (int)(1024 / r); }  // 8 [tokens][r] fp32 arrays in shared memory
 
 // K split of the grouped weight-gradient launch (tensor-core path).  When the
 // launch has fewer than two waves of 256 x N tile pairs for a GB300 (74
@@ -217,17 +240,20 @@ int wgrad_split(const noble_linear_desc *d)
     const int rb = r < 128 ? 128 : (int)r;
     int tiles = wgrad_tiles(dout, di, 256) + wgrad_tiles(dout, kOnesCols, 128);
     if (r > 0) tiles += wgrad_tiles(r, di, 256) + wgrad_tiles(dout, r, rb) + wgrad_tiles(r, r, rb);
+    if (is_cos3(d)) tiles += wgrad_tiles(r, r, rb);
     const int64_t kb = ceil_div(T, 64);
     int s = (int)ceil_div(2 * kAssumedPairs, tiles);
     if (s > kb / 16) s = (int)(kb / 16);
     return s < 1 ? 1 : s;
 }
-// Sizes of the five token-summed products (M x N), in launch order.
-void wgrad_shapes(const noble_linear_desc *d, int64_t (&mn)[5][2])
+// Sizes of the token-summed products (M x N), in launch order: dW, dW_down,
+// dW_up, dM, dbias, dM2 (three-layer cosine).
+constexpr int kWgradKinds = 6;
+void wgrad_shapes(const noble_linear_desc *d, int64_t (&mn)[kWgradKinds][2])
 {
     const int64_t di = d->d_in, dout = d->d_out, r = d->r;
-    const int64_t v[5][2] = {{dout, di}, {r, di}, {dout, r}, {r, r}, {dout, 1}};
-    for (int i = 0; i < 5; ++i) mn[i][0] = v[i][0], mn[i][1] = v[i][1];
+    const int64_t v[kWgradKinds][2] = {{dout, di}, {r, di}, {dout, r}, {r, r}, {dout, 1}, {r, r}};
+    for (int i = 0; i < kWgradKinds; ++i) mn[i][0] = v[i][0], mn[i][1] = v[i][1];
 }
 
 // Backward scratch.
@@ -238,7 +264,7 @@ void wgrad_shapes(const noble_linear_desc *d, int64_t (&mn)[5][2])
 //     launch, an all-ones [T][64] bf16 operand (dbias = dy^T 1); the fused
 //     launch's CosNet partials per 32 tokens and its ready flags.
 struct WorkLayout {
-    size_t dh, dc, a, db, mt, ones, cos_part, dm_part, bias_part, flags, wsplit[5], total;
+    size_t dh, dc, a, db, a2, db2, mt, ones, cos_part, dm_part, bias_part, flags, wsplit[kWgradKinds], total;
     int split;
     int64_t n_cos_blocks, n_dm_chunks, n_bias_chunks;
 };
@@ -250,7 +276,33 @@ WorkLayout work_layout(const noble_linear_desc *d)
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     L.dh = take(tr * esize(d));
-    if (use_tc(d)) {
+    if (is_cos3(d)) {
+        // three-layer cosine: dc (fp32) from a GEMM, the CUDA-core chain rule
+        // writes a, db, a2, db2 (bf16 operands of the tensor-core weight
+        // gradients, fp32 on the CUDA-core path) and partials per block
+        const size_t act = use_tc(d) ? 2 : 4;
+        L.dc = take(tr * 4);
+        L.a = take(tr * act);
+        L.db = take(tr * act);
+        L.a2 = take(tr * act);
+        L.db2 = take(tr * act);
+        L.n_cos_blocks = ceil_div(T, cos3_tokens_per_block(r));
+        L.cos_part = take((size_t)L.n_cos_blocks * 6 * r * 4);
+        if (use_tc(d)) {
+            L.ones = take((size_t)T * kOnesCols * 2);
+            L.split = wgrad_split(d);
+            if (L.split > 1) {
+                int64_t mn[kWgradKinds][2];
+                wgrad_shapes(d, mn);
+                for (int i = 0; i < kWgradKinds; ++i) L.wsplit[i] = take((size_t)L.split * mn[i][0] * mn[i][1] * 4);
+            }
+        } else {
+            L.n_dm_chunks = ceil_div(T, kDmChunk);
+            L.dm_part = take((size_t)L.n_dm_chunks * r * r * 4);
+            L.n_bias_chunks = ceil_div(T, kBiasChunk);
+            L.bias_part = take((size_t)L.n_bias_chunks * d->d_out * 4);
+        }
+    } else if (use_tc(d)) {
         L.a = take(tr * 2);
         L.db = take(tr * 2);
         const bool fused = fuse_bwd(d);
@@ -270,7 +322,7 @@ WorkLayout work_layout(const noble_linear_desc *d)
         }
         L.split = wgrad_split(d);
         if (L.split > 1) {
-            int64_t mn[5][2];
+            int64_t mn[kWgradKinds][2];
             wgrad_shapes(d, mn);
             for (int i = 0; i < 5; ++i) L.wsplit[i] = take((size_t)L.split * mn[i][0] * mn[i][1] * 4);
         }
@@ -308,20 +360,60 @@ noble_status simt_gemm(cudaStream_t st, int64_t M, int64_t N, simt::Seg s0, cons
 }
 
 noble_status reduce(cudaStream_t st, int64_t nparts, int64_t n, int64_t seg_len, const float *part,
-                    float *o0, float *o1 = nullptr, float *o2 = nullptr, float *o3 = nullptr)
+                    float *o0, float *o1 = nullptr, float *o2 = nullptr, float *o3 = nullptr,
+                    float *o4 = nullptr, float *o5 = nullptr)
 {
-    simt::Outs4 outs{{o0, o1, o2, o3}};
+    simt::Outs4 outs{{o0, o1, o2, o3, o4, o5, nullptr, nullptr}};
     const KernelInfo ki{"reduce_partials", kBoundHbm, (double)nparts * n, 4.0 * (nparts + 1) * n};
     return run(st, ki, [&] {
         simt::reduce_partials<<<(unsigned)ceil_div(n, 32), 256, 0, st>>>(nparts, n, seg_len, part, outs);
     });
 }
 
+// Three-layer cosine on the CUDA cores, from h (fp32) to b, b2 (saved) and c.
+template <typename TOut>
+noble_status cos3_fwd_rows(const noble_linear_desc *d, const float *h, const float *om1, const float *ph1,
+                           const float *M, const float *om2, const float *ph2, const Cos3 *c3, char *saved,
+                           TOut *c, cudaStream_t st)
+{
+    const int64_t T = d->T, r = d->r;
+    const SavedLayout SL = saved_layout(d);
+    float *b = (float *)(saved + SL.b), *b2 = (float *)(saved + SL.b2);
+    const int tpb = cos3_tokens_per_block(r);
+    const KernelInfo ki{"simt_cos3_fwd", kBoundAlu, 4.0 * T * r * r, 0.0};
+    return run(st, ki, [&] {
+        simt::cosnet3_fwd_rows<TOut><<<(unsigned)ceil_div(T, tpb), 256, 2 * tpb * r * sizeof(float), st>>>(
+            T, (int)r, tpb, h, om1, ph1, M, om2, ph2, c3->M2, c3->om3, c3->ph3, b, b2, c);
+    });
+}
+
+// Three-layer cosine backward on the CUDA cores: dh, a, db, a2, db2 and the
+// six frequency/phase gradients (reduced from per-block partials).
+template <typename TDh, typename TAct>
+noble_status cos3_bwd_rows(const noble_linear_desc *d, const char *saved, const float *dc, const float *om1,
+                           const float *ph1, const float *M, const float *om2, const float *ph2, const Cos3 *c3,
+                           TDh *dh, TAct *a, TAct *db, TAct *a2, TAct *db2, float *cpart, float *dom1, float *dph1,
+                           float *dom2, float *dph2, cudaStream_t st)
+{
+    const int64_t T = d->T, r = d->r;
+    const SavedLayout SL = saved_layout(d);
+    const WorkLayout WL = work_layout(d);
+    const float *h = (const float *)(saved + SL.h), *b = (const float *)(saved + SL.b);
+    const float *b2 = (const float *)(saved + SL.b2);
+    const int tpb = cos3_tokens_per_block(r);
+    const KernelInfo ki{"simt_cos3_bwd", kBoundAlu, 4.0 * T * r * r, 0.0};
+    NOBLE_TRY(run(st, ki, [&] {
+        simt::cosnet3_bwd_rows<TDh, TAct><<<(unsigned)WL.n_cos_blocks, 256, 8 * tpb * r * sizeof(float), st>>>(
+            T, (int)r, tpb, h, b, b2, dc, om1, ph1, M, om2, ph2, c3->M2, c3->om3, c3->ph3, dh, a, db, a2, db2, cpart);
+    }));
+    return reduce(st, WL.n_cos_blocks, 6 * r, r, cpart, dom1, dph1, dom2, dph2, c3->dom3, c3->dph3);
+}
+
 template <typename TIn>
 noble_status fwd_simt(const noble_linear_desc *d, const TIn *x, const TIn *W, const float *bias,
                       const TIn *W_down, const float *om1, const float *ph1, const float *M,
                       const float *om2, const float *ph2, const TIn *W_up, TIn *y, char *saved,
-                      cudaStream_t st)
+                      cudaStream_t st, const Cos3 *c3 = nullptr)
 {
     const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
     const SavedLayout SL = saved_layout(d);
@@ -333,7 +425,9 @@ noble_status fwd_simt(const noble_linear_desc *d, const TIn *x, const TIn *W, co
         NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, down, nullptr, nullptr, h, r)));
         const int tpb = cosnet_tokens_per_block(r);
         const Sigma sg = sigma_of(d);
-        if (sg.two_layers()) {
+        if (c3) {
+            NOBLE_TRY(cos3_fwd_rows<TIn>(d, h, om1, ph1, M, om2, ph2, c3, saved, c, st));
+        } else if (sg.two_layers()) {
             const KernelInfo ki{"simt_cosnet_fwd", kBoundAlu, 2.0 * T * r * r, 0.0};
             NOBLE_TRY(run(st, ki, [&] {
                 simt::cosnet_fwd_rows<TIn><<<(unsigned)ceil_div(T, tpb), 256, tpb * r * sizeof(float), st>>>(
@@ -357,7 +451,8 @@ noble_status bwd_simt(const noble_linear_desc *d, const TIn *dy, const TIn *x, c
                       const TIn *W_down, const float *om1, const float *ph1, const float *M,
                       const float *om2, const float *ph2, const TIn *W_up, const char *saved,
                       TIn *dx, float *dW, float *dbias, float *dW_down, float *dM, float *dom1,
-                      float *dph1, float *dom2, float *dph2, float *dW_up, char *ws, cudaStream_t st)
+                      float *dph1, float *dom2, float *dph2, float *dW_up, char *ws, cudaStream_t st,
+                      const Cos3 *c3 = nullptr)
 {
     const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
     const SavedLayout SL = saved_layout(d);
@@ -365,7 +460,28 @@ noble_status bwd_simt(const noble_linear_desc *d, const TIn *dy, const TIn *x, c
     const float *h = (const float *)(saved + SL.h), *b = (const float *)(saved + SL.b);
     const TIn *c = (const TIn *)(saved + SL.c);
     TIn *dh = (TIn *)(ws + WL.dh);
-    if (r > 0) {
+    if (r > 0 && c3) {
+        float *dc = (float *)(ws + WL.dc), *a = (float *)(ws + WL.a), *db = (float *)(ws + WL.db);
+        float *a2 = (float *)(ws + WL.a2), *db2 = (float *)(ws + WL.db2);
+        float *cpart = (float *)(ws + WL.cos_part), *dmpart = (float *)(ws + WL.dm_part);
+        simt::Seg sdc{{dy, dout, 1}, {W_up, 1, r}, dout};
+        NOBLE_TRY((simt_gemm<TIn, float>(st, T, r, sdc, nullptr, nullptr, dc, r)));
+        NOBLE_TRY((cos3_bwd_rows<TIn, float>(d, saved, dc, om1, ph1, M, om2, ph2, c3, dh, a, db, a2, db2, cpart,
+                                             dom1, dph1, dom2, dph2, st)));
+        // dM = a^T db and dM2 = a2^T db2, fixed token chunks, one after the other
+        const float *pa[2] = {a, a2}, *pd[2] = {db, db2};
+        float *outs[2] = {dM, c3->dM2};
+        for (int k = 0; k < 2; ++k) {
+            simt::Seg sdm{{pa[k], 1, r}, {pd[k], 1, r}, T};
+            NOBLE_TRY((simt_gemm<float, float>(st, r, r, sdm, nullptr, nullptr, dmpart, r, kDmChunk,
+                                               WL.n_dm_chunks, r * r)));
+            NOBLE_TRY(reduce(st, WL.n_dm_chunks, r * r, r * r, dmpart, outs[k]));
+        }
+        simt::Seg sup{{dy, 1, dout}, {c, 1, r}, T};
+        NOBLE_TRY((simt_gemm<TIn, float>(st, dout, r, sup, nullptr, nullptr, dW_up, r)));
+        simt::Seg sdn{{dh, 1, r}, {x, 1, di}, T};
+        NOBLE_TRY((simt_gemm<TIn, float>(st, r, di, sdn, nullptr, nullptr, dW_down, di)));
+    } else if (r > 0) {
         float *dc = (float *)(ws + WL.dc), *a = (float *)(ws + WL.a), *db = (float *)(ws + WL.db);
         float *Mt = (float *)(ws + WL.mt), *cpart = (float *)(ws + WL.cos_part);
         float *dmpart = (float *)(ws + WL.dm_part);
@@ -894,7 +1010,8 @@ bool mn4_ok(std::initializer_list<int64_t> mn_extents, std::initializer_list<int
 
 noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, const float *bias,
                     const bf16 *W_down, const float *om1, const float *ph1, const float *M, const float *om2,
-                    const float *ph2, const bf16 *W_up, bf16 *y, char *saved, cudaStream_t st)
+                    const float *ph2, const bf16 *W_up, bf16 *y, char *saved, cudaStream_t st,
+                    const Cos3 *c3 = nullptr)
 {
     const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
     const TcSeg main{x, W, di};
@@ -906,6 +1023,17 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     const SavedLayout SL = saved_layout(d);
     float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
     bf16 *c = (bf16 *)(saved + SL.c);
+    if (c3) {
+        // three-layer cosine: h = x W_down^T on the tensor cores (fp32 out), the
+        // cosines and r x r products on the CUDA cores, then the output GEMM
+        const ProbSpec Ph{T, r, TcSeg{x, W_down, di}, nullptr, r <= 128 ? 128 : 256};
+        const tc::EpiStore<float>::Params Eh{h, r, nullptr, 0};
+        NOBLE_TRY((tc_pair_group<false, false, tc::EpiStore<float>>(st, "tc_h_gemm", 1, &Ph, &Eh)));
+        NOBLE_TRY(cos3_fwd_rows<bf16>(d, h, om1, ph1, M, om2, ph2, c3, saved, c, st));
+        const TcSeg up{c, W_up, r};
+        const ProbSpec P{T, dout, main, &up, 256};
+        return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
+    }
     if (fuse_fwd(d)) {
         // one launch: bottleneck tiles (h, CosNet, c) and output tiles
         uint32_t *flags = (uint32_t *)(saved + SL.flags);
@@ -948,7 +1076,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
                     const float *om1, const float *ph1, const float *M, const float *om2, const float *ph2,
                     const bf16 *W_up, const char *saved, bf16 *dx, float *dW, float *dbias, float *dW_down,
                     float *dM, float *dom1, float *dph1, float *dom2, float *dph2, float *dW_up, char *ws,
-                    cudaStream_t st)
+                    cudaStream_t st, const Cos3 *c3 = nullptr)
 {
     const int64_t T = d->T, di = d->d_in, dout = d->d_out, r = d->r;
     const SavedLayout SL = saved_layout(d);
@@ -956,7 +1084,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
     bf16 *ones = (bf16 *)(ws + WL.ones);
     const bool fused = fuse_bwd(d);
-    const bool ones_dbias = dbias && (r == 0 || fused);
+    const bool ones_dbias = dbias && (r == 0 || fused || c3);
     const Sigma sg = sigma_of(d);
     if (ones_dbias) NOBLE_TRY(fill_ones(st, T * kOnesCols, ones));
     // domega1, dphi1, domega2, dphi2 (and dbias) from per-CTA or per-32-token partials
@@ -985,7 +1113,20 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
         return run(st, kr, [&] { reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J); });
     };
-    if (r > 0 && !fused) {
+    if (r > 0 && c3) {
+        // three-layer cosine: dc = dy W_up on the tensor cores (fp32 out), the
+        // chain rule on the CUDA cores (bf16 a, db, a2, db2 for the weight gradients)
+        float *dc = (float *)(ws + WL.dc);
+        const ProbSpec Pc{T, r, TcSeg{dy, W_up, dout}, nullptr, r <= 128 ? 128 : 256};
+        const tc::EpiStore<float>::Params Ec{dc, r, nullptr, 0};
+        if (mn4_ok({r}, {dout}))
+            NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<float>, true>(st, "tc_dc_gemm", 1, &Pc, &Ec)));
+        else
+            NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<float>>(st, "tc_dc_gemm", 1, &Pc, &Ec)));
+        bf16 *a2 = (bf16 *)(ws + WL.a2), *db2 = (bf16 *)(ws + WL.db2);
+        NOBLE_TRY((cos3_bwd_rows<bf16, bf16>(d, saved, dc, om1, ph1, M, om2, ph2, c3, dh, a, db, a2, db2,
+                                             (float *)(ws + WL.cos_part), dom1, dph1, dom2, dph2, st)));
+    } else if (r > 0 && !fused) {
         float *cpart = (float *)(ws + WL.cos_part);
         tc::CosnetArgs ca{};
         ca.om1 = om1, ca.ph1 = ph1, ca.om2 = om2, ca.ph2 = ph2, ca.M = M;
@@ -1041,12 +1182,12 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     // dM = a^T db, dbias = dy^T 1, dW = dy^T x
     {
         const bf16 *c = r > 0 ? (const bf16 *)(saved + SL.c) : nullptr;
-        ProbSpec P[5];
-        tc::EpiStore<float>::Params E[5];
-        float *final_out[5];
-        int64_t mn[5][2];
+        ProbSpec P[kWgradKinds];
+        tc::EpiStore<float>::Params E[kWgradKinds];
+        float *final_out[kWgradKinds];
+        int64_t mn[kWgradKinds][2];
         wgrad_shapes(d, mn);
-        int which[5];
+        int which[kWgradKinds];
         int n = 0;
         auto add = [&](int k, ProbSpec ps, float *out, int64_t ldc, bool col0) {
             P[n] = ps;
@@ -1063,6 +1204,10 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false);
             if (sg.two_layers())
                 add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);
+            if (c3) {
+                const bf16 *a2 = (const bf16 *)(ws + WL.a2), *db2 = (const bf16 *)(ws + WL.db2);
+                add(5, ProbSpec{r, r, TcSeg{a2, db2, T}, nullptr, r < 128 ? 128 : (int)r}, c3->dM2, r, false);
+            }
             else if (cudaMemsetAsync(dM, 0, (size_t)r * r * 4, st) != cudaSuccess)
                 return fail(NOBLE_ERR_CUDA, "dM: %s", cudaGetErrorString(cudaGetLastError()));
         }
@@ -1145,15 +1290,24 @@ size_t noble_linear_bwd_workspace_bytes(const noble_linear_desc *desc)
     return work_layout(desc).total;
 }
 
-noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, const void *W,
-                              const float *bias, const void *W_down, const float *omega1,
-                              const float *phi1, const float *M, const float *omega2,
-                              const float *phi2, const void *W_up, void *y, void *saved,
-                              size_t saved_bytes, noble_stream stream)
+// The forward entry point; c3 non-NULL for noble_linear_fwd_cos3.
+static noble_status fwd_entry(const noble_linear_desc *desc, const void *x, const void *W, const float *bias,
+                              const void *W_down, const float *omega1, const float *phi1, const float *M,
+                              const float *omega2, const float *phi2, const void *W_up, void *y, void *saved,
+                              size_t saved_bytes, noble_stream stream, const Cos3 *c3)
 {
     g_last_error[0] = 0;
     NOBLE_TRY(validate_desc(desc));
     const bool br = desc->r > 0, empty = desc->T == 0;
+    if (((desc->flags & kFlagSigmaCos3) != 0) != (c3 != nullptr))
+        return fail(NOBLE_ERR_INVALID_ARG, c3 ? "noble_linear_fwd_cos3 needs NOBLE_FLAG_SIGMA_COS3"
+                                              : "a NOBLE_FLAG_SIGMA_COS3 descriptor needs noble_linear_fwd_cos3");
+    if (c3) {
+        NOBLE_TRY(check_ptr(c3->M2, "M2", !br));
+        NOBLE_TRY(check_ptr(c3->om3, "omega3", !br));
+        NOBLE_TRY(check_ptr(c3->ph3, "phi3", !br));
+    }
+    const Cos3 *k3 = is_cos3(desc) ? c3 : nullptr;
     NOBLE_TRY(check_ptr(x, "x", empty));
     NOBLE_TRY(check_ptr(W, "W", false));
     NOBLE_TRY(check_ptr(bias, "bias", true));
@@ -1177,25 +1331,57 @@ noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, cons
         using bf = __nv_bfloat16;
         if (!(desc->flags & kFlagSimtOnly))
             return fwd_tc(desc, (const bf *)x, (const bf *)W, bias, (const bf *)W_down, omega1, phi1, M, omega2,
-                          phi2, (const bf *)W_up, (bf *)y, (char *)saved, st);
+                          phi2, (const bf *)W_up, (bf *)y, (char *)saved, st, k3);
         return fwd_simt<bf>(desc, (const bf *)x, (const bf *)W, bias, (const bf *)W_down, omega1, phi1, M,
-                            omega2, phi2, (const bf *)W_up, (bf *)y, (char *)saved, st);
+                            omega2, phi2, (const bf *)W_up, (bf *)y, (char *)saved, st, k3);
     }
     return fwd_simt<float>(desc, (const float *)x, (const float *)W, bias, (const float *)W_down, omega1,
-                           phi1, M, omega2, phi2, (const float *)W_up, (float *)y, (char *)saved, st);
+                           phi1, M, omega2, phi2, (const float *)W_up, (float *)y, (char *)saved, st, k3);
 }
 
-noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, const void *x,
-                              const void *W, const void *W_down, const float *omega1,
+noble_status noble_linear_fwd(const noble_linear_desc *desc, const void *x, const void *W,
+                              const float *bias, const void *W_down, const float *omega1,
                               const float *phi1, const float *M, const float *omega2,
-                              const float *phi2, const void *W_up, const void *saved,
-                              size_t saved_bytes, void *dx,
-                              float *dW, float *dbias, float *dW_down, float *dM, float *domega1,
-                              float *dphi1, float *domega2, float *dphi2, float *dW_up,
-                              void *workspace, size_t workspace_bytes, noble_stream stream)
+                              const float *phi2, const void *W_up, void *y, void *saved,
+                              size_t saved_bytes, noble_stream stream)
+{
+    return fwd_entry(desc, x, W, bias, W_down, omega1, phi1, M, omega2, phi2, W_up, y, saved, saved_bytes, stream,
+                     nullptr);
+}
+
+noble_status noble_linear_fwd_cos3(const noble_linear_desc *desc, const void *x, const void *W,
+                                   const float *bias, const void *W_down, const float *omega1,
+                                   const float *phi1, const float *M, const float *omega2,
+                                   const float *phi2, const noble_cos3_params *p3, const void *W_up,
+                                   void *y, void *saved, size_t saved_bytes, noble_stream stream)
+{
+    g_last_error[0] = 0;
+    if (!p3) return fail(NOBLE_ERR_INVALID_ARG, "p3 is NULL");
+    const Cos3 c3{p3->M2, p3->omega3, p3->phi3, nullptr, nullptr, nullptr};
+    return fwd_entry(desc, x, W, bias, W_down, omega1, phi1, M, omega2, phi2, W_up, y, saved, saved_bytes, stream,
+                     &c3);
+}
+
+// The backward entry point; c3 non-NULL for noble_linear_bwd_cos3.
+static noble_status bwd_entry(const noble_linear_desc *desc, const void *dy, const void *x, const void *W,
+                              const void *W_down, const float *omega1, const float *phi1, const float *M,
+                              const float *omega2, const float *phi2, const void *W_up, const void *saved,
+                              size_t saved_bytes, void *dx, float *dW, float *dbias, float *dW_down, float *dM,
+                              float *domega1, float *dphi1, float *domega2, float *dphi2, float *dW_up,
+                              void *workspace, size_t workspace_bytes, noble_stream stream, const Cos3 *c3)
 {
     g_last_error[0] = 0;
     NOBLE_TRY(validate_desc(desc));
+    if (((desc->flags & kFlagSigmaCos3) != 0) != (c3 != nullptr))
+        return fail(NOBLE_ERR_INVALID_ARG, c3 ? "noble_linear_bwd_cos3 needs NOBLE_FLAG_SIGMA_COS3"
+                                              : "a NOBLE_FLAG_SIGMA_COS3 descriptor needs noble_linear_bwd_cos3");
+    if (c3) {
+        const bool br3 = desc->r > 0;
+        const char *n3[] = {"M2", "omega3", "phi3", "dM2", "domega3", "dphi3"};
+        const void *p3[] = {c3->M2, c3->om3, c3->ph3, c3->dM2, c3->dom3, c3->dph3};
+        for (int i = 0; i < 6; ++i) NOBLE_TRY(check_ptr(p3[i], n3[i], !br3));
+    }
+    const Cos3 *k3 = is_cos3(desc) ? c3 : nullptr;
     if (desc->flags & kFlagInference)
         return fail(NOBLE_ERR_INVALID_ARG, "backward of an inference descriptor (NOBLE_FLAG_INFERENCE)");
     const bool br = desc->r > 0, empty = desc->T == 0;
@@ -1222,23 +1408,61 @@ noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, con
                     work_layout(desc).total);
     NOBLE_TRY(check_device());
     cudaStream_t st = (cudaStream_t)stream;
-    if (desc->T == 0)
+    if (desc->T == 0) {
+        if (k3) {
+            const int64_t r = desc->r;
+            if (cudaMemsetAsync(k3->dM2, 0, (size_t)r * r * 4, st) != cudaSuccess ||
+                cudaMemsetAsync(k3->dom3, 0, (size_t)r * 4, st) != cudaSuccess ||
+                cudaMemsetAsync(k3->dph3, 0, (size_t)r * 4, st) != cudaSuccess)
+                return fail(NOBLE_ERR_CUDA, "zero gradients: %s", cudaGetErrorString(cudaGetLastError()));
+        }
         return zero_grads(desc, dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, st);
+    }
     if (desc->dtype == NOBLE_BF16) {
         using bf = __nv_bfloat16;
         if (!(desc->flags & kFlagSimtOnly))
             return bwd_tc(desc, (const bf *)dy, (const bf *)x, (const bf *)W, (const bf *)W_down, omega1, phi1, M,
                           omega2, phi2, (const bf *)W_up, (const char *)saved, (bf *)dx, dW, dbias, dW_down, dM,
-                          domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace, st);
+                          domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace, st, k3);
         return bwd_simt<bf>(desc, (const bf *)dy, (const bf *)x, (const bf *)W, (const bf *)W_down, omega1,
                             phi1, M, omega2, phi2, (const bf *)W_up, (const char *)saved, (bf *)dx, dW,
                             dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, (char *)workspace,
-                            st);
+                            st, k3);
     }
     return bwd_simt<float>(desc, (const float *)dy, (const float *)x, (const float *)W, (const float *)W_down,
                            omega1, phi1, M, omega2, phi2, (const float *)W_up, (const char *)saved,
                            (float *)dx, dW, dbias, dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up,
-                           (char *)workspace, st);
+                           (char *)workspace, st, k3);
+}
+
+noble_status noble_linear_bwd(const noble_linear_desc *desc, const void *dy, const void *x,
+                              const void *W, const void *W_down, const float *omega1,
+                              const float *phi1, const float *M, const float *omega2,
+                              const float *phi2, const void *W_up, const void *saved,
+                              size_t saved_bytes, void *dx,
+                              float *dW, float *dbias, float *dW_down, float *dM, float *domega1,
+                              float *dphi1, float *domega2, float *dphi2, float *dW_up,
+                              void *workspace, size_t workspace_bytes, noble_stream stream)
+{
+    return bwd_entry(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up, saved, saved_bytes, dx, dW, dbias,
+                     dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, workspace, workspace_bytes, stream, nullptr);
+}
+
+noble_status noble_linear_bwd_cos3(const noble_linear_desc *desc, const void *dy, const void *x,
+                                   const void *W, const void *W_down, const float *omega1,
+                                   const float *phi1, const float *M, const float *omega2,
+                                   const float *phi2, const noble_cos3_params *p3, const void *W_up,
+                                   const void *saved, size_t saved_bytes, void *dx, float *dW,
+                                   float *dbias, float *dW_down, float *dM, float *domega1,
+                                   float *dphi1, float *domega2, float *dphi2,
+                                   const noble_cos3_grads *g3, float *dW_up, void *workspace,
+                                   size_t workspace_bytes, noble_stream stream)
+{
+    g_last_error[0] = 0;
+    if (!p3 || !g3) return fail(NOBLE_ERR_INVALID_ARG, "p3 or g3 is NULL");
+    const Cos3 c3{p3->M2, p3->omega3, p3->phi3, g3->dM2, g3->domega3, g3->dphi3};
+    return bwd_entry(desc, dy, x, W, W_down, omega1, phi1, M, omega2, phi2, W_up, saved, saved_bytes, dx, dW, dbias,
+                     dW_down, dM, domega1, dphi1, domega2, dphi2, dW_up, workspace, workspace_bytes, stream, &c3);
 }
 
 noble_status noble_get_device_status(noble_stream stream)

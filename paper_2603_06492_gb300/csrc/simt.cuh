@@ -258,6 +258,129 @@ cosnet_bwd_rows(int64_t T, int r, int act, int tokens_per_block, const float *h,
     }
 }
 
+// Three-layer cosine (the deepest row of the ablation, Section 4.4, Table 5)
+// on rows: from h [T][r] (fp32)
+//   a = cos(omega1 h + phi1), b = a M, a2 = cos(omega2 b + phi2), b2 = a2 M2,
+//   c = cos(omega3 b2 + phi3)
+// writing b, b2 (fp32) and c (TOut), each [T][r].  Block: tokens_per_block
+// rows; shared memory 2 tokens_per_block r floats.
+template <typename TOut>
+__global__ void __launch_bounds__(256)
+cosnet3_fwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const float *om1, const float *ph1,
+                 const float *M, const float *om2, const float *ph2, const float *M2, const float *om3,
+                 const float *ph3, float *b_out, float *b2_out, TOut *c_out)
+{
+    extern __shared__ float sm3[];
+    const int n = tokens_per_block * r;
+    float *a_s = sm3, *a2_s = sm3 + n;
+    const int64_t t0 = (int64_t)blockIdx.x * tokens_per_block;
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, i = idx % r;
+        const int64_t t = t0 + tt;
+        a_s[idx] = t < T ? cosf(fmaf(om1[i], h[t * r + i], ph1[i])) : 0.f;
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, j = idx % r;
+        const int64_t t = t0 + tt;
+        float s = 0.f;
+        for (int i = 0; i < r; ++i) s = fmaf(a_s[tt * r + i], M[i * r + j], s);
+        a2_s[idx] = cosf(fmaf(om2[j], s, ph2[j]));
+        if (t < T) b_out[t * r + j] = s;
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, j = idx % r;
+        const int64_t t = t0 + tt;
+        if (t >= T) continue;
+        float s = 0.f;
+        for (int i = 0; i < r; ++i) s = fmaf(a2_s[tt * r + i], M2[i * r + j], s);
+        b2_out[t * r + j] = s;
+        Elem<TOut>::store(c_out + t * r + j, cosf(fmaf(om3[j], s, ph3[j])));
+    }
+}
+
+// Backward of cosnet3_fwd_rows (chain rule through the three layers): from
+// saved h, b, b2 (fp32) and dc = dy W_up (fp32)
+//   du3 = -sin(u3) dc, db2 = omega3 du3, da2 = db2 M2^T,
+//   du2 = -sin(u2) da2, db = omega2 du2, da = db M^T,
+//   du1 = -sin(u1) da, dh = omega1 du1,  a = cos(u1), a2 = cos(u2)
+// writing dh (TDh), a, db, a2, db2 (TAct), each [T][r], and per-block column
+// sums over the block's tokens in ascending order, part[blk][q][r] with
+// q = 0 sum du1*h, 1 sum du1, 2 sum du2*b, 3 sum du2, 4 sum du3*b2, 5 sum du3.
+// Shared memory 8 tokens_per_block r floats.
+template <typename TDh, typename TAct>
+__global__ void __launch_bounds__(256)
+cosnet3_bwd_rows(int64_t T, int r, int tokens_per_block, const float *h, const float *b, const float *b2,
+                 const float *dc, const float *om1, const float *ph1, const float *M, const float *om2,
+                 const float *ph2, const float *M2, const float *om3, const float *ph3, TDh *dh_out,
+                 TAct *a_out, TAct *db_out, TAct *a2_out, TAct *db2_out, float *part)
+{
+    extern __shared__ float sm3[];
+    const int n = tokens_per_block * r;
+    float *db2_s = sm3, *db_s = sm3 + n;
+    float *q_s = sm3 + 2 * n;  // six [tokens_per_block][r] arrays, in the order of part
+    const int64_t t0 = (int64_t)blockIdx.x * tokens_per_block;
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, j = idx % r;
+        const int64_t t = t0 + tt;
+        float du3 = 0.f, bv = 0.f;
+        if (t < T) {
+            bv = b2[t * r + j];
+            du3 = -sinf(fmaf(om3[j], bv, ph3[j])) * dc[t * r + j];
+        }
+        db2_s[idx] = om3[j] * du3;
+        q_s[4 * n + idx] = du3 * bv;
+        q_s[5 * n + idx] = du3;
+        if (t < T) Elem<TAct>::store(db2_out + t * r + j, om3[j] * du3);
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, i = idx % r;
+        const int64_t t = t0 + tt;
+        float du2 = 0.f, bv = 0.f;
+        if (t < T) {
+            float da2 = 0.f;
+            for (int j = 0; j < r; ++j) da2 = fmaf(db2_s[tt * r + j], M2[i * r + j], da2);
+            bv = b[t * r + i];
+            float s2, c2;
+            sincosf(fmaf(om2[i], bv, ph2[i]), &s2, &c2);
+            du2 = -s2 * da2;
+            Elem<TAct>::store(a2_out + t * r + i, c2);
+            Elem<TAct>::store(db_out + t * r + i, om2[i] * du2);
+        }
+        db_s[idx] = om2[i] * du2;
+        q_s[2 * n + idx] = du2 * bv;
+        q_s[3 * n + idx] = du2;
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < n; idx += blockDim.x) {
+        const int tt = idx / r, i = idx % r;
+        const int64_t t = t0 + tt;
+        float du1 = 0.f, hv = 0.f;
+        if (t < T) {
+            float da = 0.f;
+            for (int j = 0; j < r; ++j) da = fmaf(db_s[tt * r + j], M[i * r + j], da);
+            hv = h[t * r + i];
+            float s1, c1;
+            sincosf(fmaf(om1[i], hv, ph1[i]), &s1, &c1);
+            du1 = -s1 * da;
+            Elem<TAct>::store(a_out + t * r + i, c1);
+            Elem<TDh>::store(dh_out + t * r + i, om1[i] * du1);
+        }
+        q_s[idx] = du1 * hv;
+        q_s[n + idx] = du1;
+    }
+    __syncthreads();
+    float *pb = part + (int64_t)blockIdx.x * 6 * r;
+    for (int k = threadIdx.x; k < 6 * r; k += blockDim.x) {
+        const int q = k / r, j = k % r;
+        float s = 0.f;
+        for (int tt = 0; tt < tokens_per_block; ++tt) s += q_s[q * n + tt * r + j];
+        pb[k] = s;
+    }
+}
+
 // part[c][o] = sum over rows t in chunk c (ascending) of X[t][o].
 template <typename TIn>
 __global__ void colsum_partial(int64_t T, int64_t n, int64_t rows_per_chunk, const TIn *X,
@@ -303,7 +426,7 @@ __global__ void __launch_bounds__(256) colsum_partial_bf16x8(int64_t T, int64_t 
 // ascending order, then the 8 warp sums are added in warp order, so the
 // result does not depend on scheduling.
 struct Outs4 {
-    float *p[4];
+    float *p[8];  // up to eight outputs of seg_len elements each
 };
 __global__ void __launch_bounds__(256) reduce_partials(int64_t nparts, int64_t n, int64_t seg_len,
                                                        const float *part, Outs4 outs)

@@ -128,6 +128,16 @@ def make_layer_inputs(layer: Layer, seed: int, init: str = "config") -> dict:
     return out
 
 
+def make_cos3_inputs(r: int, seed: int) -> dict:
+    """The extra parameters of the three-layer cosine bottleneck: M2 [r, r]
+    (b2 = a2 M2) ~ N(0, 1/r), omega3 ~ U(0.5, 2), phi3 ~ U(-pi, pi), drawn in
+    that order from their own PCG64 stream, fp32."""
+    rng = np.random.default_rng(seed)
+    return {"M2": round_fp32(rng.standard_normal((r, r)) / math.sqrt(r)),
+            "omega3": round_fp32(rng.uniform(0.5, 2.0, r)),
+            "phi3": round_fp32(rng.uniform(-math.pi, math.pi, r))}
+
+
 def to_paper_orientation(inp: dict) -> dict:
     """The same tensors in the paper's row-vector orientation (Eq. 1):
     W [d_in, d_out], W_down [d_in, r], W_up [r, d_out]; others unchanged."""

@@ -77,7 +77,7 @@ def test_bad_pointers_rejected(lib):
         _fwd(d, saved_bytes=16)
     assert e.value.status == 4
     bad = binding.make_desc(256, 128, 128, 16, "bf16")
-    bad.flags = 0x80  # unknown flag bit
+    bad.flags = 0x100  # unknown flag bit
     with pytest.raises(binding.NobleError) as e:
         _fwd(bad)
     assert e.value.status == 3
@@ -194,3 +194,20 @@ def test_activation_flags(lib):
     with pytest.raises(binding.NobleError) as e:
         _fwd(binding.make_desc(256, 128, 128, 16, "bf16", binding.NOBLE_FLAG_ACT_TANH), M=None)
     assert e.value.status == 1
+
+
+def test_cos3_flag_validation(lib):
+    # the three-layer flag excludes the other bottleneck flags; the plain entry
+    # points refuse a three-layer descriptor (before any device check)
+    for other in (binding.NOBLE_FLAG_SIGMA_COS1, binding.NOBLE_FLAG_SIGMA_IDENTITY, binding.NOBLE_FLAG_ACT_GELU):
+        bad = binding.make_desc(256, 128, 128, 16, "bf16", binding.NOBLE_FLAG_SIGMA_COS3 | other)
+        with pytest.raises(binding.NobleError) as e:
+            _fwd(bad)
+        assert e.value.status == 1
+    three = binding.make_desc(256, 128, 128, 16, "bf16", binding.NOBLE_FLAG_SIGMA_COS3)
+    with pytest.raises(binding.NobleError) as e:
+        _fwd(three)
+    assert e.value.status == 1 and "cos3" in str(e.value)
+    # h, b, b2 (fp32) and c (bf16), each 256-byte aligned
+    T, r = 256, 16
+    assert binding.noble_linear_saved_bytes(three) == 3 * T * r * 4 + T * r * 2
