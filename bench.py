@@ -110,7 +110,7 @@ class ClockSampler:
             self.thread.join(timeout=2)
 
     def summary(self):
-        sm, mx, reasons = [], [], set()
+        sm, mx, pw, reasons = [], [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
         # samples taken inside the timed region; if it was shorter than the
         # sampling interval, the last sample before it
@@ -124,12 +124,17 @@ class ClockSampler:
                 mx.append(float(f[2]))
             except ValueError:
                 continue
+            try:
+                pw.append(float(f[3]))
+            except ValueError:
+                pass
             for n, v in zip(names, f[5:9]):
                 if v.lower() in ("active", "1", "0x1"):
                     reasons.add(n)
         if not sm:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "power_w": statistics.median(pw) if pw else None,
                 "samples": len(sm), "samples_in_timed_region": len(self.lines[self.start:])}
 
 
@@ -366,9 +371,10 @@ def main():
     # plain runs alternate three times, medians compared (clock and thermal
     # drift between two single runs is of the size of the effect)
     reps_n, reps_p = [], []
-    for _ in range(3):
-        reps_n.append(timed(lambda: step(bufs), args.steps))
-        reps_p.append(timed(lambda: step(plain_bufs, plain=True), args.steps))
+    with ClockSampler(local_rank) as clk_ovh:
+        for _ in range(3):
+            reps_n.append(timed(lambda: step(bufs), args.steps))
+            reps_p.append(timed(lambda: step(plain_bufs, plain=True), args.steps))
     ms_noble_med, ms_plain = statistics.median(reps_n), statistics.median(reps_p)
 
     # forward and backward passes timed apart
@@ -577,6 +583,9 @@ def main():
             "plain_tflops": world * flops_plain / (ms_plain / args.steps * 1e-3) / 1e12,
             "overhead_vs_plain": ms_noble_med / ms_plain - 1.0,
             "overhead_method": "median of 3 alternating NOBLE / plain runs of the timed steps",
+            "overhead_reps_ms_per_step": {"noble": [round(v / args.steps, 4) for v in reps_n],
+                                          "plain": [round(v / args.steps, 4) for v in reps_p]},
+            "overhead_clocks": clk_ovh.summary(),
             "fwd_ms_per_step": ms_fwd / args.steps, "bwd_ms_per_step": ms_bwd / args.steps,
             "plain_fwd_ms_per_step": ms_fwd_p / args.steps, "plain_bwd_ms_per_step": ms_bwd_p / args.steps,
             "overhead_fwd": ms_fwd / ms_fwd_p - 1.0, "overhead_bwd": ms_bwd / ms_bwd_p - 1.0,
