@@ -31,7 +31,7 @@ import numpy as np
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from paper_2603_06492_gb300.inputs import (CONFIGS, PAPER_WORKLOAD_SEED, PAPER_WORKLOADS,  # noqa: E402
+from paper_2603_06492_gb300.inputs import (CONFIGS, PAPER_WORKLOAD_SEED, PAPER_WORKLOADS, make_cos3_inputs,  # noqa: E402
                                            layer_seed, make_layer_inputs)
 
 CONFIG_INDEX = 3
@@ -242,7 +242,8 @@ def main():
     ap.add_argument("--workload", default="", choices=["", "geglu-base", "geglu-large"],
                     help="the paper's GeGLU FFN shapes instead of a numbered configuration")
     ap.add_argument("--sigma", default="cosnet",
-                    choices=["cosnet", "cos1", "identity", "tanh1", "tanh2", "leaky1", "leaky2", "gelu1", "gelu2"],
+                    choices=["cosnet", "cos1", "identity", "tanh1", "tanh2", "leaky1", "leaky2", "gelu1", "gelu2",
+                             "cos3"],
                     help="bottleneck activation (the others: variants of the ablation, Section 4.4)")
     ap.add_argument("--fused-branch", action="store_true",
                     help="run the bottleneck inside the output GEMMs (NOBLE_FLAG_FUSED_BRANCH)")
@@ -283,7 +284,11 @@ def main():
         inp = make_layer_inputs(layer, layer_seed(seed_cfg, li))
         dev_inputs.append(binding.params_to_device(inp, layer.dtype))
         del inp
-        sig_flags = binding.SIGMA_FLAGS[args.sigma]
+        sig_flags = binding.SIGMA_FLAGS[args.sigma] if args.sigma != "cos3" else binding.NOBLE_FLAG_SIGMA_COS3
+        if args.sigma == "cos3":
+            # the three-layer cosine's second mixing matrix and third frequency / phase
+            dev_inputs[-1].update(binding.params_to_device(make_cos3_inputs(layer.r, layer_seed(seed_cfg, li) + 1),
+                                                           layer.dtype))
         if args.fused_branch:
             sig_flags |= binding.NOBLE_FLAG_FUSED_BRANCH
         bufs.append(binding.NobleLinearBuffers(layer.T, layer.d_in, layer.d_out, layer.r, layer.dtype,
@@ -429,7 +434,9 @@ def main():
     # on their own streams and overlap the compute of other layers and of the
     # neighbouring step (device inputs and outputs are double-buffered).
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and args.sigma == "cos3":
+        e2e = {"value": None, "note": "not measured for the three-layer cosine (its own entry points)"}
+    elif not args.no_e2e:
         h2d_s, d2h_s = torch.cuda.Stream(), torch.cuda.Stream()
         host, sets, h2d, d2h = [], [], 0, 0
         for d, b in zip(dev_inputs, bufs):
