@@ -55,6 +55,9 @@ noble_status check_launch(const char *what)
     return NOBLE_OK;
 }
 
+// Kernels launched so far by the current entry-point call on this thread.
+thread_local int g_call_kernels = 0;
+
 // Launch through `f`, bracketed by profiling events when profiling is on.
 template <class F>
 noble_status run(cudaStream_t st, const KernelInfo &ki, F &&f)
@@ -62,7 +65,42 @@ noble_status run(cudaStream_t st, const KernelInfo &ki, F &&f)
     const int slot = Profiler::get().begin(st);
     f();
     Profiler::get().end(slot, st, ki);
+    ++g_call_kernels;
     return check_launch(ki.name);
+}
+
+// Programmatic dependent launch: the pair GEMMs and the partial-sum
+// reductions may start while the previous kernel of the same call still runs,
+// on the SMs it leaves free; they wait for it (griddep_wait) before reading
+// anything an earlier kernel of the call wrote, and every such grid waits at
+// least once, so its completion implies its predecessors'.  The first kernel
+// of a call, and the first after a memset, is launched normally and sees all
+// prior work in the stream.
+constexpr bool kProgrammaticLaunch = true;
+bool pdl_ok() { return kProgrammaticLaunch && g_call_kernels > 0; }
+
+template <class... KArgs, class... Args>
+void launch_maybe_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t st, bool pdl,
+                      Args &&...args)
+{
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr;
+    attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr.val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = &attr;
+    cfg.numAttrs = pdl ? 1 : 0;
+    cudaLaunchKernelEx(&cfg, kern, std::forward<Args>(args)...);
+}
+
+// cudaMemsetAsync on the stream; the next kernel is then launched normally.
+cudaError_t memset_async(void *p, int v, size_t n, cudaStream_t st)
+{
+    g_call_kernels = 0;
+    return cudaMemsetAsync(p, v, n, st);
 }
 
 #define NOBLE_TRY(expr)                              \
@@ -717,6 +755,7 @@ struct ProbSpec {
     int nsplit = 1;
     int kb_per_split = 0;
     bool bneck = false;  // fused bottleneck tiles: the kernel's own epilogue, no C
+    int dep = 0;         // Problem::dep: segments reading what an earlier kernel of the call wrote
 };
 
 template <int BN_MAX> struct PStagesFor { static constexpr int value = BN_MAX >= 256 ? 4 : 6; };
@@ -820,6 +859,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         q.nsplit = P.nsplit;
         q.kb_per_split = P.kb_per_split;
         q.tile_begin = tiles;
+        q.dep = P.dep;
         q.ep = eps[i];
         {
             // TMA-store epilogue where C's layout allows it
@@ -874,7 +914,12 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
     if (FUSE == tc::pair::kFuseNone) NOBLE_TRY(pair_schedule(g, clusters));
     const tc::pair::FuseArgs fargs = fa ? *fa : tc::pair::FuseArgs{};
     const KernelInfo ki{name, kBoundTensor, flops, bytes};
-    return run(st, ki, [&] { kern<<<2 * clusters, tc::pair::kPairThreads, SM::kDynamic, st>>>(maps, g, fargs); });
+    // a fused launch waits on flags that assume every cluster resident at once: launched normally
+    const bool pdl = FUSE == tc::pair::kFuseNone && pdl_ok();
+    return run(st, ki, [&] {
+        launch_maybe_pdl(kern, dim3(2 * clusters), dim3(tc::pair::kPairThreads), SM::kDynamic, st, pdl, maps, g,
+                         fargs);
+    });
 }
 
 // Runtime r -> compile-time N tile for the r-wide products.
@@ -920,6 +965,8 @@ struct SplitJobs {
 // warp sums are added in warp order -- deterministic.
 __global__ void __launch_bounds__(256) reduce_split_kernel(SplitJobs J)
 {
+    ptx::griddep_wait();  // the partials come from the preceding kernel
+    ptx::griddep_launch();
     __shared__ float sm[8][33];
     const int lane = threadIdx.x % 32, w = threadIdx.x / 32;
     const int64_t idx = (int64_t)blockIdx.x * 32 + lane;
@@ -950,6 +997,8 @@ __global__ void __launch_bounds__(256) reduce_split_kernel(SplitJobs J)
 // multiple of 4 and every pointer 16-byte aligned.
 __global__ void __launch_bounds__(256) reduce_split_vec4_kernel(SplitJobs J)
 {
+    ptx::griddep_wait();  // the partials come from the preceding kernel
+    ptx::griddep_launch();
     const int64_t n4 = J.begin[J.njobs] / 4;
     for (int64_t q = blockIdx.x * (int64_t)blockDim.x + threadIdx.x; q < n4; q += (int64_t)gridDim.x * blockDim.x) {
         const int64_t idx = q * 4;
@@ -1031,13 +1080,14 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
         NOBLE_TRY((tc_pair_group<false, false, tc::EpiStore<float>>(st, "tc_h_gemm", 1, &Ph, &Eh)));
         NOBLE_TRY(cos3_fwd_rows<bf16>(d, h, om1, ph1, M, om2, ph2, c3, saved, c, st));
         const TcSeg up{c, W_up, r};
-        const ProbSpec P{T, dout, main, &up, 256};
+        ProbSpec P{T, dout, main, &up, 256};
+        P.dep = 2;  // c, written by the bottleneck kernel
         return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
     }
     if (fuse_fwd(d)) {
         // one launch: bottleneck tiles (h, CosNet, c) and output tiles
         uint32_t *flags = (uint32_t *)(saved + SL.flags);
-        if (cudaMemsetAsync(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
+        if (memset_async(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
             return fail(NOBLE_ERR_CUDA, "flags: %s", cudaGetErrorString(cudaGetLastError()));
         tc::pair::FuseArgs fa{};
         fa.T = T, fa.r = (int)r;
@@ -1068,7 +1118,8 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
         }
     }));
     const TcSeg up{c, W_up, r};
-    const ProbSpec P{T, dout, main, &up, 256};
+    ProbSpec P{T, dout, main, &up, 256};
+    P.dep = 2;  // c, written by the bottleneck kernel
     return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
 }
 
@@ -1111,7 +1162,10 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         }
         const int64_t total = J.begin[J.njobs];
         const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
-        return run(st, kr, [&] { reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J); });
+        const bool pdl = pdl_ok();
+        return run(st, kr, [&] {
+            launch_maybe_pdl(reduce_split_kernel, dim3((unsigned)ceil_div(total, 32)), dim3(256), 0, st, pdl, J);
+        });
     };
     if (r > 0 && c3) {
         // three-layer cosine: dc = dy W_up on the tensor cores (fp32 out), the
@@ -1153,7 +1207,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     if (fused) {
         // one launch: bottleneck tiles (dc, CosNet chain rule, dh) and dx tiles
         uint32_t *flags = (uint32_t *)(ws + WL.flags);
-        if (cudaMemsetAsync(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
+        if (memset_async(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
             return fail(NOBLE_ERR_CUDA, "flags: %s", cudaGetErrorString(cudaGetLastError()));
         float *cpart = (float *)(ws + WL.cos_part);
         tc::pair::FuseArgs fa{};
@@ -1172,7 +1226,8 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     } else {
         const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
         const TcSeg sdx2{dh, W_down, r};
-        const ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
+        ProbSpec P{T, di, TcSeg{dy, W, dout}, r > 0 ? &sdx2 : nullptr, 256};
+        P.dep = r > 0 ? 2 : 0;  // dh, written by the bottleneck kernel
         if (mn4_ok({di}, {dout, r}))
             NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>, true>(st, "tc_dx", 1, &P, &px)));
         else
@@ -1190,6 +1245,9 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         int which[kWgradKinds];
         int n = 0;
         auto add = [&](int k, ProbSpec ps, float *out, int64_t ldc, bool col0) {
+            // dW_down (dh), dM (a, db), dbias (the ones operand), dM2 (a2, db2) read
+            // what earlier kernels of this call wrote; dW and dW_up read the inputs
+            ps.dep = (k == 1 || k == 3 || k == 4 || k == 5) ? 1 : 0;
             P[n] = ps;
             E[n] = {out, ldc, nullptr, 0};
             E[n].col0 = col0 ? 1 : 0;
@@ -1208,7 +1266,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
                 const bf16 *a2 = (const bf16 *)(ws + WL.a2), *db2 = (const bf16 *)(ws + WL.db2);
                 add(5, ProbSpec{r, r, TcSeg{a2, db2, T}, nullptr, r < 128 ? 128 : (int)r}, c3->dM2, r, false);
             }
-            else if (cudaMemsetAsync(dM, 0, (size_t)r * r * 4, st) != cudaSuccess)
+            else if (memset_async(dM, 0, (size_t)r * r * 4, st) != cudaSuccess)
                 return fail(NOBLE_ERR_CUDA, "dM: %s", cudaGetErrorString(cudaGetLastError()));
         }
         if (ones_dbias) add(4, ProbSpec{dout, kOnesCols, TcSeg{dy, ones, T}, nullptr, 128}, dbias, 1, true);
@@ -1247,11 +1305,13 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
                 vec4 = vec4 && J.n[i] % 4 == 0 && J.stride[i] % 4 == 0 &&
                        reinterpret_cast<uintptr_t>(J.out[i]) % 16 == 0 && reinterpret_cast<uintptr_t>(J.part[i]) % 16 == 0;
             const int64_t blocks = std::min<int64_t>(ceil_div(total / 4, 256), 8 * (int64_t)num_sms());
+            const bool pdl = pdl_ok();
             NOBLE_TRY(run(st, kr, [&] {
                 if (vec4)
-                    reduce_split_vec4_kernel<<<(unsigned)blocks, 256, 0, st>>>(J);
+                    launch_maybe_pdl(reduce_split_vec4_kernel, dim3((unsigned)blocks), dim3(256), 0, st, pdl, J);
                 else
-                    reduce_split_kernel<<<(unsigned)ceil_div(total, 32), 256, 0, st>>>(J);
+                    launch_maybe_pdl(reduce_split_kernel, dim3((unsigned)ceil_div(total, 32)), dim3(256), 0, st,
+                                     pdl, J);
             }));
         }
     }
@@ -1297,6 +1357,7 @@ static noble_status fwd_entry(const noble_linear_desc *desc, const void *x, cons
                               size_t saved_bytes, noble_stream stream, const Cos3 *c3)
 {
     g_last_error[0] = 0;
+    g_call_kernels = 0;
     NOBLE_TRY(validate_desc(desc));
     const bool br = desc->r > 0, empty = desc->T == 0;
     if (((desc->flags & kFlagSigmaCos3) != 0) != (c3 != nullptr))
@@ -1371,6 +1432,7 @@ static noble_status bwd_entry(const noble_linear_desc *desc, const void *dy, con
                               void *workspace, size_t workspace_bytes, noble_stream stream, const Cos3 *c3)
 {
     g_last_error[0] = 0;
+    g_call_kernels = 0;
     NOBLE_TRY(validate_desc(desc));
     if (((desc->flags & kFlagSigmaCos3) != 0) != (c3 != nullptr))
         return fail(NOBLE_ERR_INVALID_ARG, c3 ? "noble_linear_bwd_cos3 needs NOBLE_FLAG_SIGMA_COS3"
@@ -1630,6 +1692,7 @@ noble_status noble_test_gemm_bf16(int64_t M, int64_t N, int64_t K0, int64_t K1, 
                                   noble_stream stream)
 {
     g_last_error[0] = 0;
+    g_call_kernels = 0;
     // the innermost dimension of every operand must be a multiple of 8 elements (16 bytes)
     if (M <= 0 || N <= 0 || K0 <= 0 || K1 < 0 || nsplit < 1 || N % 8 || (a_mn && M % 8) ||
         (!(a_mn && b_mn) && (K0 % 8 || K1 % 8)))

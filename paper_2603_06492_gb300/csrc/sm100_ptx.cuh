@@ -260,6 +260,16 @@ __device__ __forceinline__ void tmem_st_32x32b_x16(uint32_t taddr, const uint32_
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+// ------------------------------------------------------------- programmatic dependent launch
+// A kernel launched with programmatic stream serialization may start while
+// its predecessor in the stream still runs (on SMs the predecessor leaves
+// free).  griddep_wait blocks the calling thread until the predecessor grid
+// has completed and its memory operations are visible; griddep_launch lets the
+// dependent grid start once every CTA of this grid has executed it (or exited).
+// Both are no-ops for a kernel launched without the attribute.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ------------------------------------------------------------- flags in global memory
 // A ready flag set by one CTA after its stores and polled by another CTA
 // before reading those stores through TMA (the async proxy).

@@ -303,6 +303,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
     const int64_t m0 = (int64_t)blockIdx.x * kBM;
 
     if (warp == 0 && lane == 0) {
+        ptx::griddep_launch();  // the next kernel of the call may take the SMs this grid leaves free
         ptx::tma_prefetch_desc(&mA);
         ptx::tma_prefetch_desc(&mB);
         for (int s = 0; s < STAGES; ++s) {

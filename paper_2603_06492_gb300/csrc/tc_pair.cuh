@@ -540,6 +540,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
     const int cluster = blockIdx.x / 2, nclusters = gridDim.x / 2;
 
     if (warp == 0 && lane == 0) {
+        ptx::griddep_launch();  // the next kernel of the call may take SMs as this grid frees them
         for (int p = 0; p < g.nproblems; ++p) {
             ptx::tma_prefetch_desc(&maps.m[p][0]);
             ptx::tma_prefetch_desc(&maps.m[p][1]);
@@ -572,6 +573,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             // ---------------- producer (both CTAs)
             uint32_t it = 0;
             bool ok = true;
+            bool waited = false;  // for the predecessor grid (programmatic launch)
             const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
             for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
                 const int t = tile_of(slot);
@@ -595,10 +597,14 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                             break;
                         }
                     }
+                    const bool seg1 = kb >= P.kb0;
+                    if (!waited && (P.dep & (seg1 ? 2 : 1))) {
+                        ptx::griddep_wait();
+                        waited = true;
+                    }
                     const uint32_t fb = map_to_rank(full_bar(s), 0);
                     if (leader) ptx::mbar_arrive_expect_tx(full_bar(s), 2 * cta_bytes);
                     const uint32_t sA = sbase + s * S::kStage, sB = sA + S::kA;
-                    const bool seg1 = kb >= P.kb0;
                     const CUtensorMap *mA = &maps.m[tr.prob][seg1 ? 2 : 0];
                     const CUtensorMap *mB = &maps.m[tr.prob][seg1 ? 3 : 1];
                     const int k = (seg1 ? kb - P.kb0 : kb) * kBK;
@@ -620,6 +626,9 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     }
                 }
             }
+            // this grid completes only after its predecessor: what later kernels
+            // of the call read through this grid's completion is then complete too
+            if (!waited) ptx::griddep_wait();
             // the leader's ring barriers also count the peer's bytes: once they
             // complete, no copy of either CTA is still landing
             if (leader) {

@@ -24,6 +24,8 @@ struct Problem {
     int tiles_m, tiles_n;  // output tiles
     int nsplit, kb_per_split;
     int tile_begin;        // first global tile index of this problem
+    int dep;               // bit s: segment s reads what an earlier kernel of the same call wrote
+                           // (the producer waits for the predecessor grid before loading it)
     EpiParams ep;
 };
 
