@@ -685,7 +685,8 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                         ok = false;
                         break;
                     }
-                    ptx::tc_fence_after();
+                    // no tcgen05 fence here: the stages were written by TMA (the
+                    // async proxy, as the MMA) and completed on the barrier waited for
                     const uint64_t so = (uint64_t)((uint32_t)s * kStageUnits);
                     const uint64_t ad = a0 + so, bd = b0 + so;
                     mma2_bf16(d_tmem, ad, bd, idesc, i > 0 ? 1u : 0u);
