@@ -53,7 +53,7 @@ WORKLOADS = {
 # DRAM bytes (read + write) per launch from one ncu capture of the current
 # kernels (profiles/traffic_config3_ffn_qkv_fwd_bwd.md), mean over the three
 # layers of config 3.
-TRAFFIC_PER_LAUNCH = {3: {"tc_wgrad": 869.7e6, "tc_main_up_fwd": 489.5e6, "tc_dx": 553.5e6}}
+TRAFFIC_PER_LAUNCH = {3: {"tc_wgrad": 869.6e6, "tc_main_up_fwd": 484.3e6, "tc_dx": 546.3e6}}
 METRIC = "NOBLE linear fwd+bwd TFLOP/s"
 
 
