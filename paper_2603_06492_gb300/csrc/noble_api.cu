@@ -758,7 +758,6 @@ struct ProbSpec {
     int dep = 0;         // Problem::dep: segments reading what an earlier kernel of the call wrote
 };
 
-template <int BN_MAX> struct PStagesFor { static constexpr int value = BN_MAX >= 256 ? 4 : 6; };
 
 
 
