@@ -977,8 +977,20 @@ __global__ void __launch_bounds__(256) reduce_split_kernel(SplitJobs J)
     const int per = (J.nparts + 7) / 8;
     const int zb = w * per, ze = min(J.nparts, zb + per);
     float s = 0.f;
-    if (in)
-        for (int z = zb; z < ze; ++z) s += J.part[j][(int64_t)z * J.stride[j] + i];
+    if (in) {
+        // eight loads in flight, then added in ascending z as before
+        const float *pp = J.part[j] + i;
+        const int64_t st = J.stride[j];
+        int z = zb;
+        for (; z + 8 <= ze; z += 8) {
+            float v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) v[u] = pp[(int64_t)(z + u) * st];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) s += v[u];
+        }
+        for (; z < ze; ++z) s += pp[(int64_t)z * st];
+    }
     sm[w][lane] = s;
     __syncthreads();
     if (w == 0 && in) {

@@ -437,8 +437,18 @@ __global__ void __launch_bounds__(256) reduce_partials(int64_t nparts, int64_t n
     const int64_t per = (nparts + 7) / 8;
     const int64_t pb = w * per, pe = min(nparts, pb + per);
     float s = 0.f;
-    if (k < n)
-        for (int64_t p = pb; p < pe; ++p) s += part[p * n + k];
+    if (k < n) {
+        // eight loads in flight, then added in ascending p
+        int64_t p = pb;
+        for (; p + 8 <= pe; p += 8) {
+            float v[8];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) v[u] = part[(p + u) * n + k];
+#pragma unroll
+            for (int u = 0; u < 8; ++u) s += v[u];
+        }
+        for (; p < pe; ++p) s += part[p * n + k];
+    }
     sm[w][lane] = s;
     __syncthreads();
     if (w == 0 && k < n) {
