@@ -139,20 +139,28 @@ class ClockSampler:
 
 
 # ------------------------------------------------------------------ oracle arm
-def oracle_sample(layers, tokens: int, seed: int = 0):
-    """The fp64 oracle's fwd+bwd on the first ``tokens`` tokens of each layer
-    (same shapes and distributions).  Returns (seconds, flops)."""
+def oracle_sample(layers, tokens: int, seed: int = 0, sigma: str = "cosnet"):
+    """The fp64 oracle's fwd+bwd, with the bottleneck variant ``sigma``, on the
+    first ``tokens`` tokens of each layer (same shapes and distributions).
+    Returns (seconds, flops)."""
     import oracle
     from paper_2603_06492_gb300.inputs import Layer, to_paper_orientation
     t_total, flops = 0.0, 0.0
     for li, layer in enumerate(layers):
         sl = Layer(layer.name, tokens, layer.d_in, layer.d_out, layer.r, layer.dtype)
         p = to_paper_orientation(make_layer_inputs(sl, seed + li))
+        if sigma == "cos3":
+            p.update(make_cos3_inputs(sl.r, seed + li + 1))
         t0 = time.perf_counter()
-        oracle.fwd(p["x"], p["W"], p["bias"], p["W_down"], p["omega1"], p["phi1"], p["M"],
-                   p["omega2"], p["phi2"], p["W_up"])
-        oracle.bwd(p["x"], p["W"], p["W_down"], p["omega1"], p["phi1"], p["M"], p["omega2"],
-                   p["phi2"], p["W_up"], p["dy"])
+        if sigma == "cos3":
+            oracle.fwd3(p["x"], p["W"], p["bias"], p)
+            oracle.bwd3(p["x"], p["W"], p, p["dy"])
+        else:
+            mode = oracle.MODES[sigma]
+            oracle.fwd(p["x"], p["W"], p["bias"], p["W_down"], p["omega1"], p["phi1"], p["M"],
+                       p["omega2"], p["phi2"], p["W_up"], mode=mode)
+            oracle.bwd(p["x"], p["W"], p["W_down"], p["omega1"], p["phi1"], p["M"], p["omega2"],
+                       p["phi2"], p["W_up"], p["dy"], mode=mode)
         t_total += time.perf_counter() - t0
         flops += sl.flops()
     return t_total, flops
@@ -179,10 +187,10 @@ def run_reference(args, rank):
     import oracle
     oracle.build()
     for _ in range(args.warmup):
-        oracle_sample(layers, args.ref_tokens)
+        oracle_sample(layers, args.ref_tokens, sigma=args.sigma)
     secs, flops = 0.0, 0.0
     for s in range(args.steps):
-        t, f = oracle_sample(layers, args.ref_tokens, seed=100 + s)
+        t, f = oracle_sample(layers, args.ref_tokens, seed=100 + s, sigma=args.sigma)
         secs += t
         flops += f
     v = flops / secs / 1e12
@@ -192,7 +200,7 @@ def run_reference(args, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "sample": sample},
+            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "sigma": args.sigma, "sample": sample},
             "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": host_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
@@ -567,7 +575,7 @@ def main():
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
-        secs, fl = oracle_sample(layers, args.cpu_tokens)
+        secs, fl = oracle_sample(layers, args.cpu_tokens, sigma=args.sigma)
         cpu = {"value": fl / secs / 1e12, "unit": "TFLOP/s", "cores": host_cores(), "kind": "oracle",
                "sample": f"fwd+bwd of the first {args.cpu_tokens} of {layers[0].T} tokens of each layer, fp64",
                "seconds": secs}

@@ -60,3 +60,14 @@ def test_reference_arm_rank0_only():
     assert r.returncode == 0, r.stderr
     line = json.loads(r.stdout.strip().splitlines()[-1])
     assert line["impl"] == "reference" and line["value"] > 0 and line["cpu_baseline"]["kind"] == "oracle"
+
+
+@pytest.mark.parametrize("sigma", ["gelu2", "cos3"])
+def test_reference_arm_times_the_variant(sigma):
+    # the oracle arm runs the bottleneck variant the flags name
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                        "--warmup", "0", "--config", "0", "--ref-tokens", "4", "--sigma", sigma],
+                       capture_output=True, text=True, timeout=300, cwd=ROOT)
+    assert r.returncode == 0, r.stderr
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    assert line["config"]["sigma"] == sigma and line["value"] > 0
