@@ -211,3 +211,29 @@ def test_cos3_flag_validation(lib):
     # h, b, b2 (fp32) and c (bf16), each 256-byte aligned
     T, r = 256, 16
     assert binding.noble_linear_saved_bytes(three) == 3 * T * r * 4 + T * r * 2
+
+
+@pytest.mark.parametrize("r", [16, 32, 64, 128, 256])
+@pytest.mark.parametrize("T", [1, 300, 4096])
+def test_saved_layout_sizes(lib, T, r):
+    # the documented saved-buffer layouts: h, b (fp32) and c; c alone for an
+    # inference forward on the tensor-core path; h, b, b2 and c for the
+    # three-layer cosine; plus one ready flag per 128 tokens (whole row pairs)
+    # when the fused bottleneck runs (CosNet, r in {64, 128})
+    al = lambda n: (n + 255) // 256 * 256
+    tr = T * r
+    flags_bytes = al(2 * ((T + 255) // 256) * 4) if r in (64, 128) else 0
+    B = binding
+    size = lambda flags, dt="bf16": B.noble_linear_saved_bytes(B.make_desc(T, 128, 128, r, dt, flags))
+    assert size(0) == al(tr * 4) * 2 + al(tr * 2)
+    assert size(0, "fp32") == al(tr * 4) * 3
+    assert size(B.NOBLE_FLAG_INFERENCE) == al(tr * 2)
+    assert size(B.NOBLE_FLAG_INFERENCE | B.NOBLE_FLAG_SIMT_ONLY) == size(0)
+    assert size(B.NOBLE_FLAG_SIGMA_COS3) == al(tr * 4) * 3 + al(tr * 2)
+    assert size(B.NOBLE_FLAG_FUSED_BRANCH) == size(0) + flags_bytes
+    assert size(B.NOBLE_FLAG_FUSED_BRANCH | B.NOBLE_FLAG_INFERENCE) == al(tr * 2) + flags_bytes
+    # the fused bottleneck is the CosNet's only: other variants keep the plain layout
+    assert size(B.NOBLE_FLAG_FUSED_BRANCH | B.NOBLE_FLAG_ACT_GELU) == size(0)
+    for flags in (0, B.NOBLE_FLAG_SIGMA_COS1, B.NOBLE_FLAG_ACT_TANH, B.NOBLE_FLAG_SIGMA_COS3,
+                  B.NOBLE_FLAG_FUSED_BRANCH, B.NOBLE_FLAG_SIMT_ONLY):
+        assert B.noble_linear_bwd_workspace_bytes(B.make_desc(T, 128, 128, r, "bf16", flags)) > 0
