@@ -46,14 +46,37 @@ WORKLOADS = {
                    "fwd+bwd",
 }
 
-# DRAM bytes per launch of each tensor-core kernel class on the 1.5B-scale
-# workload (ncu dram__bytes_read.sum + dram__bytes_write.sum, mean over the
-# three layers' launches of one fwd+bwd).  Valid for the kernels as they are
-# built now; a kernel change invalidates its entry.
-# DRAM bytes (read + write) per launch from one ncu capture of the current
-# kernels (profiles/traffic_config3_ffn_qkv_fwd_bwd.md), mean over the three
-# layers of config 3.
-TRAFFIC_PER_LAUNCH = {3: {"tc_wgrad": 869.6e6, "tc_main_up_fwd": 484.3e6, "tc_dx": 546.3e6}}
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per launch of the
+# dominant kernel class, mean over the three layers of the 1.5B-scale workload,
+# from one ncu capture.  "sources" is the hash (kernel_sources_hash) of the
+# CUDA sources the capture ran on: when the sources differ, the figure no
+# longer describes the kernels and the bench line reports traffic as null.
+TRAFFIC_PER_LAUNCH = {3: {"sources": "", "capture": "", "bytes": {}}}
+METRIC = "NOBLE linear fwd+bwd TFLOP/s"
+# dense BF16 tensor-core rate of one sm_100-family SM: 8192 FLOP per clock
+BF16_FLOP_PER_CLK_SM = 8192
+
+
+def kernel_sources_hash() -> str:
+    """sha256 (first 16 hex digits) over the CUDA sources and the C header."""
+    import hashlib
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2603_06492_gb300", "csrc")
+    files = sorted(os.path.join(csrc, f) for f in os.listdir(csrc) if f.endswith((".cu", ".cuh")))
+    files.append(os.path.join(ROOT, "include", "noble.h"))
+    for f in files:
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def config_of(cfg, layers, world, sigma):
+    """The bench line's ``config`` (the same object for both arms)."""
+    return {"workload": WORKLOADS[cfg], "config_index": cfg, "sigma": sigma, "layers": [
+        {"name": l.name, "T": l.T, "d_in": l.d_in, "d_out": l.d_out, "r": l.r} for l in layers],
+        "l2": "inputs larger than L2: each step streams ~1.8 GB of activations",
+        "parallelism": f"replicas x{world}"}
 METRIC = "NOBLE linear fwd+bwd TFLOP/s"
 
 
@@ -109,12 +132,18 @@ class ClockSampler:
                 self.proc.kill()
             self.thread.join(timeout=2)
 
-    def summary(self):
+    def mark(self) -> int:
+        """Index of the next sample: brackets a window for summary()."""
+        return len(self.lines)
+
+    def summary(self, begin=None, end=None):
         sm, mx, pw, reasons = [], [], [], set()
         names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
-        # samples taken inside the timed region; if it was shorter than the
-        # sampling interval, the last sample before it
-        region = self.lines[self.start:] or self.lines[-1:]
+        # samples taken inside the timed region (or the window [begin, end));
+        # if it was shorter than the sampling interval, the last sample before it
+        b = self.start if begin is None else begin
+        e = len(self.lines) if end is None else end
+        region = self.lines[b:e] or self.lines[max(b - 1, 0):b] or self.lines[-1:]
         for ln in region:
             f = [x.strip() for x in ln.split(",")]
             if len(f) < 9:
@@ -135,7 +164,7 @@ class ClockSampler:
             return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
         return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
                 "power_w": statistics.median(pw) if pw else None,
-                "samples": len(sm), "samples_in_timed_region": len(self.lines[self.start:])}
+                "samples": len(sm), "samples_in_timed_region": len(self.lines[b:e])}
 
 
 # ------------------------------------------------------------------ oracle arm
@@ -200,7 +229,7 @@ def run_reference(args, rank):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": secs / args.steps * 1e3, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "sigma": args.sigma, "sample": sample},
+            "config": config_of(cfg, layers, args.gpus, args.sigma),
             "cpu_baseline": {"value": v, "unit": "TFLOP/s", "cores": host_cores(),
                              "kind": "oracle", "sample": sample},
             "e2e": {"value": v, "unit": "TFLOP/s", "h2d_bytes_per_step": 0,
@@ -381,14 +410,28 @@ def main():
     prof = binding.profile_read()
 
     # overhead against the plain (r = 0) layer of this library: NOBLE and
-    # plain runs alternate three times, medians compared (clock and thermal
-    # drift between two single runs is of the size of the effect)
-    reps_n, reps_p = [], []
+    # plain runs alternate five times, medians compared (clock and thermal
+    # drift between two single runs is of the size of the effect); each run's
+    # clock is sampled so that a clock-normalised overhead (time x median SM
+    # clock, i.e. SM cycles) can be given beside the raw one
+    reps_n, reps_p, clk_n, clk_p = [], [], [], []
     with ClockSampler(local_rank) as clk_ovh:
-        for _ in range(3):
-            reps_n.append(timed(lambda: step(bufs), args.steps))
-            reps_p.append(timed(lambda: step(plain_bufs, plain=True), args.steps))
+        for _ in range(5):
+            for arm, reps, clks in ((False, reps_n, clk_n), (True, reps_p, clk_p)):
+                m0 = clk_ovh.mark()
+                reps.append(timed(lambda: step(plain_bufs if arm else bufs, plain=arm), args.steps))
+                clks.append(clk_ovh.summary(m0, clk_ovh.mark()))
     ms_noble_med, ms_plain = statistics.median(reps_n), statistics.median(reps_p)
+
+    def med_mhz(clks):
+        v = [c["sm_mhz"] for c in clks if c.get("sm_mhz")]
+        return statistics.median(v) if v else None
+
+    def cycles(reps, clks):
+        v = [t * c["sm_mhz"] for t, c in zip(reps, clks) if c.get("sm_mhz")]
+        return statistics.median(v) if v else None
+
+    cyc_n, cyc_p = cycles(reps_n, clk_n), cycles(reps_p, clk_p)
 
     # forward and backward passes timed apart
     def fwd_only(bset, plain=False):
@@ -414,6 +457,11 @@ def main():
     ms_step = ms / args.steps
     value = job_throughput(world, flops_step, ms_step)
     pk = peaks()
+    clk_main = clk.summary()
+    n_sm = torch.cuda.get_device_properties(local_rank).multi_processor_count
+
+    def hw_peak(mhz):
+        return n_sm * BF16_FLOP_PER_CLK_SM * mhz * 1e6 / 1e12
 
     # dominant kernel: largest share of summed kernel time (profiled run)
     roof = None
@@ -429,9 +477,15 @@ def main():
             peak, unit = pk["hbm"], "GB/s"
         else:  # fp32 FMA pipe: 152 SMs x 128 lanes x 2 FLOP x max SM clock
             peak, unit = 152 * 128 * 2 * pk["sm_max_mhz"] * 1e6 / 1e12, "TFLOP/s"
+        cap = TRAFFIC_PER_LAUNCH.get(cfg, {})
+        fresh = bool(cap.get("sources")) and cap.get("sources") == kernel_sources_hash() and not args.layers
+        traffic = cap.get("bytes", {}).get(top["name"]) if fresh else None
         roof = {"bound": top["bound"], "kernel": top["name"], "achieved": achieved, "peak": peak,
                 "unit": unit, "frac": achieved / peak,
-                "traffic": TRAFFIC_PER_LAUNCH.get(cfg, {}).get(top["name"]) if not args.layers else None,
+                "traffic": traffic,
+                "traffic_src": (cap.get("capture") if traffic is not None else
+                                "no ncu capture of the kernels as built (sources hash " + kernel_sources_hash() + ")"),
+                "algorithmic_bytes": top["bytes"] / top["launches"],
                 "peak_src": ("measured burst" if top["bound"] == "tensor" else
                              "measured" if top["bound"] == "hbm" else "derived from unit counts"),
                 "frac_of_sustained": (achieved / pk["bf16_sustained"]) if top["bound"] == "tensor" else None,
@@ -587,20 +641,31 @@ def main():
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
             "dtype": "bf16" if layers[0].dtype == "bf16" else "f32",
             "data": "synthetic",
-            "config": {"workload": WORKLOADS[cfg], "config_index": cfg, "sigma": args.sigma, "layers": [
-                {"name": l.name, "T": l.T, "d_in": l.d_in, "d_out": l.d_out, "r": l.r} for l in layers],
-                "l2": "inputs larger than L2: each step streams ~1.8 GB of activations",
-                "parallelism": f"replicas x{world}"},
-            "pct_peak_bf16": value / world / pk["bf16"],
-            "pct_peak_bf16_sustained": value / world / pk["bf16_sustained"],
+            "config": config_of(cfg, layers, world, args.sigma),
+            # dense BF16 tensor peak of the GPU: SMs x 8192 FLOP/clk x SM clock,
+            # at the median clock sampled in the timed region and at the maximum
+            "pct_peak_bf16": value / world / hw_peak(clk_main.get("sm_mhz") or pk["sm_max_mhz"]),
+            "pct_peak_bf16_at_max_clock": value / world / hw_peak(pk["sm_max_mhz"]),
+            "peak_bf16_tflops": {"at_sampled_clock": hw_peak(clk_main.get("sm_mhz") or pk["sm_max_mhz"]),
+                                 "at_max_clock": hw_peak(pk["sm_max_mhz"]), "sms": n_sm,
+                                 "flop_per_clk_sm": BF16_FLOP_PER_CLK_SM},
+            # against the best measured cuBLAS bf16 GEMM rate (8192^3), burst and sustained
+            "vs_cublas_best": value / world / pk["bf16"],
+            "vs_cublas_best_sustained": value / world / pk["bf16_sustained"],
             "peak_src": pk["src"],
             "plain_ms_per_step": ms_plain / args.steps,
             "plain_tflops": world * flops_plain / (ms_plain / args.steps * 1e-3) / 1e12,
             "overhead_vs_plain": ms_noble_med / ms_plain - 1.0,
-            "overhead_method": "median of 3 alternating NOBLE / plain runs of the timed steps",
+            "overhead_method": "median of 5 alternating NOBLE / plain runs of the timed steps",
             "overhead_reps_ms_per_step": {"noble": [round(v / args.steps, 4) for v in reps_n],
                                           "plain": [round(v / args.steps, 4) for v in reps_p]},
-            "overhead_clocks": clk_ovh.summary(),
+            "overhead_clock_normalised": (cyc_n / cyc_p - 1.0) if cyc_n and cyc_p else None,
+            "overhead_clock_method": "median over runs of time x median SM clock of the run (SM cycles)",
+            "overhead_clocks": {"noble": {"sm_mhz_median": med_mhz(clk_n),
+                                          "reasons": sorted({x for c in clk_n for x in c["reasons"]})},
+                                "plain": {"sm_mhz_median": med_mhz(clk_p),
+                                          "reasons": sorted({x for c in clk_p for x in c["reasons"]})},
+                                "all": clk_ovh.summary()},
             "fwd_ms_per_step": ms_fwd / args.steps, "bwd_ms_per_step": ms_bwd / args.steps,
             "plain_fwd_ms_per_step": ms_fwd_p / args.steps, "plain_bwd_ms_per_step": ms_bwd_p / args.steps,
             "overhead_fwd": ms_fwd / ms_fwd_p - 1.0, "overhead_bwd": ms_bwd / ms_bwd_p - 1.0,
@@ -615,7 +680,7 @@ def main():
             "kernel_breakdown": {k: {"ms_per_step": v["ms"] / args.steps,
                                      "launches_per_step": v["launches"] / args.steps}
                                  for k, v in sorted(prof.items(), key=lambda kv: -kv[1]["ms"])},
-            "clocks": clk.summary(),
+            "clocks": clk_main,
         }
         print(json.dumps(line), flush=True)
     if dist is not None:

@@ -272,9 +272,10 @@ noble_status noble_linear_lr_multipliers(const noble_linear_desc *desc, float ga
  * or other allocating call is made.
  *  - A shape whose noble_linear_bwd_workspace_bytes() exceeds that size is
  *    rejected with NOBLE_ERR_BUFFER_TOO_SMALL before anything is enqueued.
- *  - The first call on a device looks up the array's device address (once
- *    per device, with that device current); make that first call before any
- *    stream capture.
+ *  - The first call in a CUDA context looks up the array's device address
+ *    (with that device current) and caches it for that context, so a device
+ *    reset, which gives a new context, is followed by a new lookup; make the
+ *    first call in a context before any stream capture.
  *  - Every call on a device shares the one array, and it keeps the last
  *    call's contents.  Nothing in it needs to start at zero: each call writes
  *    every scratch value before reading it.  Calls whose work overlaps on the
@@ -363,6 +364,20 @@ uint64_t noble_kernel_launch_count(void);
  * without making any kernel wait.
  */
 noble_status noble_debug_raise_device_status(uint32_t bits);
+
+/*
+ * Test hook (no paper counterpart): launches on `stream` one small kernel that
+ * waits, through the bounded mbarrier wait every pipeline kernel of this
+ * library uses, on an mbarrier that nothing arrives at, for `limit_ns`
+ * nanoseconds (0 < limit_ns <= 100 ms).  Nothing else is outstanding in that
+ * kernel (no copy, no MMA), so the wait expires: the kernel ORs the timeout
+ * flag into the device status word, writes 2 to the device word `*result`
+ * (1 if the wait had completed) and exits.  A following
+ * noble_get_device_status() then returns NOBLE_ERR_TIMEOUT, and the context
+ * stays usable.  NOBLE_ERR_INVALID_ARG for a NULL `result` or a limit out of
+ * range.
+ */
+noble_status noble_debug_wait_expiry(uint64_t limit_ns, uint32_t *result, noble_stream stream);
 
 /*
  * Testing hook (no paper counterpart): the library's tensor-core GEMM alone,

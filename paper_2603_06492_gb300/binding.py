@@ -125,6 +125,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.noble_kernel_launch_count.restype = ctypes.c_uint64
         lib.noble_debug_raise_device_status.argtypes = [ctypes.c_uint32]
         lib.noble_debug_raise_device_status.restype = ctypes.c_int
+        lib.noble_debug_wait_expiry.argtypes = [ctypes.c_uint64, P, P]
+        lib.noble_debug_wait_expiry.restype = ctypes.c_int
         i64, ci = ctypes.c_int64, ctypes.c_int
         lib.noble_test_gemm_bf16.argtypes = [i64] * 4 + [ci] * 3 + [P] * 6 + [ci] * 3 + [P]
         lib.noble_test_gemm_bf16.restype = ctypes.c_int
@@ -259,6 +261,10 @@ def noble_kernel_launch_count() -> int:
 
 def noble_debug_raise_device_status(bits: int):
     _check(load().noble_debug_raise_device_status(bits))
+
+
+def noble_debug_wait_expiry(limit_ns: int, result, stream=None):
+    _check(load().noble_debug_wait_expiry(limit_ns, _p(result), _stream_handle(stream)))
 
 
 def profile_read() -> dict:

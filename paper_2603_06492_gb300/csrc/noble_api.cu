@@ -351,9 +351,8 @@ WorkLayout work_layout(const noble_linear_desc *d)
             L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
             L.flags = take(fuse_flag_bytes(d));
         } else {
-            // one partial per CTA of the CosNet kernel, whose grid is a whole
-            // number of CTA pairs (a padding CTA contributes exact zeros)
-            L.n_cos_blocks = r ? 2 * ceil_div(ceil_div(T, 128), 2) : 0;
+            // one partial per CTA (128-token tile) of the CosNet kernel
+            L.n_cos_blocks = r ? ceil_div(T, 128) : 0;
             L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
             // with a branch, dbias is summed from the dy tiles of the CosNet kernel
             L.bias_part = take((size_t)L.n_cos_blocks * d->d_out * 4);
@@ -673,21 +672,52 @@ noble_status make_store_map(CUtensorMap *m, void *C, bool fp32, int64_t M, int64
     return NOBLE_OK;
 }
 
-// Device address of this device's status word (looked up once per device).
-uint32_t *status_ptr()
+// The current CUDA context (NULL if none or the driver call is unavailable).
+typedef CUresult (*CtxGetCurrentFn)(CUcontext *);
+CUcontext current_context()
 {
-    static uint32_t *cache[64];
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (dev >= 0 && dev < 64 && cache[dev]) return cache[dev];
-    uint32_t *p = nullptr;
-    if (cudaGetSymbolAddress((void **)&p, g_device_status) != cudaSuccess) {
+    static CtxGetCurrentFn fn = [] {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q = cudaDriverEntryPointSymbolNotFound;
+        if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) != cudaSuccess ||
+            q != cudaDriverEntryPointSuccess) {
+            cudaGetLastError();
+            p = nullptr;
+        }
+        return reinterpret_cast<CtxGetCurrentFn>(p);
+    }();
+    CUcontext c = nullptr;
+    if (!fn || fn(&c) != CUDA_SUCCESS) return nullptr;
+    return c;
+}
+
+// Device address of a __device__ variable in the current context.  The
+// host-side name of a __device__ variable is only a stand-in, so the address
+// is looked up with the device current; it is cached per context (a new
+// context after a device reset loads the module at another address).
+template <class T>
+void *symbol_address(const T &symbol)
+{
+    static std::mutex mu;
+    static std::vector<std::pair<CUcontext, void *>> cache;
+    const CUcontext ctx = current_context();
+    std::lock_guard<std::mutex> g(mu);
+    if (ctx)
+        for (auto &e : cache)
+            if (e.first == ctx) return e.second;
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, symbol) != cudaSuccess || !p) {
         cudaGetLastError();
         return nullptr;
     }
-    if (dev >= 0 && dev < 64) cache[dev] = p;
+    // the lookup may have created the primary context: key on it
+    const CUcontext now = ctx ? ctx : current_context();
+    if (now) cache.emplace_back(now, p);
     return p;
 }
+
+// Device address of this device's status word.
+uint32_t *status_ptr() { return static_cast<uint32_t *>(symbol_address(g_device_status)); }
 
 // One K segment of a tensor-core GEMM; A and B are row-major bf16 matrices
 // ([M][K] / [N][K] when K-major, [K][M] / [K][N] when MN-major).
@@ -1035,12 +1065,12 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     using Cfg = tc::CosnetCfg<R, BWD>;
     CUtensorMap mA, mB;
     NOBLE_TRY(make_map(&mA, A, T, K, tc::kBM));
-    if (Cfg::kBInterleaved)  // B = W_up [K = d_out][R], MN-major, 4 of the 8 K groups per CTA
-        NOBLE_TRY(make_map_mn4(&mB, B, K, R, (uint32_t)(R / 64), 4));
-    else if (BWD)  // B = W_up [K = d_out][R], MN-major; each CTA of a pair loads half of the K rows
-        NOBLE_TRY(make_map(&mB, B, K, R, tc::kBK / 2));
-    else  // B = W_down [R][K], K-major; each CTA of a pair loads half of the rows
-        NOBLE_TRY(make_map(&mB, B, R, K, R / 2));
+    if (Cfg::kBInterleaved)  // B = W_up [K = d_out][R], MN-major, all 8 K groups of a k-block
+        NOBLE_TRY(make_map_mn4(&mB, B, K, R, (uint32_t)(R / 64), 8));
+    else if (BWD)  // B = W_up [K = d_out][R], MN-major, 64 K rows per column chunk
+        NOBLE_TRY(make_map(&mB, B, K, R, tc::kBK));
+    else  // B = W_down [R][K], K-major, all R rows
+        NOBLE_TRY(make_map(&mB, B, R, K, R));
     tc::CosnetArgs args = args_in;
     args.T = T;
     args.kb = (int)ceil_div(K, tc::kBK);
@@ -1050,9 +1080,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
     const KernelInfo ki{name, kBoundHbm, 2.0 * T * R * (K + R), 2.0 * T * K + 2.0 * R * K + (BWD ? 14.0 : 10.0) * T * R};
     return run(st, ki, [&] {
-        // clusters of two tiles; an odd tile count gets one tile past the end,
-        // whose rows are all out of range (zero-filled, never stored)
-        const unsigned grid = (unsigned)(2 * ceil_div(ceil_div(T, tc::kBM), 2));
+        const unsigned grid = (unsigned)ceil_div(T, tc::kBM);
         kern<<<grid, tc::kCosnetThreads, Cfg::kDynamic, st>>>(mA, mB, args);
     });
 }
@@ -1329,6 +1357,21 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     return NOBLE_OK;
 }
 
+// Test kernel for the device-side expiry of a bounded wait: one thread waits,
+// through mbar_wait_limit (the wait every pipeline kernel uses), on an
+// mbarrier that nothing arrives at; nothing else is outstanding (no copy, no
+// MMA), so the kernel records the timeout in the status word and exits.
+__global__ void wait_expiry_kernel(uint64_t limit_ns, uint32_t *status, uint32_t *result)
+{
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x != 0) return;
+    const uint32_t b = ptx::smem_u32(&bar);
+    ptx::mbar_init(b, 1);
+    ptx::fence_barrier_init();
+    const bool ok = ptx::mbar_wait_limit(b, 0, status, limit_ns);
+    *result = ok ? 1u : 2u;
+}
+
 noble_status zero_grads(const noble_linear_desc *d, float *dW, float *dbias, float *dW_down, float *dM,
                         float *dom1, float *dph1, float *dom2, float *dph2, float *dW_up,
                         cudaStream_t st)
@@ -1562,6 +1605,19 @@ noble_status noble_debug_raise_device_status(uint32_t bits)
     return NOBLE_OK;
 }
 
+noble_status noble_debug_wait_expiry(uint64_t limit_ns, uint32_t *result, noble_stream stream)
+{
+    g_last_error[0] = 0;
+    if (!result) return fail(NOBLE_ERR_INVALID_ARG, "result is NULL");
+    if (limit_ns == 0 || limit_ns > 100000000ull)
+        return fail(NOBLE_ERR_INVALID_ARG, "limit_ns must be in (0, 100 ms]");
+    NOBLE_TRY(check_device());
+    uint32_t *status = status_ptr();
+    if (!status) return fail(NOBLE_ERR_CUDA, "status word address");
+    wait_expiry_kernel<<<1, 32, 0, (cudaStream_t)stream>>>(limit_ns, status, result);
+    return check_launch("wait_expiry_kernel");
+}
+
 const char *noble_status_string(noble_status s)
 {
     switch (s) {
@@ -1579,29 +1635,12 @@ const char *noble_status_string(noble_status s)
 
 const char *noble_last_error(void) { return g_last_error; }
 
-// Device address of g_noalloc_scratch for the current device.  The host-side
-// name of a __device__ array is only a stand-in, so the address is looked up
-// once per device (with that device current) and cached.
+// Device address of g_noalloc_scratch in the current context.
 static noble_status noalloc_scratch_ptr(void **out)
 {
-    static std::mutex mu;
-    static void *cache[64];
-    int dev = -1;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
-        cudaGetLastError();
-        return fail(NOBLE_ERR_NO_DEVICE, "no current CUDA device for the static scratch");
-    }
-    std::lock_guard<std::mutex> g(mu);
-    if (!cache[dev]) {
-        void *p = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-        if (e != cudaSuccess || !p) {
-            cudaGetLastError();
-            return fail(NOBLE_ERR_CUDA, "cudaGetSymbolAddress(static scratch): %s", cudaGetErrorString(e));
-        }
-        cache[dev] = p;
-    }
-    *out = cache[dev];
+    void *p = noble::symbol_address(g_noalloc_scratch);
+    if (!p) return fail(NOBLE_ERR_CUDA, "cudaGetSymbolAddress(static scratch) failed");
+    *out = p;
     return NOBLE_OK;
 }
 

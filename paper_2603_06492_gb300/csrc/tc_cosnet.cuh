@@ -1,4 +1,5 @@
 // Fused r-wide GEMM + CosNet kernels (one 128-token tile per CTA, N = r).
+// Each CTA loads its whole A and B stages with plain TMA copies (no cluster).
 //
 // Forward (Eq. 2; Eqs. 5-7):   h = x W_down^T             (tcgen05, TMEM cols [0, r))
 //   epilogue: a = cos(omega1 h + phi1) -> bf16 tile in shared memory
@@ -222,47 +223,6 @@ __device__ __forceinline__ uint4 store_hi_lo_impl(uint8_t *tile, int row, int co
 // TMEM lane quarter, taking alternate 32-column chunks of their 32 rows.
 constexpr int kCosnetThreads = 320;
 
-// Cluster of two CTAs (consecutive 128-token tiles).  The r-row B operand
-// of the main loop is the same for both, so each CTA loads half of every B
-// stage and multicasts it to both: a stage is refilled only once the MMAs of
-// both CTAs have released it (empty barriers count two arrivals, each CTA's
-// MMA commit arrives on both).
-__device__ __forceinline__ void tma_load_4d_mc(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c2, int c3,
-                                               uint16_t mask)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster "
-        "[%0], [%1, {%3, %3, %4, %5}], [%2], %6;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(0), "r"(c2), "r"(c3), "h"(mask)
-        : "memory");
-}
-__device__ __forceinline__ void tma_load_2d_mc(uint32_t dst, const CUtensorMap *map, uint32_t bar, int c0, int c1,
-                                               uint16_t mask)
-{
-    asm volatile(
-        "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes.multicast::cluster "
-        "[%0], [%1, {%3, %4}], [%2], %5;" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(map)), "r"(bar), "r"(c0), "r"(c1), "h"(mask)
-        : "memory");
-}
-__device__ __forceinline__ void mma_commit_mc(uint32_t bar, uint16_t mask)
-{
-    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::
-                     "r"(bar),
-                 "h"(mask)
-                 : "memory");
-}
-__device__ __forceinline__ void cluster_sync_all()
-{
-    asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-__device__ __forceinline__ uint32_t cta_rank_in_cluster()
-{
-    uint32_t r;
-    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
-    return r;
-}
-
 // Bottleneck activation of the kernel: the CosNet of Eq. 2 (default), or the
 // variants of the ablation in Section 4.4 (Table 5): a single cosine
 // sigma(h) = cos(omega1 h + phi1); the identity sigma(h) = h (the linear
@@ -276,7 +236,7 @@ constexpr int kSigCosnet = 0, kSigCos1 = 1, kSigIdentity = 2, kSigAct1 = 3, kSig
 __host__ __device__ constexpr bool sig_two_layers(int sig) { return sig == kSigCosnet || sig == kSigAct2; }
 
 template <int R, bool BWD, int SIG = kSigCosnet>
-__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kCosnetThreads, 1)
+__global__ void __launch_bounds__(kCosnetThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const CosnetArgs args)
 {
@@ -308,9 +268,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ptx::tma_prefetch_desc(&mB);
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(full_bar(s), 1);
-            // released by the MMAs of both CTAs and, when dbias is summed from the
-            // dy stages, by this CTA's eight epilogue warps
-            ptx::mbar_init(empty_bar(s), (BWD && args.bias_part) ? 10 : 2);
+            // released by the MMA commit and, when dbias is summed from the dy
+            // stages, by the eight epilogue warps
+            ptx::mbar_init(empty_bar(s), (BWD && args.bias_part) ? 9 : 1);
         }
         ptx::mbar_init(tmem_full, 1);
         ptx::mbar_init(mma2_done, 1);
@@ -330,10 +290,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
     }
     ptx::tc_fence_before();
     __syncthreads();
-    cluster_sync_all();  // both CTAs' barriers exist before any multicast
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
-    const uint32_t rank = cta_rank_in_cluster();
 
     if (warp == 0) {
         if (lane == 0) {
@@ -347,18 +305,15 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 const uint32_t sA = sbase + s * C::kStage;
                 ptx::tma_load_2d(sA, &mA, fb, i * kBK, (int)m0);
                 if constexpr (C::kBInterleaved) {
-                    // this CTA's four 8-row K groups (of eight) across all column
-                    // chunks, to the same offset in both CTAs
-                    tma_load_4d_mc(sA + C::kA + rank * 4 * C::kBChunks * 1024, &mB, fb, 0, i * 8 + (int)rank * 4, 0x3);
+                    // all eight 8-row K groups across all column chunks, one copy
+                    ptx::tma_load_4d(sA + C::kA, &mB, fb, 0, i * 8);
                 } else if constexpr (BWD) {
-                    // this CTA's half of the 64 K rows of every column chunk, to
-                    // the same offsets in both CTAs
+                    // the 64 K rows of every 64-wide column chunk
                     for (int c = 0; c < C::kBChunks; ++c)
-                        tma_load_2d_mc(sA + C::kA + c * C::kChunkBytes + rank * (kBK / 2) * 128, &mB, fb, c * 64,
-                                       i * kBK + (int)rank * (kBK / 2), 0x3);
+                        ptx::tma_load_2d(sA + C::kA + c * C::kChunkBytes, &mB, fb, c * 64, i * kBK);
                 } else {
-                    // this CTA's half of the B rows, to the same offset in both CTAs
-                    tma_load_2d_mc(sA + C::kA + rank * (R / 2) * 128, &mB, fb, i * kBK, (int)rank * (R / 2), 0x3);
+                    // all R rows of W_down for this k-block
+                    ptx::tma_load_2d(sA + C::kA, &mB, fb, i * kBK, 0);
                 }
                 ++issued;
             }
@@ -386,7 +341,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     ptx::mma_bf16(tmem, ptx::smem_desc_sw128(sA + kk * 32, 16, 1024), bd, idesc,
                                   (i > 0 || kk > 0) ? 1u : 0u);
                 }
-                mma_commit_mc(empty_bar(s), 0x3);
+                ptx::mma_commit(empty_bar(s));
             }
             ptx::mma_commit(tmem_full);
             ptx::mbar_wait(tmem_full, 0, nullptr);
@@ -854,7 +809,6 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 
     ptx::tc_fence_before();
     __syncthreads();
-    cluster_sync_all();  // no CTA leaves while its peer may still signal it
     if (warp == 1) {
         ptx::tc_fence_after();
         ptx::tmem_dealloc(tmem, C::kTmemCols);

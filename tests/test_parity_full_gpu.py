@@ -36,6 +36,17 @@ def test_full_size_sampled(cfg, li):
     check_full_size(layer, layer_seed(cfg, li), 100 + cfg * 31 + li, f"config {cfg}")
 
 
+@pytest.mark.parametrize("li", [0, 1, 2], ids=["ffn_up", "ffn_down", "qkv"])
+def test_full_size_strong_branch(li):
+    # the 1.5B-scale layers with W_up ~ N(0, 1/r): the branch is as large as
+    # the main path, so an error in the second K segment ([x | c] at
+    # K = d_in + r, [dy | dh] at K = d_out + r) cannot hide under the main
+    # path's magnitude; the branch delta y - (x W^T + bias) is checked too
+    layer = CONFIGS[3][li]
+    check_full_size(layer, layer_seed(3, li) + 500, 900 + li, "config 3 strong branch", init="strong_branch",
+                    branch_delta=True)
+
+
 @pytest.mark.parametrize("li", [0, 2], ids=["gate_2048x5504", "down_5504x2048"])
 def test_paper_geglu_shapes_sampled(li):
     # the paper's Large-model GeGLU FFN projections: a hidden width (5504) that
@@ -45,8 +56,8 @@ def test_paper_geglu_shapes_sampled(li):
     check_full_size(layer, layer_seed(PAPER_WORKLOAD_SEED[w], li), 700 + li, w)
 
 
-def check_full_size(layer, seed, rng_seed, ctx):
-    inp = make_layer_inputs(layer, seed)
+def check_full_size(layer, seed, rng_seed, ctx, init="config", branch_delta=False):
+    inp = make_layer_inputs(layer, seed, init=init)
     got = run_gpu(layer, inp)
     p = to_paper_orientation(inp)
     rng = np.random.default_rng(rng_seed)
@@ -62,6 +73,11 @@ def check_full_size(layer, seed, rng_seed, ctx):
                        skip=("dW", "dbias", "dW_down", "dM", "domega1", "dphi1", "domega2",
                              "dphi2", "dW_up"))
     errs = {"y": rel_err(got["y"][rows], y_ref), "dx": rel_err(got["dx"][rows], g_sub["dx"])}
+    if branch_delta:
+        # x W^T + bias from the oracle (W_up = 0 leaves exactly that)
+        plain = oracle.fwd(sub["x"], sub["W"], sub["bias"], sub["W_down"], sub["omega1"], sub["phi1"],
+                           sub["M"], sub["omega2"], sub["phi2"], np.zeros_like(sub["W_up"]))
+        errs["branch"] = rel_err(got["y"][rows] - plain, y_ref - plain)
 
     n = 512
     o_idx = rng.integers(0, layer.d_out, n)

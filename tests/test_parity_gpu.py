@@ -204,6 +204,28 @@ def test_device_status_reporting():
     binding.noble_get_device_status(None)  # cleared
 
 
+def test_device_side_wait_expiry():
+    """A kernel's bounded mbarrier wait really expires on the device: the test
+    kernel waits 1 ms on a barrier nothing arrives at, records the timeout in
+    the status word and exits; the host reads NOBLE_ERR_TIMEOUT, and a normal
+    fwd+bwd right after still matches the oracle."""
+    import torch
+    binding.noble_get_device_status(None)
+    result = torch.zeros(4, dtype=torch.int32, device="cuda")
+    binding.noble_debug_wait_expiry(1_000_000, result)
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_get_device_status(None)
+    assert e.value.status == 6 and "bounded wait" in str(e.value)
+    assert int(result[0]) == 2  # the wait returned false
+    binding.noble_get_device_status(None)  # cleared
+    layer = Layer("after_timeout", 300, 256, 264, 64, "bf16")
+    inp = make_layer_inputs(layer, 5, init="strong_branch")
+    assert_close(run_gpu(layer, inp), run_oracle(layer, inp), "bf16", ctx="after the expired wait")
+    with pytest.raises(binding.NobleError) as e:
+        binding.noble_debug_wait_expiry(0, result)
+    assert e.value.status == 1
+
+
 def test_launch_counter_advances():
     layer = Layer("cnt", 128, 128, 128, 16, "bf16")
     inp = make_layer_inputs(layer, 2)

@@ -8,12 +8,12 @@ come back as exact zeros.
 
 LeakyReLU's derivative is a decision on the sign of h (and of b): the GPU
 takes it in fp32, the oracle in fp64, and where a pre-activation is within
-rounding of zero the two may take different branches.  The inputs are drawn
-by a seed search over the oracle's own h and b for one with no h within
-2e-5 and no b within 2e-4 of zero (relative to the largest magnitude; the
-GPU's h and b carry ~1e-6 and ~1e-5 relative error).  Where 200 seeds give
-none (two layers at the larger shapes: tens of thousands of b values), only
-the forward output y, which is continuous in h and b, is compared."""
+rounding of zero the two may take different branches.  Rows are independent,
+so the tokens whose oracle h lies within 2e-5, or b within 2e-4, of zero
+(relative to the largest magnitude; the GPU's h and b carry ~1e-6 and ~1e-5
+relative error) get a zero dy row: every term that multiplies the ambiguous
+derivative is then exactly zero on both sides, and all outputs are compared.
+The forward output y is continuous in h and b and is compared on every row."""
 import numpy as np
 import pytest
 
@@ -69,21 +69,23 @@ def oracle_variant(inp, mode):
 
 
 def variant_inputs(layer, variant, seed, init="strong_branch"):
-    """(inputs, clean): seeded inputs; for LeakyReLU the first seed from `seed`
-    whose pre-activations (the oracle's h, and b with two layers) keep away
-    from 0 (clean), else the first seed's inputs (not clean)."""
+    """Seeded inputs; for LeakyReLU, dy is zero on the tokens whose
+    pre-activations (the oracle's h, and b with two layers) come within
+    rounding of 0.  Returns (inputs, number of zeroed rows)."""
+    inp = make_layer_inputs(layer, seed, init=init)
     if not variant.startswith("leaky"):
-        return make_layer_inputs(layer, seed, init=init), True
-    for s in range(seed, seed + 200):
-        inp = make_layer_inputs(layer, s, init=init)
-        p = to_paper_orientation(inp)
-        args = [p[k] for k in ("W_down", "omega1", "phi1", "M", "omega2", "phi2", "W_up")]
-        _, h, b, _ = oracle.fwd(p["x"], p["W"], p["bias"], *args, mode=oracle.MODES[variant],
-                                want_intermediates=True)
-        pre = [(h, 2e-5)] + ([(b, 2e-4)] if variant.endswith("2") else [])
-        if all(np.min(np.abs(v)) > tol * np.max(np.abs(v)) for v, tol in pre):
-            return inp, True
-    return make_layer_inputs(layer, seed, init=init), False
+        return inp, 0
+    p = to_paper_orientation(inp)
+    args = [p[k] for k in ("W_down", "omega1", "phi1", "M", "omega2", "phi2", "W_up")]
+    _, h, b, _ = oracle.fwd(p["x"], p["W"], p["bias"], *args, mode=oracle.MODES[variant],
+                            want_intermediates=True)
+    pre = [(h, 2e-5)] + ([(b, 2e-4)] if variant.endswith("2") else [])
+    near = np.zeros(layer.T, dtype=bool)
+    for v, tol in pre:
+        near |= np.any(np.abs(v) <= tol * np.max(np.abs(v)), axis=1)
+    inp = dict(inp)
+    inp["dy"] = np.where(near[:, None], 0.0, inp["dy"]).astype(inp["dy"].dtype)
+    return inp, int(near.sum())
 
 
 @pytest.mark.parametrize("variant", sorted(VARIANTS))
@@ -93,10 +95,11 @@ def variant_inputs(layer, variant, seed, init="strong_branch"):
 def test_variant_matches_oracle(variant, dtype, shape):
     flags, mode, unused = VARIANTS[variant]
     layer = Layer(variant, *shape, dtype)
-    inp, clean = variant_inputs(layer, variant, 41)
+    inp, zeroed = variant_inputs(layer, variant, 41)
+    assert zeroed < layer.T // 4, zeroed  # most rows still carry a gradient
     got = run_variant(layer, inp, flags, unused)
     ref = oracle_variant(inp, mode)
-    assert_close(got, ref, dtype, names=None if clean else ["y"], ctx=f"{variant} {dtype} {shape}")
+    assert_close(got, ref, dtype, ctx=f"{variant} {dtype} {shape} ({zeroed} dy rows zeroed)")
     for k in ZERO[variant]:
         assert np.all(got[k] == 0), k
 
@@ -106,7 +109,6 @@ def test_variant_simt_path_agrees(variant):
     """bf16 on the CUDA-core kernels (NOBLE_FLAG_SIMT_ONLY) against the oracle too."""
     flags, mode, unused = VARIANTS[variant]
     layer = Layer(variant, 200, 136, 264, 32, "bf16")
-    inp, clean = variant_inputs(layer, variant, 43, init="config")
-    assert clean
+    inp, _ = variant_inputs(layer, variant, 43, init="config")
     got = run_variant(layer, inp, flags | binding.NOBLE_FLAG_SIMT_ONLY, unused)
     assert_close(got, oracle_variant(inp, mode), "bf16", ctx=f"{variant} simt")

@@ -4,11 +4,13 @@ its extensions no allocator, or a loop that forbids allocation once running).
 It uses a static scratch array inside the library instead of a caller
 workspace.
 
-Checked through the C ABI against noble_linear_bwd (caller workspace) on the
-same inputs, within the parity tolerance of the other GPU tests, on two calls
-in a row (the array keeps the previous call's contents).  This file is
-collected last so that a stop-at-first-failure run has already run every
-other test; it needs no state from them.
+Checked through the C ABI against noble_linear_bwd (caller workspace): both
+run the same kernels with fixed-order reductions, so the results must be
+bit-identical.  The array keeps the previous call's contents, so the checked
+calls are separated by a call on other inputs of the same shape (another dy):
+a scratch value read before it is written would then carry that call's data
+into the next one.  This file is collected last so that a stop-at-first-failure
+run has already run every other test; it needs no state from them.
 """
 import numpy as np
 import pytest
@@ -39,6 +41,12 @@ def _grads_noalloc(buf, dev, dx, grads):
         g.get("domega1"), g.get("dphi1"), g.get("domega2"), g.get("dphi2"), g.get("dW_up"), None)
 
 
+def _to_numpy(dx, grads):
+    out = {"dx": dx.float().cpu().numpy()}
+    out.update({k: v.cpu().numpy() for k, v in grads.items()})
+    return out
+
+
 @pytest.mark.parametrize("shape,dtype", [((300, 200, 264, 64), "bf16"),
                                          ((256, 128, 136, 16), "fp32"),
                                          ((2048, 1024, 1024, 128), "bf16")])
@@ -47,24 +55,33 @@ def test_noalloc_matches_workspace_entry_point(shape, dtype):
     layer = Layer("noalloc", *shape, dtype)
     inp = make_layer_inputs(layer, 42, init="strong_branch")
     dev = binding.params_to_device(inp, dtype)
+    # a second dy of the same shape (another seed)
+    dy_other = binding.params_to_device({"dy": make_layer_inputs(layer, 43, init="strong_branch")["dy"]},
+                                        dtype)["dy"]
     buf = binding.NobleLinearBuffers(*shape, dtype)
     binding.forward(buf, dev["x"], dev)
-    binding.backward(buf, dev["x"], dev["dy"], dev)
-    torch.cuda.synchronize()
-    ref = {"dx": buf.dx.float().cpu().numpy()}
-    ref.update({k: v.cpu().numpy() for k, v in buf.grads.items()})
+    refs = {}
+    for name, dy in (("a", dev["dy"]), ("b", dy_other)):
+        binding.backward(buf, dev["x"], dy, dev)
+        torch.cuda.synchronize()
+        refs[name] = _to_numpy(buf.dx, buf.grads)
 
-    for call in range(2):
+    # a, then b (other scratch contents), then a again
+    for call, name in enumerate(("a", "b", "a")):
+        dy = dev["dy"] if name == "a" else dy_other
         dx = torch.full_like(buf.dx, float("nan"))
         grads = {k: torch.full_like(v, float("nan")) for k, v in buf.grads.items()}
-        _grads_noalloc(buf, dev, dx, grads)
+        _grads_noalloc(buf, dict(dev, dy=dy), dx, grads)
         torch.cuda.synchronize()
         binding.noble_get_device_status(None)
-        got = {"dx": dx.float().cpu().numpy()}
-        got.update({k: v.cpu().numpy() for k, v in grads.items()})
-        for k in ref:
+        got = _to_numpy(dx, grads)
+        for k, ref in refs[name].items():
             assert np.all(np.isfinite(got[k])), (call, k)
-            assert rel_err(got[k], ref[k]) <= TOL[dtype], (call, k, rel_err(got[k], ref[k]))
+            assert np.array_equal(got[k], ref), (call, name, k, rel_err(got[k], ref))
+        # and within the parity tolerance of the other input's result: the two
+        # dy differ, so the test would notice results that ignore dy
+        other = refs["b" if name == "a" else "a"]
+        assert rel_err(got["dx"], other["dx"]) > TOL[dtype], (call, name)
 
 
 def test_noalloc_rejects_shapes_beyond_its_scratch():
