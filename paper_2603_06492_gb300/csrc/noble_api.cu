@@ -210,14 +210,32 @@ size_t esize(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 ? 2 : 4
 bool use_tc(const noble_linear_desc *d) { return d->dtype == NOBLE_BF16 && !(d->flags & kFlagSimtOnly); }
 
 // Tensor-core launches that run the bottleneck inside the output GEMM
-// (tc_pair.cuh, FUSE), on request: the CosNet with r in {64, 128}.  The
-// backward's MN-major operands also need d_in a multiple of 64 (4-D TMA layout).
+// (tc_pair.cuh, FUSE), on request: the CosNet with r in {64, 128}, whose
+// leader tiles hold the first r output columns (d_out >= r).  The backward's
+// MN-major operands also need d_in a multiple of 64 (4-D TMA layout) and
+// d_in >= r.
 bool fuse_fwd(const noble_linear_desc *d)
 {
     return use_tc(d) && sigma_of(d).sig == tc::kSigCosnet && !is_cos3(d) && (d->r == 64 || d->r == 128) && d->T > 0 &&
-           (d->flags & kFlagFusedBranch);
+           d->d_out >= d->r && (d->flags & kFlagFusedBranch);
 }
-bool fuse_bwd(const noble_linear_desc *d) { return fuse_fwd(d) && d->d_in % 64 == 0; }
+bool fuse_bwd(const noble_linear_desc *d)
+{
+    return use_tc(d) && sigma_of(d).sig == tc::kSigCosnet && !is_cos3(d) && (d->r == 64 || d->r == 128) && d->T > 0 &&
+           d->d_in >= d->r && d->d_in % 64 == 0 && (d->flags & kFlagFusedBranch);
+}
+// Output columns of a fused launch after the leader's first r: nfull in
+// 256-wide tiles, then a last part of at most 128 columns (if any) in
+// 128-wide tiles, so that no tile multiplies more than 128 empty columns.
+struct FusedSplit {
+    int64_t nfull, ntail;
+};
+FusedSplit fused_split(int64_t n, int64_t r)
+{
+    const int64_t rest = n - r, rem = rest % 256;
+    if (rem > 0 && rem <= 128) return {rest - rem, rem};
+    return {rest, 0};
+}
 // ready flags of a fused launch: one per 128-row block of whole row pairs
 size_t fuse_flag_bytes(const noble_linear_desc *d) { return (size_t)(2 * ((d->T + 255) / 256)) * 4; }
 
@@ -344,12 +362,15 @@ WorkLayout work_layout(const noble_linear_desc *d)
         L.a = take(tr * 2);
         L.db = take(tr * 2);
         const bool fused = fuse_bwd(d);
-        L.ones = (r && !fused) ? 0 : take((size_t)T * kOnesCols * 2);  // dbias = dy^T 1
+        L.ones = r ? 0 : take((size_t)T * kOnesCols * 2);  // dbias = dy^T 1
         if (fused) {
-            // one partial per 32 tokens (an epilogue warp's rows)
+            // CosNet sums per 32 tokens (an epilogue warp's rows), dbias
+            // partials per 128 tokens (a CTA's rows of a leader tile)
             L.n_cos_blocks = ceil_div(T, 32);
             L.cos_part = take((size_t)L.n_cos_blocks * 4 * r * 4);
             L.flags = take(fuse_flag_bytes(d));
+            L.n_bias_chunks = ceil_div(T, 128);
+            L.bias_part = take((size_t)L.n_bias_chunks * d->d_out * 4);
         } else {
             // one partial per CTA (128-token tile) of the CosNet kernel
             L.n_cos_blocks = r ? ceil_div(T, 128) : 0;
@@ -607,12 +628,14 @@ EncodeTiledFn encode_fn()
 
 // 2-D TMA map over a row-major bf16 matrix [rows][cols]: box of 64 columns
 // (128 bytes) by box_rows rows, 128-byte swizzle, zero fill out of bounds.
-noble_status make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t cols, uint32_t box_rows)
+// `pitch` is the row pitch in elements (0: cols, a contiguous matrix).
+noble_status make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t cols, uint32_t box_rows,
+                      int64_t pitch = 0)
 {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
     cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
-    cuuint64_t strides[1] = {(cuuint64_t)cols * 2};
+    cuuint64_t strides[1] = {(cuuint64_t)(pitch ? pitch : cols) * 2};
     cuuint32_t box[2] = {64, box_rows};
     cuuint32_t estr[2] = {1, 1};
     CUresult r = enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
@@ -629,14 +652,15 @@ noble_status make_map(CUtensorMap *m, const void *ptr, int64_t rows, int64_t col
 // dimensions (inner first) {64 elements, 8 rows, MN/64 chunks, K/8 groups} with
 // strides {P, 128 B, 8 P} for the row pitch P, box {64, 8, nchunks, kgroups}.
 // Requires MN % 64 == 0 and K % 8 == 0, so that every in-range coordinate of
-// the 4-D description is an element of the matrix.
+// the 4-D description is an element of the matrix.  `pitch` (elements, 0: MN)
+// allows a column range of a wider matrix.
 noble_status make_map_mn4(CUtensorMap *m, const void *ptr, int64_t K, int64_t MN, uint32_t nchunks,
-                          uint32_t kgroups = 8)
+                          uint32_t kgroups = 8, int64_t pitch = 0)
 {
     EncodeTiledFn enc = encode_fn();
     if (!enc) return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
     if (MN % 64 || K % 8) return fail(NOBLE_ERR_INVALID_ARG, "4-D MN-major map needs MN %% 64 == 0 and K %% 8 == 0");
-    const cuuint64_t P = (cuuint64_t)MN * 2;
+    const cuuint64_t P = (cuuint64_t)(pitch ? pitch : MN) * 2;
     cuuint64_t dims[4] = {64, 8, (cuuint64_t)MN / 64, (cuuint64_t)K / 8};
     cuuint64_t strides[3] = {P, 128, 8 * P};
     cuuint32_t box[4] = {64, 8, nchunks, kgroups};
@@ -724,6 +748,7 @@ uint32_t *status_ptr() { return static_cast<uint32_t *>(symbol_address(g_device_
 struct TcSeg {
     const void *A, *B;
     int64_t K;
+    int64_t ldb = 0;  // row pitch of B in elements (0: contiguous); MN-major B only
 };
 
 template <int BN> struct StagesFor { static constexpr int value = BN >= 256 ? 4 : BN >= 128 ? 6 : 8; };
@@ -784,8 +809,11 @@ struct ProbSpec {
     int bn;           // N tile (multiple of 32; of 64 when B is MN-major)
     int nsplit = 1;
     int kb_per_split = 0;
-    bool bneck = false;  // fused bottleneck tiles: the kernel's own epilogue, no C
     int dep = 0;         // Problem::dep: segments reading what an earlier kernel of the call wrote
+    // fused bottleneck launch, leader problem: segment 0's B operand of CTA
+    // rank 1 (the branch weights; N = r rows or columns, like rank 0's)
+    const void *B0_rank1 = nullptr;
+    int64_t B0_rank1_ld = 0;
 };
 
 
@@ -864,18 +892,30 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         if (P.M == 0 || P.N == 0) continue;
         if (P.bn != 128 && P.bn != 256) return fail(NOBLE_ERR_INVALID_ARG, "%s: pair tile width %d", name, P.bn);
         const uint32_t bh = (uint32_t)P.bn / 2;
-        auto mk = [&](CUtensorMap *m, const void *p, bool mn, int64_t mnrows, int64_t K, uint32_t box_rows) {
-            if (mn && MN4) return make_map_mn4(m, p, K, mnrows, box_rows / 64);
-            return mn ? make_map(m, p, K, mnrows, 64) : make_map(m, p, mnrows, K, box_rows);
+        auto mk = [&](CUtensorMap *m, const void *p, bool mn, int64_t mnrows, int64_t K, uint32_t box_rows,
+                      int64_t ld = 0) {
+            if (mn && MN4) return make_map_mn4(m, p, K, mnrows, box_rows / 64, 8, ld);
+            return mn ? make_map(m, p, K, mnrows, 64, ld) : make_map(m, p, mnrows, K, box_rows);
         };
+        // a fused launch's leader problem multiplies N = 2r columns (r of the
+        // output, r of the branch); its output tile is the first r
+        const bool lead = FUSE != tc::pair::kFuseNone && i == 0;
+        const int64_t nb_rows = lead ? P.bn / 2 : P.N;
         NOBLE_TRY(mk(&maps.m[np][0], P.s0.A, A_MN, P.M, P.s0.K, tc::kBM));
-        NOBLE_TRY(mk(&maps.m[np][1], P.s0.B, B_MN, P.N, P.s0.K, bh));
+        NOBLE_TRY(mk(&maps.m[np][1], P.s0.B, B_MN, nb_rows, P.s0.K, bh, P.s0.ldb));
         if (P.s1) {
             NOBLE_TRY(mk(&maps.m[np][2], P.s1->A, A_MN, P.M, P.s1->K, tc::kBM));
-            NOBLE_TRY(mk(&maps.m[np][3], P.s1->B, B_MN, P.N, P.s1->K, bh));
+            NOBLE_TRY(mk(&maps.m[np][3], P.s1->B, B_MN, nb_rows, P.s1->K, bh, P.s1->ldb));
         } else {
             maps.m[np][2] = maps.m[np][0];
             maps.m[np][3] = maps.m[np][1];
+        }
+        if (lead) {
+            if (!P.B0_rank1 || !P.s1 || P.bn != 2 * P.N)
+                return fail(NOBLE_ERR_INVALID_ARG, "%s: fused leader problem", name);
+            NOBLE_TRY(mk(&maps.m[np][5], P.B0_rank1, B_MN, nb_rows, P.s0.K, bh, P.B0_rank1_ld));
+        } else {
+            maps.m[np][5] = maps.m[np][1];
         }
         auto &q = g.p[np];
         q.M = P.M;
@@ -895,7 +935,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
             using OutT = typename Epi::out_type;
             constexpr int64_t es = sizeof(OutT);
             const auto &e = eps[i];
-            const bool ok = !P.bneck && !e.col0 && reinterpret_cast<uintptr_t>(e.C) % 16 == 0 &&
+            const bool ok = !e.col0 && reinterpret_cast<uintptr_t>(e.C) % 16 == 0 &&
                             (e.ldc * es) % 16 == 0 && P.N % 4 == 0 &&
                             (P.nsplit == 1 || (e.split_stride * es) % 16 == 0);
             q.ep.tma = ok ? 1 : 0;
@@ -906,6 +946,11 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         const double K = (double)P.s0.K + (P.s1 ? (double)P.s1->K : 0.0);
         flops += 2.0 * P.M * P.N * K;
         bytes += 2.0 * (P.M + P.N) * K;
+        if (lead) {
+            // the branch's product in segment 0 and the r x r product (three terms)
+            flops += 2.0 * P.M * P.N * (double)P.s0.K + 3.0 * 2.0 * P.M * P.N * P.N;
+            bytes += 2.0 * P.N * (double)P.s0.K;
+        }
         ++np;
     }
     if (np == 0) return NOBLE_OK;
@@ -939,7 +984,7 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
         if (dev >= 0 && dev < 64) max_clusters_cache[dev] = max_clusters;
     }
     const int clusters = tiles < max_clusters ? tiles : max_clusters;
-    // a fused launch walks its own dependency order (tc_pair.cuh: fused_tile)
+    // a fused launch walks its own dependency order (tc_pair.cuh: share_tile)
     if (FUSE == tc::pair::kFuseNone) NOBLE_TRY(pair_schedule(g, clusters));
     const tc::pair::FuseArgs fargs = fa ? *fa : tc::pair::FuseArgs{};
     const KernelInfo ki{name, kBoundTensor, flops, bytes};
@@ -987,6 +1032,7 @@ struct SplitJobs {
     float *out[5];
     int64_t n[5], stride[5], begin[6];  // stride: elements between consecutive partials
     int nparts;
+    int jparts[5];  // partials of job j when non-zero (else nparts; reduce_split_kernel only)
     int njobs;
 };
 // Block = 8 warps over 32 consecutive outputs: warp w adds partials
@@ -1004,8 +1050,9 @@ __global__ void __launch_bounds__(256) reduce_split_kernel(SplitJobs J)
     if (in)
         while (idx >= J.begin[j + 1]) ++j;
     const int64_t i = in ? idx - J.begin[j] : 0;
-    const int per = (J.nparts + 7) / 8;
-    const int zb = w * per, ze = min(J.nparts, zb + per);
+    const int np = J.jparts[j] ? J.jparts[j] : J.nparts;
+    const int per = (np + 7) / 8;
+    const int zb = w * per, ze = min(np, zb + per);
     float s = 0.f;
     if (in) {
         // eight loads in flight, then added in ascending z as before
@@ -1124,7 +1171,9 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
         return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
     }
     if (fuse_fwd(d)) {
-        // one launch: bottleneck tiles (h, CosNet, c) and output tiles
+        // one launch: per row pair a leader tile x [W rows 0..r ; W_down]^T (the
+        // first r output columns, h beside them; CosNet in its epilogue, then
+        // + c W_up^T), and the output tiles of columns [r, d_out)
         uint32_t *flags = (uint32_t *)(saved + SL.flags);
         if (memset_async(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
             return fail(NOBLE_ERR_CUDA, "flags: %s", cudaGetErrorString(cudaGetLastError()));
@@ -1133,11 +1182,17 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
         fa.om1 = om1, fa.ph1 = ph1, fa.om2 = om2, fa.ph2 = ph2, fa.M = M;
         fa.h_out = SL.only_c ? nullptr : h, fa.b_out = SL.only_c ? nullptr : b, fa.c_out = c;
         fa.flags = flags;
-        const TcSeg up{c, W_up, r};
-        ProbSpec P[2] = {ProbSpec{T, r, TcSeg{x, W_down, di}, nullptr, 128}, ProbSpec{T, dout, main, &up, 256}};
-        P[0].bneck = true;
-        const tc::EpiStore<bf16>::Params E[2] = {{nullptr, 0, nullptr, 0}, py};
-        return tc_pair_group<false, false, tc::EpiStore<bf16>, false, tc::pair::kFuseFwd>(st, "tc_main_up_fwd", 2, P,
+        // columns [r, r + nf) in 256-wide tiles, a last part of at most 128 in 128-wide ones
+        const FusedSplit fs = fused_split(dout, r);
+        const int64_t o2 = r + fs.nfull;
+        const TcSeg up0{c, W_up, r}, up1{c, W_up + r * r, r}, up2{c, W_up + o2 * r, r};
+        ProbSpec P[3] = {ProbSpec{T, r, main, &up0, 2 * (int)r},
+                         ProbSpec{T, fs.nfull, TcSeg{x, W + r * di, di}, &up1, 256},
+                         ProbSpec{T, fs.ntail, TcSeg{x, W + o2 * di, di}, &up2, 128}};
+        P[0].B0_rank1 = W_down;
+        const tc::EpiStore<bf16>::Params E[3] = {py, {y + r, dout, bias ? bias + r : nullptr, 0},
+                                                 {y + o2, dout, bias ? bias + o2 : nullptr, 0}};
+        return tc_pair_group<false, false, tc::EpiStore<bf16>, false, tc::pair::kFuseFwd>(st, "tc_main_up_fwd", 3, P,
                                                                                            E, &fa);
     }
     tc::CosnetArgs a{};
@@ -1174,7 +1229,7 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
     bf16 *ones = (bf16 *)(ws + WL.ones);
     const bool fused = fuse_bwd(d);
-    const bool ones_dbias = dbias && (r == 0 || fused || c3);
+    const bool ones_dbias = dbias && (r == 0 || c3);
     const Sigma sg = sigma_of(d);
     if (ones_dbias) NOBLE_TRY(fill_ones(st, T * kOnesCols, ones));
     // domega1, dphi1, domega2, dphi2 (and dbias) from per-CTA or per-32-token partials
@@ -1198,6 +1253,8 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             J.stride[4] = dout;
             J.begin[5] = J.begin[4] + dout;
             J.njobs = 5;
+            // the fused launch keeps dbias partials per 128 tokens
+            if (fused) J.jparts[4] = (int)WL.n_bias_chunks;
         }
         const int64_t total = J.begin[J.njobs];
         const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
@@ -1244,24 +1301,36 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     }
     // dx = [dy | dh] [W ; W_down]
     if (fused) {
-        // one launch: bottleneck tiles (dc, CosNet chain rule, dh) and dx tiles
+        // one launch: per row pair a leader tile dy [W cols 0..r | W_up] (the
+        // first r columns of dx, dc beside them; the CosNet chain rule and the
+        // dbias partials in its epilogue, then + dh W_down), and the dx tiles
+        // of columns [r, d_in)
         uint32_t *flags = (uint32_t *)(ws + WL.flags);
         if (memset_async(flags, 0, fuse_flag_bytes(d), st) != cudaSuccess)
             return fail(NOBLE_ERR_CUDA, "flags: %s", cudaGetErrorString(cudaGetLastError()));
         float *cpart = (float *)(ws + WL.cos_part);
+        float *bpart = (float *)(ws + WL.bias_part);
         tc::pair::FuseArgs fa{};
         fa.T = T, fa.r = (int)r;
         fa.om1 = om1, fa.ph1 = ph1, fa.om2 = om2, fa.ph2 = ph2, fa.M = M;
         fa.h_in = (const float *)(saved + SL.h), fa.b_in = (const float *)(saved + SL.b);
         fa.dh_out = dh, fa.a_out = a, fa.db_out = db, fa.part = cpart, fa.flags = flags;
-        const tc::EpiStore<bf16>::Params E[2] = {{nullptr, 0, nullptr, 0}, {dx, di, nullptr, 0}};
-        const TcSeg sdx2{dh, W_down, r};
-        ProbSpec P[2] = {ProbSpec{T, r, TcSeg{dy, W_up, dout}, nullptr, 128},
-                         ProbSpec{T, di, TcSeg{dy, W, dout}, &sdx2, 256}};
-        P[0].bneck = true;
-        NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>, true, tc::pair::kFuseBwd>(st, "tc_dx", 2, P, E,
+        fa.bias_part = dbias ? bpart : nullptr;
+        fa.kdim = dout;
+        const FusedSplit fs = fused_split(di, r);
+        const int64_t o2 = r + fs.nfull;
+        const tc::EpiStore<bf16>::Params E[3] = {
+            {dx, di, nullptr, 0}, {dx + r, di, nullptr, 0}, {dx + o2, di, nullptr, 0}};
+        // MN-major B operands: column ranges of W [d_out][d_in] and W_down [r][d_in]
+        const TcSeg s0L{dy, W, dout, di}, s1L{dh, W_down, r, di};
+        const TcSeg s0O{dy, W + r, dout, di}, s1O{dh, W_down + r, r, di};
+        const TcSeg s0T{dy, W + o2, dout, di}, s1T{dh, W_down + o2, r, di};
+        ProbSpec P[3] = {ProbSpec{T, r, s0L, &s1L, 2 * (int)r}, ProbSpec{T, fs.nfull, s0O, &s1O, 256},
+                         ProbSpec{T, fs.ntail, s0T, &s1T, 128}};
+        P[0].B0_rank1 = W_up;
+        NOBLE_TRY((tc_pair_group<false, true, tc::EpiStore<bf16>, true, tc::pair::kFuseBwd>(st, "tc_dx", 3, P, E,
                                                                                            &fa)));
-        NOBLE_TRY(reduce_cosnet(cpart, nullptr));
+        NOBLE_TRY(reduce_cosnet(cpart, dbias ? bpart : nullptr));
     } else {
         const tc::EpiStore<bf16>::Params px{dx, di, nullptr, 0};
         const TcSeg sdx2{dh, W_down, r};

@@ -20,28 +20,36 @@
 //     arrives on the LEADER's `tempty` (16 arrivals: 8 warps x 2 CTAs).
 // All waits are bounded as in the single-CTA kernels.
 //
-// Fused bottleneck (FUSE = kFuseFwd / kFuseBwd, on request through
-// NOBLE_FLAG_FUSED_BRANCH; the separate kernels of tc_cosnet.cuh are the
-// default because they are faster at the measured shapes): problem 0 of the launch is
-// the r-wide GEMM of the low-rank branch, h = x W_down^T (forward) or
-// dc = dy W_up (backward), one 256 x r tile per row pair, and problem 1 the
-// output GEMM whose second K segment reads c = CosNet(h) (forward, Eq. 1-2)
-// or dh (backward) of the same rows.  A bottleneck tile's epilogue runs the
-// CosNet of Eq. 2 (or its chain rule) on the accumulator:
+// Fused bottleneck (FUSE = kFuseFwd / kFuseBwd, the CosNet with r in {64, 128}):
+// the r-wide product of the low-rank branch, h = x W_down^T (forward) or
+// dc = dy W_up (backward), shares the A stages of the output GEMM instead of
+// streaming x or dy once more.  Problem 0 of the launch holds one "leader"
+// tile per row pair, of N = 2r: its B operand is [W rows 0..r ; W_down] (CTA
+// rank 0 loads the first r rows, rank 1 the branch's r rows), so one MMA
+// stream yields the output columns [0, r) and the branch pre-activation side
+// by side in TMEM.  Problem 1 holds the remaining output columns [r, N_out).
+// A leader's epilogue, after its first K segment:
+//   park      the output columns [0, r) in registers
 //   phase 1   a = cos(omega1 h + phi1)      | du2 = -sin(omega2 b + phi2) dc,
 //                                           |   db = omega2 du2
-//             as bf16 high and low parts written back into TMEM columns [0, r)
+//             as bf16 high and low parts written back into TMEM columns [r, 2r)
 //   product   b = a M  (or da = db M^T), a second pair MMA with A in TMEM and
 //             the mixing matrix (bf16 high/low, this CTA's half of its
-//             columns) in the epilogue staging buffer, into columns
-//             [128, 128 + r) of the same accumulator
+//             columns) in the epilogue staging buffer, into columns [0, r)
 //   phase 2   c = cos(omega2 b + phi2)      | du1 = -sin(omega1 h + phi1) da,
 //                                           |   dh = omega1 du1, a = cos(u1)
+//   restore   the parked columns into [0, r)
 // then stores c (dh) for its 128 rows and releases a flag per 128-row block.
-// The producer of an output tile polls that flag (bounded) before loading
-// its second segment.  Tiles run in the order of fused_tile, which puts
-// every bottleneck tile before the output tiles that wait for it, so with all
-// clusters resident every wait ends.
+// Every tile's second K segment (c W_up^T, or dh W_down) waits for that flag
+// in the producer.  The MMA warp issues the leader's second segment only
+// after the next tile's first segment, so the tensor pipe keeps working while
+// the epilogue runs the bottleneck; it issues the second product when the
+// epilogue signals its operand ready, polling between k-blocks.  In the
+// backward the epilogue warps also sum dy's columns over each leader stage
+// (dbias partials per 128 rows) before the stage is released.
+// Tiles run in the order of share_tile: waves of leaders, each followed by
+// the output tiles of its row pairs, so with all clusters resident every
+// flag wait ends.
 #pragma once
 
 #include "tc_persistent.cuh"
@@ -180,7 +188,6 @@ __device__ __forceinline__ PairTile locate_pair(const GroupArgs<EpiParams> &g, i
 }
 
 constexpr int kFuseNone = 0, kFuseFwd = 1, kFuseBwd = 2;
-constexpr uint32_t kR2Col = 128;  // TMEM column of the bottleneck's second accumulator
 
 struct FuseArgs {
     int64_t T;
@@ -192,37 +199,47 @@ struct FuseArgs {
     const float *h_in, *b_in;    // backward: saved h, b
     __nv_bfloat16 *dh_out, *a_out, *db_out;
     float *part;                 // backward: [ceil(T / 32)][4][r] column sums per 32 tokens
+    float *bias_part;            // backward: [ceil(T / 128)][kdim] column sums of dy, or NULL
+    int64_t kdim;                // backward: columns of dy (d_out)
     uint32_t *flags;             // [2 * row pairs], zero at launch
 };
 
-// Fused tile order: the bottleneck tiles of row-pair group 0, then for each
-// group g the bottleneck tiles of group g + 1 followed by the output tiles of
-// group g (groups of 8 row pairs as in locate_pair).
+// Fused tile order over `slot` (0 .. total tiles), in chunks of W row pairs,
+// W = 8 floor(clusters / 8) (at least 8): the leader tiles (problem 0) of
+// chunk 0, then for each chunk k the leaders of chunk k + 1 followed by the
+// output tiles of chunk k (problems 1, 2, ..., each in locate_pair's group
+// walk, which keeps groups of 8 row pairs together).  Every output tile thus
+// comes at least one chunk of leaders after its own leader.
 template <class EpiParams>
-__device__ __forceinline__ int fused_tile(const GroupArgs<EpiParams> &g, int p)
+__device__ __forceinline__ int share_tile(const GroupArgs<EpiParams> &g, int p, int nclusters)
 {
-    const Problem<EpiParams> &C = g.p[0], &O = g.p[1];
-    const int pairs = (C.tiles_m + 1) / 2;
-    const int ng = (pairs + 7) / 8;
-    const int tn = O.tiles_n;
-    const int c0 = min(8, pairs);
-    if (p < c0) return C.tile_begin + p;
-    p -= c0;
-    // block gi = [C(gi + 1)] [O(gi)]; blocks below ng - 2 are all 8 + 8 tn long
-    const int full = 8 + 8 * tn;
-    int gi = 0;
-    if (ng > 2) {
-        gi = min(p / full, ng - 2);
-        p -= gi * full;
-    }
+    const Problem<EpiParams> &L = g.p[0];
+    const int pairs = (L.tiles_m + 1) / 2;
+    int tn = 0;
+    for (int q = 1; q < g.nproblems; ++q) tn += g.p[q].tiles_n;
+    int W = (nclusters / 8) * 8;
+    if (W < 8) W = 8;
+    const int K = (pairs + W - 1) / W;
+    auto nl = [&](int k) { return min(W, pairs - k * W); };
+    if (p < nl(0)) return L.tile_begin + p;
+    p -= nl(0);
 #pragma unroll 1
-    for (; gi < ng; ++gi) {
-        const int cn = gi + 1 < ng ? min(8, pairs - 8 * (gi + 1)) : 0;
-        const int on = min(8, pairs - 8 * gi) * tn;
-        if (p < cn) return C.tile_begin + 8 * (gi + 1) + p;
-        p -= cn;
-        if (p < on) return O.tile_begin + 8 * gi * tn + p;
-        p -= on;
+    for (int k = 0; k < K; ++k) {
+        if (k + 1 < K) {
+            const int n = nl(k + 1);
+            if (p < n) return L.tile_begin + (k + 1) * W + p;
+            p -= n;
+        }
+        const int n = nl(k);
+        if (p < n * tn) {
+#pragma unroll 1
+            for (int q = 1; q < g.nproblems; ++q) {
+                const int m = n * g.p[q].tiles_n;
+                if (p < m) return g.p[q].tile_begin + k * W * g.p[q].tiles_n + p;
+                p -= m;
+            }
+        }
+        p -= n * tn;
     }
     return -1;
 }
@@ -250,60 +267,69 @@ __device__ __forceinline__ int slot_tile(const GroupArgs<EpiParams> &g, int slot
 // Warps 0 (TMA), 1 (MMA, TMEM owner) and eight epilogue warps.
 constexpr int kPairThreads = 320;
 
+// Order in which a cluster issues the K segments of its tiles in a fused
+// launch (producer and MMA warp alike; the epilogue warps replay it to know
+// the ring position of a leader's stages).  Segment 0 of every tile comes in
+// tile order.  Segment 1 of a deferred tile -- a leader, or the cluster's
+// first tile -- comes only after the next tile's segment 0 (or before it,
+// when that tile is deferred too), so that a leader's bottleneck epilogue,
+// or the leader a first output tile waits for, overlaps a main loop; segment
+// 1 of any other tile comes right after its segment 0.
+struct SegOrder {
+    bool prev_defer = false;
+    // Calls emit(seg, which) for the next tile in order, where which = 0 names
+    // this tile and 1 the pending previous deferred tile.
+    template <class F>
+    __device__ __forceinline__ void tile(bool defer, F &&emit)
+    {
+        if (prev_defer && defer) emit(1, 1);
+        emit(0, 0);
+        if (prev_defer && !defer) emit(1, 1);
+        if (!defer) emit(1, 0);
+        prev_defer = defer;
+    }
+    template <class F>
+    __device__ __forceinline__ void finish(F &&emit)
+    {
+        if (prev_defer) emit(1, 1);
+        prev_defer = false;
+    }
+};
+
 // ---------------------------------------------------------------- fused bottleneck
 // The mixing matrix as the B operand of the second product: this CTA's half of
-// its rows n (output columns of b or da), n in [rank r/2, (rank + 1) r/2), all
-// K = r, as bf16 high and low parts (x = x_hi + x_lo), K-major with the
+// its rows n (output columns of b or da), n in [rank R/2, (rank + 1) R/2), all
+// K = R, as bf16 high and low parts (x = x_hi + x_lo), K-major with the
 // 128-byte swizzle in k-blocks of 64.  Forward B[n][k] = M[k][n]
 // (b_j = sum_i a_i M[i][j]); backward B[n][k] = M[n][k] (da_i = sum_j db_j M[i][j]).
 // Epilogue thread et (0..255) converts the groups gi = et + 256 it of eight
 // consecutive k of one row n.
-template <int FUSE>
-__device__ __forceinline__ void mix_load(const FuseArgs &fa, uint32_t rank, int et, float (&mr)[4][8])
+template <int R>
+struct Mix {
+    static constexpr int kHr = R / 2;
+    static constexpr int kGroups = kHr * (R / 8);
+    static constexpr int kIters = (kGroups + 255) / 256;
+    static constexpr uint32_t kPartBytes = (uint32_t)(R / 64) * kHr * 128u;  // one of hi / lo
+};
+
+template <int R, int FUSE>
+__device__ __forceinline__ void mix_load(const FuseArgs &fa, uint32_t rank, int et, float (&mr)[Mix<R>::kIters][8])
 {
-    const int r = fa.r, hr = r / 2, ngroups = hr * (r / 8);
+    using X = Mix<R>;
 #pragma unroll
-    for (int it = 0; it < 4; ++it) {
+    for (int it = 0; it < X::kIters; ++it) {
         const int gi = et + 256 * it;
-        if (gi >= ngroups) continue;
-        const int n = (int)rank * hr + gi % hr, k = 8 * (gi / hr);
+        if (gi >= X::kGroups) continue;
+        const int n = (int)rank * X::kHr + gi % X::kHr, k = 8 * (gi / X::kHr);
         if constexpr (FUSE == kFuseBwd) {
-            const float4 *src = reinterpret_cast<const float4 *>(fa.M + (int64_t)n * r + k);
+            const float4 *src = reinterpret_cast<const float4 *>(fa.M + (int64_t)n * R + k);
             const float4 u = __ldg(src), w = __ldg(src + 1);
             mr[it][0] = u.x, mr[it][1] = u.y, mr[it][2] = u.z, mr[it][3] = u.w;
             mr[it][4] = w.x, mr[it][5] = w.y, mr[it][6] = w.z, mr[it][7] = w.w;
         } else {
 #pragma unroll
-            for (int q = 0; q < 8; ++q) mr[it][q] = __ldg(fa.M + (int64_t)(k + q) * r + n);
+            for (int q = 0; q < 8; ++q) mr[it][q] = __ldg(fa.M + (int64_t)(k + q) * R + n);
         }
-    }
-}
-
-__device__ __forceinline__ uint32_t mix_part_bytes(int r) { return (uint32_t)(r / 64) * (uint32_t)(r / 2) * 128u; }
-
-__device__ __forceinline__ void mix_store(int r, uint8_t *dst, int et, const float (&mr)[4][8])
-{
-    const int hr = r / 2, ngroups = hr * (r / 8);
-    const uint32_t part = mix_part_bytes(r);
-#pragma unroll
-    for (int it = 0; it < 4; ++it) {
-        const int gi = et + 256 * it;
-        if (gi >= ngroups) continue;
-        const int nl = gi % hr, k = 8 * (gi / hr);
-        uint4 hi, lo;
-        uint32_t *ph = &hi.x, *pl = &lo.x;
-#pragma unroll
-        for (int q = 0; q < 4; ++q) {
-            const __nv_bfloat162 h2 = __floats2bfloat162_rn(mr[it][2 * q], mr[it][2 * q + 1]);
-            const float2 hf = __bfloat1622float2(h2);
-            const __nv_bfloat162 l2 = __floats2bfloat162_rn(mr[it][2 * q] - hf.x, mr[it][2 * q + 1] - hf.y);
-            ph[q] = *reinterpret_cast<const uint32_t *>(&h2);
-            pl[q] = *reinterpret_cast<const uint32_t *>(&l2);
-        }
-        const uint32_t off = (uint32_t)(k / 64) * hr * 128u + (uint32_t)nl * 128u +
-                             ((((uint32_t)(k % 64) >> 3) ^ ((uint32_t)nl & 7u)) << 4);
-        *reinterpret_cast<uint4 *>(dst + off) = hi;
-        *reinterpret_cast<uint4 *>(dst + part + off) = lo;
     }
 }
 
@@ -317,33 +343,86 @@ __device__ __forceinline__ void split_hi_lo(float x0, float x1, uint32_t &hi, ui
     lo = *reinterpret_cast<const uint32_t *>(&l2);
 }
 
-// Epilogue of a bottleneck tile (see the header), run by all eight epilogue
-// warps of a CTA on its 128 rows; `acc` is the tile's TMEM accumulator.  A
-// thread owns one row and the 32-column chunks c = 32 half + 64 i < r.
-// Returns false, uniformly over the eight warps, after a timed-out wait.
-template <int FUSE>
-__device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *stg, uint32_t acc, int warp, int lane, int64_t m0,
-                                    uint32_t rank, uint32_t a_ready_leader, uint32_t b_full, uint32_t parity,
-                                    uint32_t *status)
+template <int R>
+__device__ __forceinline__ void mix_store(uint8_t *dst, int et, const float (&mr)[Mix<R>::kIters][8])
 {
-    const int r = fa.r;
+    using X = Mix<R>;
+#pragma unroll
+    for (int it = 0; it < X::kIters; ++it) {
+        const int gi = et + 256 * it;
+        if (gi >= X::kGroups) continue;
+        const int nl = gi % X::kHr, k = 8 * (gi / X::kHr);
+        uint4 hi, lo;
+        split_hi_lo(mr[it][0], mr[it][1], hi.x, lo.x);
+        split_hi_lo(mr[it][2], mr[it][3], hi.y, lo.y);
+        split_hi_lo(mr[it][4], mr[it][5], hi.z, lo.z);
+        split_hi_lo(mr[it][6], mr[it][7], hi.w, lo.w);
+        const uint32_t off = (uint32_t)(k / 64) * X::kHr * 128u + (uint32_t)nl * 128u +
+                             ((((uint32_t)(k % 64) >> 3) ^ ((uint32_t)nl & 7u)) << 4);
+        *reinterpret_cast<uint4 *>(dst + off) = hi;
+        *reinterpret_cast<uint4 *>(dst + X::kPartBytes + off) = lo;
+    }
+}
+
+// Column sums of one A stage (128 rows x 64 bf16 columns, K-major, 128-byte
+// swizzle): epilogue warp ew (0..7) takes columns [8 ew, 8 ew + 8); lane l
+// adds rows 4l .. 4l + 3 in order, then the lanes are combined by a fixed
+// xor butterfly.  Every lane returns the eight sums.
+__device__ __forceinline__ void stage_colsum8(const uint8_t *sA, int ew, int lane, float (&s)[8])
+{
+#pragma unroll
+    for (int i = 0; i < 8; ++i) s[i] = 0.f;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int row = 4 * lane + q;
+        const uint4 u = *reinterpret_cast<const uint4 *>(sA + row * 128 + (((uint32_t)ew ^ (uint32_t)(row & 7)) << 4));
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[i]));
+            s[2 * i] += f.x;
+            s[2 * i + 1] += f.y;
+        }
+    }
+#pragma unroll
+    for (int m = 16; m >= 1; m >>= 1)
+#pragma unroll
+        for (int i = 0; i < 8; ++i) s[i] += __shfl_xor_sync(0xffffffffu, s[i], m);
+}
+
+// Bottleneck epilogue of a leader tile (see the header), run by all eight
+// epilogue warps of a CTA on its 128 rows.  `acc` is the tile's TMEM
+// accumulator after segment 0: columns [0, R) hold the output columns
+// [0, R) so far, [R, 2R) the branch pre-activation (h or dc).  A thread owns
+// one row and the 32-column chunks c = 32 half + 64 i < R.  On return the
+// output columns are back in [0, R) and c (or dh, a, db and the column sums)
+// are stored.  Returns false, uniformly over the eight warps, after a
+// timed-out wait.
+template <int R, int FUSE>
+__device__ __noinline__ bool leader_epilogue(const FuseArgs &fa, uint8_t *stg, uint32_t acc, int warp, int lane,
+                                             int64_t m0, uint32_t rank, uint32_t a_ready_leader, uint32_t b_full,
+                                             uint32_t parity, uint32_t *status)
+{
+    constexpr int NC = R / 64;  // 32-column chunks per thread
     const int quarter = warp % 4, half = (warp - 2) / 4;
     const int64_t t0 = m0 + quarter * 32;  // the warp's first row
     const bool live = t0 + lane < fa.T;
     const uint32_t lane_addr = acc + ((uint32_t)(quarter * 32) << 16);
     const int et = (warp - 2) * 32 + lane;
-    float *part = FUSE == kFuseBwd ? fa.part + (t0 / 32) * 4 * (int64_t)r : nullptr;
-    // ---- phase 1: first accumulator (h or dc).  The row operand of the
-    // second product (a or db) replaces each 32-column chunk it came from:
-    // bf16 high parts of its 32 values in the chunk's first 16 columns, low
-    // parts in the last 16 (two values per 32-bit column, lower k in the low
-    // half), so each warp overwrites only columns it has read itself.
+    float *part = FUSE == kFuseBwd ? fa.part + (t0 / 32) * 4 * (int64_t)R : nullptr;
+    // ---- park the output columns: the second product writes b (da) there
+    float park[NC][32];
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < NC; ++i) ptx::tmem_ld_32x32b_x32(lane_addr + 32 * half + 64 * i, park[i]);
+    // ---- phase 1: h or dc -> the row operand of the second product (a or
+    // db), bf16 high parts of a chunk's 32 values in its first 16 columns and
+    // low parts in the last 16 (two values per 32-bit column, lower k in the
+    // low half), each warp overwriting only columns it has read itself
+#pragma unroll
+    for (int i = 0; i < NC; ++i) {
         const int c = 32 * half + 64 * i;
-        if (c >= r) continue;
         float v[32];
-        ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
+        ptx::tmem_ld_32x32b_x32(lane_addr + R + c, v);
         uint32_t ohi[16], olo[16];
         if constexpr (FUSE == kFuseFwd) {
             if (fa.h_out) {
@@ -352,7 +431,7 @@ __device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *st
                 for (int g = 0; g < 8; ++g)
 #pragma unroll
                     for (int q = 0; q < 4; ++q) w[g][q] = __float_as_uint(v[4 * g + q]);
-                store_segments<8>(w, fa.h_out + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+                store_segments<8>(w, fa.h_out + t0 * R + c, (int64_t)R * 4, t0, fa.T);
             }
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
@@ -367,7 +446,7 @@ __device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *st
             float bv[32];
             {
                 uint32_t w[8][4];
-                load_segments<8>(w, fa.b_in + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+                load_segments<8>(w, fa.b_in + t0 * R + c, (int64_t)R * 4, t0, fa.T);
 #pragma unroll
                 for (int g = 0; g < 8; ++g)
 #pragma unroll
@@ -385,30 +464,30 @@ __device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *st
                 split_hi_lo(w0 * d0, w1 * d1, ohi[e], olo[e]);
                 wdb[e / 4][e % 4] = ohi[e];
             }
-            store_segments<4>(wdb, fa.db_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
+            store_segments<4>(wdb, fa.db_out + t0 * R + c, (int64_t)R * 2, t0, fa.T);
 #pragma unroll
             for (int e = 0; e < 32; ++e) bv[e] *= v[e];  // du2 b
             const float s2 = warp_colsum32(bv);
             const float s3 = warp_colsum32(v);
             if (t0 < fa.T) {
-                part[2 * r + c + lane] = s2;
-                part[3 * r + c + lane] = s3;
+                part[2 * R + c + lane] = s2;
+                part[3 * R + c + lane] = s3;
             }
         }
-        ptx::tmem_st_32x32b_x16(lane_addr + c, ohi);
-        ptx::tmem_st_32x32b_x16(lane_addr + c + 16, olo);
+        ptx::tmem_st_32x32b_x16(lane_addr + R + c, ohi);
+        ptx::tmem_st_32x32b_x16(lane_addr + R + c + 16, olo);
     }
     // ---- the mixing matrix goes into the staging buffer once every warp's
     // TMA stores have left it
     {
-        float mr[4][8];
-        mix_load<FUSE>(fa, rank, et, mr);
+        float mr[Mix<R>::kIters][8];
+        mix_load<R, FUSE>(fa, rank, et, mr);
         if (lane == 0) ptx::bulk_wait_read_all();
         __syncwarp();
         ptx::tc_fence_before();
         ptx::named_barrier_sync(1, 256);
         ptx::tc_fence_after();
-        mix_store(r, stg, et, mr);
+        mix_store<R>(stg, et, mr);
     }
     ptx::fence_proxy_async_smem_cluster();  // generic writes, read by the leader's MMA (async proxy)
     ptx::tc_fence_before();
@@ -418,13 +497,12 @@ __device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *st
     ok = ptx::named_barrier_and(1, 256, __all_sync(0xffffffffu, ok));
     if (!ok) return false;
     ptx::tc_fence_after();
-    // ---- phase 2: second accumulator (b or da)
+    // ---- phase 2: b or da in columns [0, R); then the parked columns go back
 #pragma unroll
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < NC; ++i) {
         const int c = 32 * half + 64 * i;
-        if (c >= r) continue;
         float v[32];
-        ptx::tmem_ld_32x32b_x32(lane_addr + kR2Col + c, v);
+        ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
         if constexpr (FUSE == kFuseFwd) {
             // v = b: c = cos(omega2 b + phi2)
             uint32_t wc[4][4];
@@ -441,21 +519,20 @@ __device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *st
                 for (int g = 0; g < 8; ++g)
 #pragma unroll
                     for (int q = 0; q < 4; ++q) w[g][q] = __float_as_uint(v[4 * g + q]);
-                store_segments<8>(w, fa.b_out + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+                store_segments<8>(w, fa.b_out + t0 * R + c, (int64_t)R * 4, t0, fa.T);
             }
-            store_segments<4>(wc, fa.c_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
+            store_segments<4>(wc, fa.c_out + t0 * R + c, (int64_t)R * 2, t0, fa.T);
         } else {
             // v = da; with h of this row: du1 = -sin(u1) da, dh = omega1 du1, a = cos(u1)
             float hv[32];
             {
                 uint32_t w[8][4];
-                load_segments<8>(w, fa.h_in + t0 * r + c, (int64_t)r * 4, t0, fa.T);
+                load_segments<8>(w, fa.h_in + t0 * R + c, (int64_t)R * 4, t0, fa.T);
 #pragma unroll
                 for (int g = 0; g < 8; ++g)
 #pragma unroll
                     for (int q = 0; q < 4; ++q) hv[4 * g + q] = __uint_as_float(w[g][q]);
             }
-            // du1 kept in v
             uint32_t wdh[4][4], wa[4][4];
 #pragma unroll
             for (int e = 0; e < 16; ++e) {
@@ -474,20 +551,162 @@ __device__ __noinline__ bool bottleneck_epilogue(const FuseArgs &fa, uint8_t *st
                 wdh[e / 4][e % 4] = ptx::pack_bf16x2(dh2[0], dh2[1]);
                 wa[e / 4][e % 4] = ptx::pack_bf16x2(av2[0], av2[1]);
             }
-            store_segments<4>(wdh, fa.dh_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
-            store_segments<4>(wa, fa.a_out + t0 * r + c, (int64_t)r * 2, t0, fa.T);
+            store_segments<4>(wdh, fa.dh_out + t0 * R + c, (int64_t)R * 2, t0, fa.T);
+            store_segments<4>(wa, fa.a_out + t0 * R + c, (int64_t)R * 2, t0, fa.T);
 #pragma unroll
             for (int e = 0; e < 32; ++e) hv[e] *= v[e];  // du1 h
             const float s0 = warp_colsum32(hv);
             const float s1 = warp_colsum32(v);
             if (t0 < fa.T) {
                 part[c + lane] = s0;
-                part[r + c + lane] = s1;
+                part[R + c + lane] = s1;
             }
         }
+        ptx::tmem_st_32x32b_x32(lane_addr + c, park[i]);
     }
     return true;
 }
+
+// MMA issuer of a fused launch (one thread of the leader CTA).  The k-block
+// loop matches the default one: two ring stages per wait, their eight MMAs
+// back to back.  Every wait is the suspending try_wait, bounded, and issues
+// the pending second product of the last leader as soon as its epilogue has
+// the row operand ready.
+template <int STAGES, bool B_MN, bool MN4, int FUSE, class EpiParams>
+struct FusedIssuer {
+    const GroupArgs<EpiParams> &g;
+    const FuseArgs &fa;
+    uint32_t tmem, sbase, kA, kStage, kStgOff, bar0;
+    uint32_t *status;
+    int s = 0;
+    uint32_t ph = 0;
+    bool ok = true;
+    bool m2_pending = false;
+    uint32_t m2_acc = 0, m2_parity = 0, nlead = 0;
+
+    __device__ __forceinline__ uint32_t full_bar(int i) const { return bar0 + 8u * i; }
+    __device__ __forceinline__ uint32_t empty_bar(int i) const { return bar0 + 8u * (STAGES + i); }
+    __device__ __forceinline__ uint32_t tfull_bar(int b) const { return bar0 + 8u * (2 * STAGES + b); }
+    __device__ __forceinline__ uint32_t a_ready() const { return bar0 + 8u * (2 * STAGES + 5); }
+    __device__ __forceinline__ uint32_t b_full() const { return bar0 + 8u * (2 * STAGES + 6); }
+    __device__ __forceinline__ uint32_t consumed_bar(int i) const { return bar0 + 8u * (2 * STAGES + 8 + i); }
+
+    // b | da (columns [0, r)) = (a | db in TMEM columns [r, 2r): per 32-column
+    // chunk 16 columns of bf16 high parts, then 16 of low parts) x (matrix
+    // hi/lo in the staging buffers of both CTAs), as hi*hi + lo*hi + hi*lo
+    __device__ __forceinline__ void second_product()
+    {
+        ptx::tc_fence_after();
+        const int r = fa.r;
+        const uint32_t idesc2 = ptx::idesc_bf16(2 * kBM, r, false, false);
+        const uint32_t mhi = sbase + kStgOff, mlo = mhi + (uint32_t)(r / 64) * (uint32_t)(r / 2) * 128u;
+#pragma unroll 1
+        for (int kk = 0; kk < r / 16; ++kk) {
+            const uint32_t off = (uint32_t)(kk / 4) * (uint32_t)(r / 2) * 128u + (uint32_t)(kk % 4) * 32u;
+            const uint64_t dmh = ptx::smem_desc_sw128(mhi + off, 16, 1024);
+            const uint64_t dml = ptx::smem_desc_sw128(mlo + off, 16, 1024);
+            const uint32_t ahi = m2_acc + (uint32_t)r + (uint32_t)(kk / 2) * 32u + (uint32_t)(kk % 2) * 8u;
+            const uint32_t alo = ahi + 16u;
+            mma2_bf16_ta(m2_acc, ahi, dmh, idesc2, kk > 0 ? 1u : 0u);
+            mma2_bf16_ta(m2_acc, alo, dmh, idesc2, 1u);
+            mma2_bf16_ta(m2_acc, ahi, dml, idesc2, 1u);
+        }
+        mma2_commit_mc(b_full(), 0x3);
+        m2_pending = false;
+    }
+
+    __device__ __forceinline__ bool wait(uint32_t bar, uint32_t parity)
+    {
+        if (m2_pending && ptx::mbar_test_wait(a_ready(), m2_parity)) second_product();
+        if (ptx::mbar_try_wait(bar, parity)) return true;
+        const uint64_t t0 = ptx::globaltimer_ns();
+        while (true) {
+#pragma unroll 1
+            for (int i = 0; i < 64; ++i) {
+                if (m2_pending && ptx::mbar_test_wait(a_ready(), m2_parity)) second_product();
+                if (ptx::mbar_try_wait(bar, parity)) return true;
+            }
+            if (ptx::globaltimer_ns() - t0 > ptx::kWaitLimitNs) {
+                raise_status(status, kStatusTimeout);
+                ok = false;
+                return false;
+            }
+        }
+    }
+
+    // a leader's segment 0 is issued: its epilogue starts, its second product is pending
+    __device__ __forceinline__ void lead_issued(int buf, uint32_t xfull)
+    {
+        mma2_commit_mc(xfull, 0x3);
+        m2_pending = true;
+        m2_acc = tmem + (uint32_t)buf * 256u;
+        m2_parity = nlead & 1;
+        ++nlead;
+    }
+
+    // the k-blocks of segment sg of tile tr into accumulator buffer buf
+    __device__ __forceinline__ void seg(const PairTile &tr, int sg, int buf)
+    {
+        if (!ok) return;
+        const auto &P = g.p[tr.prob];
+        const bool bias_stage = FUSE == kFuseBwd && tr.prob == 0 && sg == 0 && fa.bias_part != nullptr;
+        const uint32_t d_tmem = tmem + (uint32_t)buf * 256u;
+        const uint32_t idesc = ptx::idesc_bf16(2 * kBM, P.bn, false, B_MN);
+        const uint32_t nchB = (uint32_t)P.bn / 128;  // 64-wide B chunks held per CTA
+        const uint64_t a0 = ptx::smem_desc_sw128(sbase, 16, 1024);
+        const uint64_t b0 = B_MN ? (MN4 ? ptx::smem_desc_sw128(sbase + kA, 1024, 1024 * nchB)
+                                        : ptx::smem_desc_sw128(sbase + kA, kChunkBytes, 1024))
+                                 : ptx::smem_desc_sw128(sbase + kA, 16, 1024);
+        const uint32_t stepB = B_MN ? (MN4 ? 128u * nchB : 2048u / 16) : 32u / 16;
+        const uint32_t kStageUnits = kStage / 16;
+        const int nkb = sg ? P.kb1 : P.kb0;
+        const uint32_t acc0 = sg ? 1u : 0u;
+        for (int i = 0; i < nkb; i += 2) {
+            const bool two = i + 1 < nkb;
+            int s2 = s + 1;
+            uint32_t ph2 = ph;
+            if (s2 == STAGES) {
+                s2 = 0;
+                ph2 ^= 1;
+            }
+            // the stages are usually full already: look for the epilogue's
+            // signal here too, not only while waiting
+            if (m2_pending && ptx::mbar_test_wait(a_ready(), m2_parity)) second_product();
+            if (!wait(full_bar(s), ph) || (two && !wait(full_bar(s2), ph2))) return;
+            const uint64_t so = (uint64_t)((uint32_t)s * kStageUnits);
+            const uint64_t ad = a0 + so, bd = b0 + so;
+            mma2_bf16(d_tmem, ad, bd, idesc, (i > 0 ? 1u : acc0));
+#pragma unroll
+            for (int kk = 1; kk < kBK / 16; ++kk) mma2_bf16(d_tmem, ad + kk * 2u, bd + kk * stepB, idesc, 1u);
+            mma2_commit_mc(empty_bar(s), 0x3);
+            if (bias_stage) mma2_commit_mc(consumed_bar(s), 0x3);
+            if (two) {
+                const uint64_t so2 = (uint64_t)((uint32_t)s2 * kStageUnits);
+                const uint64_t ad2 = a0 + so2, bd2 = b0 + so2;
+#pragma unroll
+                for (int kk = 0; kk < kBK / 16; ++kk) mma2_bf16(d_tmem, ad2 + kk * 2u, bd2 + kk * stepB, idesc, 1u);
+                mma2_commit_mc(empty_bar(s2), 0x3);
+                if (bias_stage) mma2_commit_mc(consumed_bar(s2), 0x3);
+                s = s2 + 1;
+                ph = ph2;
+                if (s == STAGES) {
+                    s = 0;
+                    ph ^= 1;
+                }
+            } else {
+                s = s2;
+                ph = ph2;
+            }
+        }
+    }
+
+    // segment 1 of tile tr, which completes its accumulator
+    __device__ __forceinline__ void finish_seg(const PairTile &tr, int buf)
+    {
+        seg(tr, 1, buf);
+        if (ok) mma2_commit_mc(tfull_bar(buf), 0x3);
+    }
+};
 
 template <int STAGES>
 struct PairSmem {
@@ -497,8 +716,9 @@ struct PairSmem {
     static constexpr uint32_t kStgOff = STAGES * kStage;  // epilogue staging, 4 KB per epilogue warp
     static constexpr uint32_t kStgBytes = 8 * 4096;
     static constexpr uint32_t kBarOff = kStgOff + kStgBytes;
-    static constexpr uint32_t kNumBars = 2 * STAGES + 7;  // full, empty, tfull[2], tempty[2], mma_done,
-                                                          // a_ready, b_full (fused bottleneck)
+    // full, empty, tfull[2], tempty[2], mma_done; fused bottleneck: a_ready,
+    // b_full, xfull, consumed[STAGES]
+    static constexpr uint32_t kNumBars = 3 * STAGES + 8;
     static constexpr uint32_t kBytes = kBarOff + 8 * kNumBars + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
@@ -508,8 +728,8 @@ struct PairSmem {
 //   [8-row K group][64-wide MN chunk][8 rows][128 B]
 // (chunk stride 1 KB, group stride nchunks KB) instead of two or more 2-D
 // boxes giving [MN chunk][64 K rows][128 B] (chunk stride 8 KB, group 1 KB).
-// FUSE: kFuseNone, or a fused bottleneck launch (problem 0 bottleneck tiles
-// of N = r <= 128 with bn = 128, problem 1 output tiles, see the header).
+// FUSE: kFuseNone, or a fused bottleneck launch (problem 0 leader tiles of
+// N = 2r, problem 1 the other output tiles, see the header; A K-major).
 template <bool A_MN, bool B_MN, int STAGES, class Epi, bool MN4 = false, int FUSE = kFuseNone>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupArgs<typename Epi::Params> g,
@@ -531,7 +751,9 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
     const uint32_t mma_done = bar0 + 8u * (2 * STAGES + 4);
     const uint32_t a_ready = bar0 + 8u * (2 * STAGES + 5);  // fused: row operand in TMEM, matrix in smem
     const uint32_t b_full = bar0 + 8u * (2 * STAGES + 6);   // fused: second product complete
-    auto tile_of = [&](int slot) { return FUSE != kFuseNone ? fused_tile(g, slot) : slot_tile(g, slot); };
+    const uint32_t xfull = bar0 + 8u * (2 * STAGES + 7);    // fused: a leader's segment 0 complete
+    // fused backward: the MMAs of a leader stage are done (its dy rows are summed for dbias)
+    auto consumed_bar = [&](int s) { return bar0 + 8u * (2 * STAGES + 8 + s); };
     uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(smem + S::kBarOff + 8 * S::kNumBars);
 
     const int warp = threadIdx.x / 32, lane = threadIdx.x % 32;
@@ -544,10 +766,18 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         for (int p = 0; p < g.nproblems; ++p) {
             ptx::tma_prefetch_desc(&maps.m[p][0]);
             ptx::tma_prefetch_desc(&maps.m[p][1]);
+            if (FUSE != kFuseNone) {
+                ptx::tma_prefetch_desc(&maps.m[p][2]);
+                ptx::tma_prefetch_desc(&maps.m[p][3]);
+            }
         }
+        if (FUSE != kFuseNone) ptx::tma_prefetch_desc(&maps.m[0][5]);
         for (int s = 0; s < STAGES; ++s) {
             ptx::mbar_init(full_bar(s), 1);
-            ptx::mbar_init(empty_bar(s), 1);
+            // fused backward: the MMA commit and eight arrivals, from the
+            // epilogue warps after summing a leader stage, else from the producer
+            ptx::mbar_init(empty_bar(s), FUSE == kFuseBwd ? 9 : 1);
+            ptx::mbar_init(consumed_bar(s), 1);
         }
         for (int b = 0; b < 2; ++b) {
             ptx::mbar_init(tfull_bar(b), 1);
@@ -556,6 +786,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         ptx::mbar_init(mma_done, 1);
         ptx::mbar_init(a_ready, 16);  // 8 epilogue warps in each CTA of the pair
         ptx::mbar_init(b_full, 1);
+        ptx::mbar_init(xfull, 1);
         ptx::fence_barrier_init();
     }
     if (warp == 1) {
@@ -568,7 +799,230 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
     ptx::tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
+    if constexpr (FUSE != kFuseNone) {
+        // ======================= fused bottleneck launch (see the header)
+        const int nslots = g.total_tiles;
+        if (warp == 0) {
+            if (lane == 0) {
+                // ---------------- producer (both CTAs)
+                uint32_t it = 0;
+                bool ok = true;
+                SegOrder order;
+                PairTile prev{};
+                bool first = true;
+                // the k-blocks of segment sg of tile tr into the ring
+                auto load_seg = [&](const PairTile &tr, int sg) -> bool {
+                    const auto &P = g.p[tr.prob];
+                    const bool lead = tr.prob == 0;
+                    const int bh = P.bn / 2;  // B columns held by this CTA
+                    const int kb_begin = sg ? P.kb0 : 0, kb_end = sg ? P.kb0 + P.kb1 : P.kb0;
+                    // the second segment reads c (dh) of this CTA's 128 rows,
+                    // stored by the leader of its row pair
+                    if (sg == 1 && kb_end > kb_begin && !ptx::flag_wait(fa.flags + tr.m0 / kBM, g.status))
+                        return false;
+                    const bool bias_stage = FUSE == kFuseBwd && lead && sg == 0 && fa.bias_part != nullptr;
+                    const uint32_t b_bytes = (uint32_t)bh * kBK * 2;
+                    // a leader's second segment: rank 1 holds no B (its half of
+                    // the accumulator columns is not read again)
+                    const bool load_b = !(lead && sg == 1 && rank == 1);
+                    const uint32_t tx = 2 * S::kA + (lead && sg == 1 ? b_bytes : 2 * b_bytes);
+                    const CUtensorMap *mA = &maps.m[tr.prob][sg ? 2 : 0];
+                    const CUtensorMap *mB =
+                        lead && sg == 0 && rank == 1 ? &maps.m[tr.prob][5] : &maps.m[tr.prob][sg ? 3 : 1];
+                    const int nb = lead ? 0 : (int)tr.n0 + (int)rank * bh;
+                    for (int kb = kb_begin; kb < kb_end; ++kb, ++it) {
+                        const int s = it % STAGES;
+                        const uint32_t ph = (it / STAGES) & 1;
+                        if (!ptx::mbar_wait(empty_bar(s), ph ^ 1, g.status)) return false;
+                        if constexpr (FUSE == kFuseBwd)
+                            if (!bias_stage) ptx::mbar_arrive_cnt(empty_bar(s), 8);
+                        const uint32_t fb = map_to_rank(full_bar(s), 0);
+                        if (leader) ptx::mbar_arrive_expect_tx(full_bar(s), tx);
+                        const uint32_t sA = sbase + s * S::kStage, sB = sA + S::kA;
+                        const int k = (kb - kb_begin) * kBK;
+                        tma_load_2d_pair(sA, mA, fb, k, (int)tr.m0);
+                        if (load_b) {
+                            if (B_MN && MN4) {
+                                tma_load_4d_pair(sB, mB, fb, nb / 64, k / 8);
+                            } else if (B_MN) {
+                                for (int c = 0; c < bh / 64; ++c)
+                                    tma_load_2d_pair(sB + c * kChunkBytes, mB, fb, nb + 64 * c, k);
+                            } else {
+                                tma_load_2d_pair(sB, mB, fb, k, nb);
+                            }
+                        }
+                    }
+                    return true;
+                };
+                for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
+                    const int t = share_tile(g, slot, nclusters);
+                    if (t < 0) continue;
+                    const PairTile tr = locate_pair(g, t, rank);
+                    const bool defer = tr.prob == 0 || first;
+                    first = false;
+                    order.tile(defer, [&](int sg, int which) {
+                        if (ok) ok = load_seg(which ? prev : tr, sg);
+                    });
+                    if (defer) prev = tr;
+                }
+                order.finish([&](int sg, int) {
+                    if (ok) ok = load_seg(prev, sg);
+                });
+                // the leader's ring barriers also count the peer's bytes: once
+                // they complete, no copy of either CTA is still landing
+                if (leader) {
+                    const uint32_t first = it > (uint32_t)STAGES ? it - STAGES : 0;
+                    for (uint32_t i = first; i < it; ++i)
+                        ptx::mbar_wait(full_bar(i % STAGES), (i / STAGES) & 1, nullptr);
+                }
+            }
+        } else if (warp == 1) {
+            if (lane == 0 && leader) {
+                // ---------------- MMA issuer (leader CTA only)
+                FusedIssuer<STAGES, B_MN, MN4, FUSE, typename Epi::Params> is{
+                    g, fa, tmem, sbase, S::kA, S::kStage, S::kStgOff, bar0, g.status};
+                int j = 0;
+                bool prev_defer = false;
+                PairTile prev{};
+                int prev_buf = 0;
+                for (int slot = cluster; is.ok; slot += nclusters) {
+                    if (slot >= nslots) {
+                        if (prev_defer) is.finish_seg(prev, prev_buf);
+                        break;
+                    }
+                    const int t = share_tile(g, slot, nclusters);
+                    if (t < 0) continue;
+                    const PairTile tr = locate_pair(g, t, 0);
+                    const bool lead = tr.prob == 0;
+                    const bool defer = lead || j == 0;
+                    const int b = j & 1;
+                    const uint32_t use = (uint32_t)(j >> 1);
+                    if (prev_defer && defer) is.finish_seg(prev, prev_buf);
+                    if (!is.wait(tempty_bar(b), (use & 1) ^ 1)) break;
+                    ptx::tc_fence_after();
+                    is.seg(tr, 0, b);
+                    if (is.ok && lead) is.lead_issued(b, xfull);
+                    if (!defer) {
+                        if (prev_defer) is.finish_seg(prev, prev_buf);
+                        is.finish_seg(tr, b);
+                    }
+                    if (defer) {
+                        prev = tr;
+                        prev_buf = b;
+                    }
+                    prev_defer = defer;
+                    ++j;
+                }
+                mma2_commit_mc(mma_done, 0x1);
+                ptx::mbar_wait(mma_done, 0, nullptr);
+            }
+        } else {
+            // ---------------- epilogue (both CTAs): own 128 accumulator rows
+            const int quarter = warp % 4;
+            const int half = (warp - 2) / 4;  // two warps per TMEM lane quarter split the columns
+            const uint32_t leader_tempty0 = map_to_rank(tempty_bar(0), 0);
+            const uint32_t leader_tempty1 = map_to_rank(tempty_bar(1), 0);
+            const uint32_t leader_a_ready = map_to_rank(a_ready, 0);
+            const uint32_t stg = sbase + S::kStgOff + (uint32_t)(warp - 2) * 4096u;
+            uint8_t *stg_ptr = smem + S::kStgOff + (warp - 2) * 4096;
+            int j = 0;
+            uint32_t nlead = 0;
+            uint32_t it = 0;    // ring position, replaying the issue order
+            uint32_t cons = 0;  // per stage: parity of the next consumed_bar phase
+            int prev_kb1 = 0;
+            SegOrder order;
+            for (int slot = cluster; slot < nslots; slot += nclusters) {
+                const int t = share_tile(g, slot, nclusters);
+                if (t < 0) continue;
+                const PairTile tr = locate_pair(g, t, rank);
+                const auto &P = g.p[tr.prob];
+                const bool lead = tr.prob == 0;
+                const int b = j & 1;
+                const uint32_t use = (uint32_t)(j >> 1);
+                uint32_t it_x = 0;
+                order.tile(lead || j == 0, [&](int sg, int which) {
+                    if (which) {
+                        it += prev_kb1;
+                    } else if (sg == 0) {
+                        it_x = it;
+                        it += P.kb0;
+                    } else {
+                        it += P.kb1;
+                    }
+                });
+                if (lead || j == 0) prev_kb1 = P.kb1;
+                bool ok = true;
+                if (lead) {
+                    if constexpr (FUSE == kFuseBwd) {
+                        if (fa.bias_part) {
+                            // dbias partials: the column sums of this CTA's dy rows,
+                            // stage by stage once the MMAs have read it
+                            const int ew = warp - 2;
+                            for (int i = 0; i < P.kb0; ++i) {
+                                const int s = (int)((it_x + i) % STAGES);
+                                const uint32_t par = (cons >> s) & 1u;
+                                cons ^= 1u << s;
+                                ok = __all_sync(0xffffffffu, ptx::mbar_wait(consumed_bar(s), par, g.status));
+                                if (!ok) break;
+                                float cs[8];
+                                stage_colsum8(smem + s * S::kStage, ew, lane, cs);
+                                // the stage is refilled by the copy engine (async
+                                // proxy) once released: order these reads before that
+                                ptx::fence_proxy_async_smem();
+                                __syncwarp();
+                                if (lane == 0) ptx::mbar_arrive(empty_bar(s));
+                                float v = cs[0];
+#pragma unroll
+                                for (int q = 1; q < 8; ++q)
+                                    if (lane == q) v = cs[q];
+                                const int64_t col = (int64_t)i * kBK + 8 * ew + lane;
+                                if (lane < 8 && tr.m0 < fa.T && col < fa.kdim)
+                                    fa.bias_part[(tr.m0 / kBM) * fa.kdim + col] = v;
+                            }
+                        }
+                    }
+                    ok = ok && ptx::mbar_wait(xfull, nlead & 1, g.status);
+                    ok = ptx::named_barrier_and(1, 256, __all_sync(0xffffffffu, ok));
+                    if (!ok) break;
+                    ptx::tc_fence_after();
+                    const uint32_t acc = tmem + b * kAccCols;
+                    ok = fa.r == 128 ? leader_epilogue<128, FUSE>(fa, smem + S::kStgOff, acc, warp, lane, tr.m0, rank,
+                                                                  leader_a_ready, b_full, nlead & 1, g.status)
+                                     : leader_epilogue<64, FUSE>(fa, smem + S::kStgOff, acc, warp, lane, tr.m0, rank,
+                                                                 leader_a_ready, b_full, nlead & 1, g.status);
+                    if (!ok) break;
+                    // publish this CTA's c (dh) rows and its restored accumulator:
+                    // the producers of this row block's second segments wait for it
+                    ptx::tc_fence_before();
+                    ptx::fence_proxy_async_global();
+                    ptx::named_barrier_sync(1, 256);
+                    if (warp == 2 && lane == 0) {
+                        __threadfence();
+                        ptx::fence_proxy_async_global();
+                        ptx::st_release_gpu(fa.flags + tr.m0 / kBM, 1u);
+                    }
+                    ++nlead;
+                }
+                ok = ptx::mbar_wait(tfull_bar(b), use & 1, g.status);
+                // named barriers above: leave together or not at all
+                ok = ptx::named_barrier_and(1, 256, __all_sync(0xffffffffu, ok));
+                if (!ok) break;
+                ptx::tc_fence_after();
+                const int bn_out = lead ? fa.r : P.bn;  // a leader stores its first r columns
+                if (P.ep.tma)
+                    Epi::run_tma(P.ep, &maps.m[tr.prob][4], stg_ptr, stg, tmem + b * kAccCols, bn_out, quarter, lane,
+                                 tr.m0, tr.n0, P.N, tr.z, half);
+                else
+                    Epi::run_dyn(P.ep, tmem + b * kAccCols, bn_out, quarter, lane, tr.m0, tr.n0, P.M, P.N, tr.z,
+                                 32 * half, 64);
+                ptx::tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive_cluster(b ? leader_tempty1 : leader_tempty0);
+                ++j;
+            }
+            if (lane == 0) ptx::bulk_wait_all();  // stores done before the staging buffer goes away
+        }
+    } else if (warp == 0) {
         if (lane == 0) {
             // ---------------- producer (both CTAs)
             uint32_t it = 0;
@@ -576,7 +1030,7 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             bool waited = false;  // for the predecessor grid (programmatic launch)
             const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
             for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
-                const int t = tile_of(slot);
+                const int t = slot_tile(g, slot);
                 if (t < 0) continue;
                 const PairTile tr = locate_pair(g, t, rank);
                 const auto &P = g.p[tr.prob];
@@ -588,14 +1042,6 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     if (!ptx::mbar_wait(empty_bar(s), ph ^ 1, g.status)) {
                         ok = false;
                         break;
-                    }
-                    if constexpr (FUSE != kFuseNone) {
-                        // the second segment of an output tile reads c (dh) of
-                        // this CTA's 128 rows, stored by a bottleneck tile
-                        if (tr.prob == 1 && kb == P.kb0 && !ptx::flag_wait(fa.flags + tr.m0 / kBM, g.status)) {
-                            ok = false;
-                            break;
-                        }
                     }
                     const bool seg1 = kb >= P.kb0;
                     if (!waited && (P.dep & (seg1 ? 2 : 1))) {
@@ -652,9 +1098,8 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
             constexpr uint32_t kStepA = A_MN ? (MN4 ? 4096 / 16 : 2048 / 16) : 32 / 16;
             constexpr uint32_t kStageUnits = S::kStage / 16;
             const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
-            uint32_t nc = 0;  // bottleneck tiles so far
             for (int slot = cluster; ok && slot < nslots; slot += nclusters) {
-                const int t = tile_of(slot);
+                const int t = slot_tile(g, slot);
                 if (t < 0) continue;
                 const PairTile tr = locate_pair(g, t, 0);
                 const auto &P = g.p[tr.prob];
@@ -713,33 +1158,6 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                     }
                 }
                 mma2_commit_mc(tfull_bar(b), 0x3);
-                if constexpr (FUSE != kFuseNone) {
-                    if (ok && tr.prob == 0) {
-                        // second product of the bottleneck tile: b | da (cols
-                        // kR2Col..) = (a | db in TMEM cols [0, r): per 32-column
-                        // chunk 16 columns of bf16 high parts, then 16 of low
-                        // parts) x (matrix hi/lo in the staging buffers of both
-                        // CTAs), as hi*hi + lo*hi + hi*lo
-                        if (!ptx::mbar_wait(a_ready, nc & 1, g.status)) break;
-                        ptx::tc_fence_after();
-                        const int r = fa.r;
-                        const uint32_t acc = tmem + b * kAccCols;
-                        const uint32_t idesc2 = ptx::idesc_bf16(2 * kBM, r, false, false);
-                        const uint32_t mhi = sbase + S::kStgOff, mlo = mhi + mix_part_bytes(r);
-                        for (int kk = 0; kk < r / 16; ++kk) {
-                            const uint32_t off = (uint32_t)(kk / 4) * (uint32_t)(r / 2) * 128u + (uint32_t)(kk % 4) * 32u;
-                            const uint64_t dmh = ptx::smem_desc_sw128(mhi + off, 16, 1024);
-                            const uint64_t dml = ptx::smem_desc_sw128(mlo + off, 16, 1024);
-                            const uint32_t ahi = acc + (uint32_t)(kk / 2) * 32u + (uint32_t)(kk % 2) * 8u;
-                            const uint32_t alo = ahi + 16u;
-                            mma2_bf16_ta(acc + kR2Col, ahi, dmh, idesc2, kk > 0 ? 1u : 0u);
-                            mma2_bf16_ta(acc + kR2Col, alo, dmh, idesc2, 1u);
-                            mma2_bf16_ta(acc + kR2Col, ahi, dml, idesc2, 1u);
-                        }
-                        mma2_commit_mc(b_full, 0x3);
-                        ++nc;
-                    }
-                }
                 ++j;
             }
             mma2_commit_mc(mma_done, 0x1);
@@ -754,43 +1172,18 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
         const uint32_t stg = sbase + S::kStgOff + (uint32_t)(warp - 2) * 4096u;
         uint8_t *stg_ptr = smem + S::kStgOff + (warp - 2) * 4096;
         int j = 0;
-        uint32_t nc = 0;  // bottleneck tiles so far
-        const uint32_t leader_a_ready = map_to_rank(a_ready, 0);
         const int nslots = g.sched_len ? g.sched_len : g.total_tiles;
         for (int slot = cluster; slot < nslots; slot += nclusters) {
-            const int t = tile_of(slot);
+            const int t = slot_tile(g, slot);
             if (t < 0) continue;
             const PairTile tr = locate_pair(g, t, rank);
             const auto &P = g.p[tr.prob];
             const int b = j & 1;
             const uint32_t use = (uint32_t)(j >> 1);
-            const bool bneck = FUSE != kFuseNone && tr.prob == 0;
             bool ok = ptx::mbar_wait(tfull_bar(b), use & 1, g.status);
             ok = __all_sync(0xffffffffu, ok);
-            // fused launches use named barriers below: leave together or not at all
-            if constexpr (FUSE != kFuseNone) ok = ptx::named_barrier_and(1, 256, ok);
             if (!ok) break;
             ptx::tc_fence_after();
-            if constexpr (FUSE != kFuseNone) {
-                if (bneck) {
-                    if (!bottleneck_epilogue<FUSE>(fa, smem + S::kStgOff, tmem + b * kAccCols, warp, lane, tr.m0,
-                                                   rank, leader_a_ready, b_full, nc & 1, g.status))
-                        break;
-                    ptx::tc_fence_before();
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive_cluster(b ? leader_tempty1 : leader_tempty0);
-                    // every warp's stores of this CTA's rows are issued: publish them
-                    ptx::named_barrier_sync(1, 256);
-                    if (warp == 2 && lane == 0) {
-                        __threadfence();
-                        ptx::fence_proxy_async_global();
-                        ptx::st_release_gpu(fa.flags + tr.m0 / kBM, 1u);
-                    }
-                    ++nc;
-                    ++j;
-                    continue;
-                }
-            }
             if (P.ep.tma)
                 Epi::run_tma(P.ep, &maps.m[tr.prob][4], stg_ptr, stg, tmem + b * kAccCols, P.bn, quarter, lane, tr.m0,
                              tr.n0, P.N, tr.z, half);

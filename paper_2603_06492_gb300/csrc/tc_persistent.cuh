@@ -45,7 +45,9 @@ struct GroupArgs {
 };
 
 struct GroupMaps {
-    CUtensorMap m[kMaxProblems][5];  // A0, B0, A1, B1, C (pair kernel's TMA-store epilogue)
+    // A0, B0, A1, B1, C (pair kernel's TMA-store epilogue), and for a fused
+    // launch's leader problem the B0 of CTA rank 1 (the branch weights)
+    CUtensorMap m[kMaxProblems][6];
 };
 
 }  // namespace tc

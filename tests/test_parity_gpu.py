@@ -62,6 +62,9 @@ FUSED = [
     (5000, 192, 264, 64),
     (2049, 512, 1000, 128),
     (300, 136, 264, 64),   # d_in % 64 != 0: fused forward, separate backward
+    (600, 128, 128, 128),  # d_in = d_out = r: leader tiles only
+    (1000, 320, 192, 64),  # forward: leader + 128-wide tail; backward: leader + 256-wide tiles
+    (20000, 192, 448, 64),  # more row pairs than clusters: several waves of leaders
 ]
 
 
