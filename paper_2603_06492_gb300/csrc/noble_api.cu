@@ -75,7 +75,9 @@ noble_status run(cudaStream_t st, const KernelInfo &ki, F &&f)
 // anything an earlier kernel of the call wrote, and every such grid waits at
 // least once, so its completion implies its predecessors'.  The first kernel
 // of a call, and the first after a memset, is launched normally and sees all
-// prior work in the stream.
+// prior work in the stream -- except the CosNet kernels, which wait for their
+// predecessor grid in every thread before any global read, so that their
+// set-up may overlap the previous kernel whatever it is.
 constexpr bool kProgrammaticLaunch = true;
 bool pdl_ok() { return kProgrammaticLaunch && g_call_kernels > 0; }
 
@@ -1126,9 +1128,13 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kDynamic) != cudaSuccess)
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
     const KernelInfo ki{name, kBoundHbm, 2.0 * T * R * (K + R), 2.0 * T * K + 2.0 * R * K + (BWD ? 14.0 : 10.0) * T * R};
+    // a programmatic dependent of whatever precedes it in the stream, also as
+    // the first kernel of a call: every thread waits for the predecessor grid
+    // (griddep_wait) before its first global read
     return run(st, ki, [&] {
         const unsigned grid = (unsigned)ceil_div(T, tc::kBM);
-        kern<<<grid, tc::kCosnetThreads, Cfg::kDynamic, st>>>(mA, mB, args);
+        launch_maybe_pdl(kern, dim3(grid), dim3(tc::kCosnetThreads), Cfg::kDynamic, st, kProgrammaticLaunch, mA, mB,
+                         args);
     });
 }
 

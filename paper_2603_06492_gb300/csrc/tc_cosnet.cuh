@@ -78,7 +78,7 @@ struct CosnetCfg {
     static constexpr int kKSteps = R < 64 ? R / 16 : 4;   // MMA K-steps per k-block
     static constexpr uint32_t kMkbBytes = 2 * R * 128;    // one k-block of M_hi and M_lo
     static constexpr uint32_t kTileBytes = kMkb * kBM * 128;  // epilogue row-operand tile, bf16
-    static constexpr uint32_t kExtra = 4 * R * 4 + 4 * 4 * R * 4 + 2048 + 256;  // params, column sums, barriers
+    static constexpr uint32_t kExtra = 4 * R * 4 + 4 * 4 * R * 4 + 256;  // params, column sums, barriers
     static constexpr uint32_t kFit = (227u * 1024u - 1024u - kExtra) / kStage;
     static constexpr int kStages = kFit > 8 ? 8 : (int)kFit;
     static_assert(kStages >= 2, "pipeline depth");
@@ -92,8 +92,7 @@ struct CosnetCfg {
     static constexpr uint32_t kMOff = 2 * kTileBytes;  // 1024-aligned
     static constexpr uint32_t kParamOff = kRing;        // omega/phi copies, 4 x R floats
     static constexpr uint32_t kPartOff = kParamOff + 4 * R * 4;  // [4 warps][4][R] floats
-    static constexpr uint32_t kBiasRedOff = kPartOff + 4 * 4 * R * 4;  // [8 warps][64] floats
-    static constexpr uint32_t kBarOff = kBiasRedOff + 8 * 64 * 4;
+    static constexpr uint32_t kBarOff = kPartOff + 4 * 4 * R * 4;
     static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 3) + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
@@ -174,9 +173,11 @@ __device__ __forceinline__ void store_segments(uint32_t (&w)[P][4], void *dst, i
         if (t0 + gb + i < T)
             *reinterpret_cast<uint4 *>(p + (int64_t)(gb + i) * pitch) = make_uint4(w[i][0], w[i][1], w[i][2], w[i][3]);
 }
-// Load the warp's segments (zeros for rows at or past T).
+// Issue the loads of the warp's segments (zeros for rows at or past T);
+// transpose_pieces<P>(w) then gives each lane its own row's pieces.
 template <int P>
-__device__ __forceinline__ void load_segments(uint32_t (&w)[P][4], const void *src, int64_t pitch, int64_t t0, int64_t T)
+__device__ __forceinline__ void load_segments_raw(uint32_t (&w)[P][4], const void *src, int64_t pitch, int64_t t0,
+                                                  int64_t T)
 {
     const int lane = threadIdx.x & 31;
     const int gb = lane & ~(P - 1);
@@ -187,7 +188,66 @@ __device__ __forceinline__ void load_segments(uint32_t (&w)[P][4], const void *s
         if (t0 + gb + i < T) v = __ldg(reinterpret_cast<const uint4 *>(p + (int64_t)(gb + i) * pitch));
         w[i][0] = v.x, w[i][1] = v.y, w[i][2] = v.z, w[i][3] = v.w;
     }
+}
+// Load the warp's segments (zeros for rows at or past T).
+template <int P>
+__device__ __forceinline__ void load_segments(uint32_t (&w)[P][4], const void *src, int64_t pitch, int64_t t0, int64_t T)
+{
+    load_segments_raw<P>(w, src, pitch, t0, T);
     transpose_pieces<P>(w);
+}
+
+// Column sums of one A stage (128 rows x 64 bf16 columns, K-major, 128-byte
+// swizzle): epilogue warp ew (0..7) takes columns [8 ew, 8 ew + 8), one
+// 16-byte piece per row.  Lane l adds rows l, l + 32, l + 64, l + 96 in that
+// order (rows l and l + 8 sit in different banks, so each load is four
+// conflict-free wavefronts), then the lanes are combined by recursive halving
+// (lane bits 4, 3, 2 select the column, bits 1, 0 finish the sum).  Returns
+// the sum of column 8 ew + col_of_lane(lane) on every lane; the order of the
+// additions is fixed.
+__device__ __forceinline__ int stage_colsum_col(int lane) { return ((lane >> 4) & 1) * 4 + ((lane >> 3) & 1) * 2 + ((lane >> 2) & 1); }
+__device__ __forceinline__ float stage_colsum8(const uint8_t *sA, int ew, int lane)
+{
+    float v[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i) v[i] = 0.f;
+    const uint32_t piece = ((uint32_t)ew ^ (uint32_t)(lane & 7)) << 4;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+        const int row = lane + 32 * q;
+        const uint4 u = *reinterpret_cast<const uint4 *>(sA + row * 128 + piece);
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[i]));
+            v[2 * i] += f.x;
+            v[2 * i + 1] += f.y;
+        }
+    }
+    {
+        const bool up = (lane & 16) != 0;
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const float send = up ? v[i] : v[i + 4], keep = up ? v[i + 4] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 16);
+        }
+    }
+    {
+        const bool up = (lane & 8) != 0;
+#pragma unroll
+        for (int i = 0; i < 2; ++i) {
+            const float send = up ? v[i] : v[i + 2], keep = up ? v[i + 2] : v[i];
+            v[i] = keep + __shfl_xor_sync(0xffffffffu, send, 8);
+        }
+    }
+    {
+        const bool up = (lane & 4) != 0;
+        const float send = up ? v[0] : v[1], keep = up ? v[1] : v[0];
+        v[0] = keep + __shfl_xor_sync(0xffffffffu, send, 4);
+    }
+    v[0] += __shfl_xor_sync(0xffffffffu, v[0], 2);
+    v[0] += __shfl_xor_sync(0xffffffffu, v[0], 1);
+    return v[0];
 }
 
 // Byte offset of element (row, col) in a 128-row bf16 K-major tile stored as
@@ -281,6 +341,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         ptx::tmem_alloc(ptx::smem_u32(tmem_slot), C::kTmemCols);
         ptx::tmem_relinquish();
     }
+    // launched as a programmatic dependent: the set-up above overlaps the
+    // previous kernel of the stream; nothing it wrote is read before this
+    ptx::griddep_wait();
     for (int i = threadIdx.x; i < R; i += blockDim.x) {
         // parameters a variant does not use may be NULL
         prm[i] = args.om1 ? args.om1[i] : 0.f;
@@ -417,63 +480,44 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         };
         // the first pass's part of M is read while the main loop runs
         if constexpr (sig_two_layers(SIG)) m_load(0);
-        if constexpr (BWD) {
-            // the tile's saved h and b rows are read after the main loop: bring
-            // them into L2 meanwhile
-            const int64_t nbytes = (min((int64_t)kBM, args.T - m0) > 0 ? min((int64_t)kBM, args.T - m0) : 0) * R * 4;
+        // the tile's saved h and b rows are read after the main loop: they are
+        // brought into L2 some k-blocks before its end (earlier, the streamed
+        // dy would evict them again), or at once without a dbias loop
+        auto prefetch_saved = [&] {
+            const int64_t rows = min((int64_t)kBM, args.T - m0);
+            const int64_t nbytes = (rows > 0 ? rows : 0) * R * 4;
             const uint8_t *hrow = reinterpret_cast<const uint8_t *>(args.h_in + m0 * R);
             const uint8_t *brow = reinterpret_cast<const uint8_t *>(args.b_in + m0 * R);
             for (int64_t off = (int64_t)et * 128; off < nbytes; off += 256 * 128) {
                 asm volatile("prefetch.global.L2 [%0];" ::"l"(hrow + off));
                 asm volatile("prefetch.global.L2 [%0];" ::"l"(brow + off));
             }
-        }
+        };
+        constexpr int kPrefetchAhead = 16;  // k-blocks, several microseconds of the main loop
+        if constexpr (BWD)
+            if (!args.bias_part) prefetch_saved();
         bool bias_ok = true;
         if constexpr (BWD) {
             if (args.bias_part) {
-                // dbias partials while the main loop runs: warp ew sums rows
-                // [16 ew, 16 ew + 16) of each dy stage for columns 2 lane, 2 lane + 1
-                // (rows ascending), then the eight warps' sums are added in order.
+                // dbias partials while the main loop runs: epilogue warp ew owns
+                // columns [8 ew, 8 ew + 8) of each dy stage and sums all 128 rows
+                // (stage_colsum8, a fixed order), so no warp waits for another
+                // before the stage goes back to the producer
                 const int ew = warp - 2;
-                float *red = reinterpret_cast<float *>(smem + C::kBiasRedOff);
                 for (int i = 0; i < args.kb; ++i) {
                     const int s = i % STAGES;
                     const uint32_t ph = (i / STAGES) & 1;
-                    bool w = bias_ok && ptx::mbar_wait(full_bar(s), ph, args.status);
-                    w = __all_sync(0xffffffffu, w);
-                    float s0 = 0.f, s1 = 0.f;
-                    if (w) {
-                        const uint8_t *sA = smem + s * C::kStage;
-#pragma unroll
-                        for (int rr = 0; rr < 16; ++rr) {
-                            const int rw = ew * 16 + rr;
-                            const uint32_t off =
-                                rw * 128 + ((((uint32_t)lane >> 2) ^ (rw & 7)) << 4) + ((lane & 3) << 2);
-                            const float2 f =
-                                __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(sA + off));
-                            s0 += f.x;
-                            s1 += f.y;
-                        }
-                        // the stage is refilled by the copy engine (async proxy)
-                        // once released: order these generic reads before that
-                        ptx::fence_proxy_async_smem();
-                        __syncwarp();
-                        if (lane == 0) ptx::mbar_arrive(empty_bar(s));
-                    }
-                    red[ew * 64 + 2 * lane] = s0;
-                    red[ew * 64 + 2 * lane + 1] = s1;
-                    // every epilogue warp reaches this barrier once per k-block,
-                    // whatever its waits returned
-                    bias_ok = ptx::named_barrier_and(2, 256, w);
-                    if (bias_ok && ew < 2) {
-                        const int cl = ew * 32 + lane;
-                        float sum = 0.f;
-#pragma unroll
-                        for (int w8 = 0; w8 < 8; ++w8) sum += red[w8 * 64 + cl];
-                        const int64_t col = (int64_t)i * 64 + cl;
-                        if (col < args.kdim) args.bias_part[(int64_t)blockIdx.x * args.kdim + col] = sum;
-                    }
-                    ptx::named_barrier_sync(2, 256);
+                    if (i == max(0, args.kb - kPrefetchAhead)) prefetch_saved();
+                    bias_ok = __all_sync(0xffffffffu, bias_ok && ptx::mbar_wait(full_bar(s), ph, args.status));
+                    if (!bias_ok) break;
+                    const float v = stage_colsum8(smem + s * C::kStage, ew, lane);
+                    // the stage is refilled by the copy engine (async proxy)
+                    // once released: order these generic reads before that
+                    ptx::fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) ptx::mbar_arrive(empty_bar(s));
+                    const int64_t col = (int64_t)i * kBK + 8 * ew + stage_colsum_col(lane);
+                    if ((lane & 3) == 0 && col < args.kdim) args.bias_part[(int64_t)blockIdx.x * args.kdim + col] = v;
                 }
             }
         }
@@ -622,10 +666,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                             for (int q = 0; q < 4; ++q) bv[4 * i + q] = __uint_as_float(w[i][q]);
                     }
-                    float q2[32], q3[32];
+                    // the column-sum operands replace their inputs in place
+                    // (bv: du2 b, v: du2), which keeps the register count low
                     uint32_t wdb[W / 8][4];
 #pragma unroll
-                    for (int i = W; i < 32; ++i) q2[i] = 0.f, q3[i] = 0.f;
+                    for (int i = W; i < 32; ++i) bv[i] = 0.f, v[i] = 0.f;
 #pragma unroll
                     for (int g = 0; g < W / 8; ++g) {
                         float o[8];
@@ -635,21 +680,21 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                             if constexpr (SIG == kSigAct2) {
                                 // f(b): db = f'(b) dc, no frequency or phase
                                 o[i] = live ? act::df(args.act, bv[j]) * v[j] : 0.f;
-                                q2[j] = 0.f;
-                                q3[j] = 0.f;
+                                bv[j] = 0.f;
+                                v[j] = 0.f;
                             } else {
                                 const float du2 = live ? -sin_reduced(fmaf(om2[k], bv[j], ph2[k])) * v[j] : 0.f;
                                 o[i] = om2[k] * du2;
-                                q2[j] = du2 * bv[j];
-                                q3[j] = du2;
+                                bv[j] *= du2;
+                                v[j] = du2;
                             }
                         }
                         const uint4 q = store_hi_lo(tile, row, c + 8 * g, o);
                         wdb[g][0] = q.x, wdb[g][1] = q.y, wdb[g][2] = q.z, wdb[g][3] = q.w;
                     }
                     store_segments<W / 8>(wdb, args.db_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
-                    const float s2 = warp_colsum32(q2);
-                    const float s3 = warp_colsum32(q3);
+                    const float s2 = warp_colsum32(bv);
+                    const float s3 = warp_colsum32(v);
                     if (c + lane < R) {
                         cpart[(quarter * 4 + 2) * R + c + lane] = s2;
                         cpart[(quarter * 4 + 3) * R + c + lane] = s3;
@@ -751,10 +796,9 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                             for (int q = 0; q < 4; ++q) hv[4 * i + q] = __uint_as_float(w[i][q]);
                     }
-                    float q0[32], q1[32];
-                    uint32_t wdh[W / 8][4], wa[W / 8][4];
+                                        uint32_t wdh[W / 8][4], wa[W / 8][4];
 #pragma unroll
-                    for (int i = W; i < 32; ++i) q0[i] = 0.f, q1[i] = 0.f;
+                    for (int i = W; i < 32; ++i) hv[i] = 0.f, v[i] = 0.f;
 #pragma unroll
                     for (int g = 0; g < W / 8; ++g) {
                         float dh[8], av[8];
@@ -765,16 +809,16 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                                 // f(h): dh = f'(h) da, a = f(h)
                                 dh[i] = live ? act::df(args.act, hv[j]) * v[j] : 0.f;
                                 av[i] = act::f(args.act, hv[j]);
-                                q0[j] = 0.f;
-                                q1[j] = 0.f;
+                                hv[j] = 0.f;
+                                v[j] = 0.f;
                             } else {
                                 float s1, c1;
                                 sincos_reduced(fmaf(om1[k], hv[j], ph1[k]), &s1, &c1);
                                 const float du1 = live ? -s1 * v[j] : 0.f;
                                 dh[i] = om1[k] * du1;
                                 av[i] = c1;
-                                q0[j] = du1 * hv[j];
-                                q1[j] = du1;
+                                hv[j] *= du1;  // the column-sum operands, in place
+                                v[j] = du1;
                             }
                         }
 #pragma unroll
@@ -785,8 +829,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     }
                     store_segments<W / 8>(wdh, args.dh_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                     store_segments<W / 8>(wa, args.a_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
-                    const float s0 = warp_colsum32(q0);
-                    const float s1 = warp_colsum32(q1);
+                    const float s0 = warp_colsum32(hv);
+                    const float s1 = warp_colsum32(v);
                     if (c + lane < R) {
                         cpart[(quarter * 4 + 0) * R + c + lane] = s0;
                         cpart[(quarter * 4 + 1) * R + c + lane] = s1;

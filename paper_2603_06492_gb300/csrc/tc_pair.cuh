@@ -364,32 +364,6 @@ __device__ __forceinline__ void mix_store(uint8_t *dst, int et, const float (&mr
     }
 }
 
-// Column sums of one A stage (128 rows x 64 bf16 columns, K-major, 128-byte
-// swizzle): epilogue warp ew (0..7) takes columns [8 ew, 8 ew + 8); lane l
-// adds rows 4l .. 4l + 3 in order, then the lanes are combined by a fixed
-// xor butterfly.  Every lane returns the eight sums.
-__device__ __forceinline__ void stage_colsum8(const uint8_t *sA, int ew, int lane, float (&s)[8])
-{
-#pragma unroll
-    for (int i = 0; i < 8; ++i) s[i] = 0.f;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const int row = 4 * lane + q;
-        const uint4 u = *reinterpret_cast<const uint4 *>(sA + row * 128 + (((uint32_t)ew ^ (uint32_t)(row & 7)) << 4));
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            const float2 f = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162 *>(&w[i]));
-            s[2 * i] += f.x;
-            s[2 * i + 1] += f.y;
-        }
-    }
-#pragma unroll
-    for (int m = 16; m >= 1; m >>= 1)
-#pragma unroll
-        for (int i = 0; i < 8; ++i) s[i] += __shfl_xor_sync(0xffffffffu, s[i], m);
-}
-
 // Bottleneck epilogue of a leader tile (see the header), run by all eight
 // epilogue warps of a CTA on its 128 rows.  `acc` is the tile's TMEM
 // accumulator after segment 0: columns [0, R) hold the output columns
@@ -964,19 +938,14 @@ gemm_pair(const __grid_constant__ GroupMaps maps, const __grid_constant__ GroupA
                                 cons ^= 1u << s;
                                 ok = __all_sync(0xffffffffu, ptx::mbar_wait(consumed_bar(s), par, g.status));
                                 if (!ok) break;
-                                float cs[8];
-                                stage_colsum8(smem + s * S::kStage, ew, lane, cs);
+                                const float v = stage_colsum8(smem + s * S::kStage, ew, lane);
                                 // the stage is refilled by the copy engine (async
                                 // proxy) once released: order these reads before that
                                 ptx::fence_proxy_async_smem();
                                 __syncwarp();
                                 if (lane == 0) ptx::mbar_arrive(empty_bar(s));
-                                float v = cs[0];
-#pragma unroll
-                                for (int q = 1; q < 8; ++q)
-                                    if (lane == q) v = cs[q];
-                                const int64_t col = (int64_t)i * kBK + 8 * ew + lane;
-                                if (lane < 8 && tr.m0 < fa.T && col < fa.kdim)
+                                const int64_t col = (int64_t)i * kBK + 8 * ew + stage_colsum_col(lane);
+                                if ((lane & 3) == 0 && tr.m0 < fa.T && col < fa.kdim)
                                     fa.bias_part[(tr.m0 / kBM) * fa.kdim + col] = v;
                             }
                         }
