@@ -259,6 +259,39 @@ noble_status noble_linear_lr_multipliers(const noble_linear_desc *desc, float ga
                                          float omega_mult, float phi_mult, float out[5]);
 
 /*
+ * Gradient bucket for data-parallel training (the paper trains on 8 GPUs
+ * with data parallelism, Section 4.1.1).  Tokens are split across ranks; the
+ * forward needs no exchange, and every parameter gradient is a sum over
+ * tokens, so the one exchange of a step is an all-reduce (sum) of the
+ * parameter gradients.  This describes one flat fp32 buffer holding all of a
+ * layer's parameter gradients, so that noble_linear_bwd writes straight into
+ * it (pass bucket + offset[i] as the i-th gradient pointer) and one
+ * collective per layer reduces them.
+ *
+ * Order of the slots (index: gradient, element count):
+ *   0 dW [d_out][d_in]   1 dbias [d_out]    2 dW_down [r][d_in]
+ *   3 dW_up [d_out][r]   4 dM [r][r]        5 domega1 [r]   6 dphi1 [r]
+ *   7 domega2 [r]        8 dphi2 [r]
+ *   9 dM2 [r][r]  10 domega3 [r]  11 dphi3 [r]  (NOBLE_FLAG_SIGMA_COS3 only)
+ * offset[i] is the byte offset of slot i from the start of the bucket, a
+ * multiple of NOBLE_GRAD_ALIGN; count[i] its element count (0 for a slot the
+ * descriptor does not have: the branch slots when r == 0, the three-layer
+ * slots without NOBLE_FLAG_SIGMA_COS3).  total_bytes is the bucket size, a
+ * multiple of NOBLE_GRAD_ALIGN.  Padding between slots is never written.
+ * Host only; no CUDA call.  NOBLE_ERR_INVALID_ARG for NULL pointers or an
+ * invalid descriptor.
+ */
+#define NOBLE_GRAD_COUNT 12
+#define NOBLE_GRAD_ALIGN 256u
+typedef struct {
+    size_t offset[NOBLE_GRAD_COUNT];
+    size_t count[NOBLE_GRAD_COUNT];
+    size_t total_bytes;
+} noble_grad_bucket;
+
+noble_status noble_linear_grad_bucket(const noble_linear_desc *desc, noble_grad_bucket *out);
+
+/*
  * Backward pass without a caller workspace, for callers that cannot allocate
  * device memory: code that runs inside a host framework or plugin which owns
  * every device allocation and hands its extensions no allocator, or a

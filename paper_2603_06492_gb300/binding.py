@@ -64,6 +64,17 @@ class AdamwHparams(ctypes.Structure):
                 ("eps", ctypes.c_float), ("weight_decay", ctypes.c_float), ("step", ctypes.c_int64)]
 
 
+GRAD_COUNT, GRAD_ALIGN = 12, 256
+# slots of the gradient bucket, in the order noble_linear_grad_bucket gives
+BUCKET_SLOTS = ("dW", "dbias", "dW_down", "dW_up", "dM", "domega1", "dphi1", "domega2", "dphi2",
+                "dM2", "domega3", "dphi3")
+
+
+class GradBucket(ctypes.Structure):
+    _fields_ = [("offset", ctypes.c_size_t * GRAD_COUNT), ("count", ctypes.c_size_t * GRAD_COUNT),
+                ("total_bytes", ctypes.c_size_t)]
+
+
 class Cos3Params(ctypes.Structure):
     _fields_ = [("M2", ctypes.c_void_p), ("omega3", ctypes.c_void_p), ("phi3", ctypes.c_void_p)]
 
@@ -143,6 +154,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.noble_adamw_step.restype = ctypes.c_int
         lib.noble_linear_lr_multipliers.argtypes = [D] + [ctypes.c_float] * 4 + [ctypes.POINTER(ctypes.c_float)]
         lib.noble_linear_lr_multipliers.restype = ctypes.c_int
+        lib.noble_linear_grad_bucket.argtypes = [D, ctypes.POINTER(GradBucket)]
+        lib.noble_linear_grad_bucket.restype = ctypes.c_int
         _lib = lib
         return lib
 
@@ -251,6 +264,32 @@ def noble_linear_lr_multipliers(desc, gamma=0.3, gamma_M=0.45, omega_mult=3.0, p
     return list(out)
 
 
+def noble_linear_grad_bucket(desc) -> dict:
+    """Layout of the layer's flat fp32 gradient bucket: {slot: (byte offset,
+    element count)} for the slots the descriptor has, and "total_bytes"."""
+    b = GradBucket()
+    _check(load().noble_linear_grad_bucket(ctypes.byref(desc), ctypes.byref(b)))
+    out = {name: (b.offset[i], b.count[i]) for i, name in enumerate(BUCKET_SLOTS) if b.count[i] > 0}
+    out["total_bytes"] = b.total_bytes
+    return out
+
+
+def bucket_views(bucket, layout: dict, shapes: dict) -> dict:
+    """Views of a flat fp32 bucket tensor (torch) as the layer's gradients."""
+    out = {}
+    for name, (off, n) in layout.items():
+        if name == "total_bytes":
+            continue
+        out[name] = bucket[off // 4: off // 4 + n].view(shapes[name])
+    return out
+
+
+def grad_shapes(d_in, d_out, r) -> dict:
+    return {"dW": (d_out, d_in), "dbias": (d_out,), "dW_down": (r, d_in), "dW_up": (d_out, r), "dM": (r, r),
+            "domega1": (r,), "dphi1": (r,), "domega2": (r,), "dphi2": (r,), "dM2": (r, r), "domega3": (r,),
+            "dphi3": (r,)}
+
+
 def noble_get_device_status(stream=None):
     _check(load().noble_get_device_status(stream))
 
@@ -299,6 +338,9 @@ class NobleLinearBuffers:
     """Caller-owned device buffers for one layer shape (allocated with torch)."""
 
     def __init__(self, T, d_in, d_out, r, dtype, device="cuda", with_grads=True, flags=0):
+        """With gradients, they are views of one flat fp32 bucket (``self.bucket``,
+        laid out by noble_linear_grad_bucket), which a data-parallel step
+        all-reduces in one collective."""
         import torch
         self.desc = make_desc(T, d_in, d_out, r, dtype, flags)
         tdt = torch.bfloat16 if self.desc.dtype == NOBLE_BF16 else torch.float32
@@ -311,20 +353,9 @@ class NobleLinearBuffers:
             f32 = dict(dtype=torch.float32, device=device)
             self.dx = torch.empty((T, d_in), dtype=tdt, device=device)
             self.workspace = torch.empty(self.workspace_bytes, dtype=torch.uint8, device=device)
-            self.grads = {"dW": torch.empty((d_out, d_in), **f32),
-                          "dbias": torch.empty(d_out, **f32)}
-            if r > 0:
-                self.grads.update({"dW_down": torch.empty((r, d_in), **f32),
-                                   "dM": torch.empty((r, r), **f32),
-                                   "domega1": torch.empty(r, **f32),
-                                   "dphi1": torch.empty(r, **f32),
-                                   "domega2": torch.empty(r, **f32),
-                                   "dphi2": torch.empty(r, **f32),
-                                   "dW_up": torch.empty((d_out, r), **f32)})
-                if flags & NOBLE_FLAG_SIGMA_COS3:
-                    self.grads.update({"dM2": torch.empty((r, r), **f32),
-                                       "domega3": torch.empty(r, **f32),
-                                       "dphi3": torch.empty(r, **f32)})
+            self.layout = noble_linear_grad_bucket(self.desc)
+            self.bucket = torch.zeros(self.layout["total_bytes"] // 4, **f32)
+            self.grads = bucket_views(self.bucket, self.layout, grad_shapes(d_in, d_out, r))
 
 
 def forward(buf: NobleLinearBuffers, x, params: dict, stream=None):

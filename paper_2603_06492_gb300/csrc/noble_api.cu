@@ -1795,6 +1795,26 @@ noble_status noble_adamw_step(const noble_adamw_tensor *tensors, int n_tensors, 
     return NOBLE_OK;
 }
 
+noble_status noble_linear_grad_bucket(const noble_linear_desc *desc, noble_grad_bucket *out)
+{
+    g_last_error[0] = 0;
+    if (!desc || !out) return fail(NOBLE_ERR_INVALID_ARG, "desc / out is NULL");
+    NOBLE_TRY(validate_desc(desc));
+    const int64_t di = desc->d_in, dout = desc->d_out, r = desc->r;
+    const bool cos3 = (desc->flags & kFlagSigmaCos3) != 0 && r > 0;
+    // element counts in the documented order; absent gradients take no room
+    const int64_t n[NOBLE_GRAD_COUNT] = {dout * di, dout, r * di, dout * r, r * r, r, r, r, r,
+                                         cos3 ? r * r : 0, cos3 ? r : 0, cos3 ? r : 0};
+    size_t off = 0;
+    for (int i = 0; i < NOBLE_GRAD_COUNT; ++i) {
+        out->offset[i] = off;
+        out->count[i] = (size_t)n[i];
+        off += ((size_t)n[i] * sizeof(float) + NOBLE_GRAD_ALIGN - 1) / NOBLE_GRAD_ALIGN * NOBLE_GRAD_ALIGN;
+    }
+    out->total_bytes = off;
+    return NOBLE_OK;
+}
+
 noble_status noble_linear_lr_multipliers(const noble_linear_desc *desc, float gamma, float gamma_M, float omega_mult,
                                          float phi_mult, float out[5])
 {
