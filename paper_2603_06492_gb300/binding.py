@@ -277,10 +277,10 @@ def noble_linear_grad_bucket(desc) -> dict:
 def bucket_views(bucket, layout: dict, shapes: dict) -> dict:
     """Views of a flat fp32 bucket tensor (torch) as the layer's gradients."""
     out = {}
-    for name, (off, n) in layout.items():
-        if name == "total_bytes":
-            continue
-        out[name] = bucket[off // 4: off // 4 + n].view(shapes[name])
+    for name, slot in layout.items():
+        if name != "total_bytes":
+            off, n = slot
+            out[name] = bucket[off // 4: off // 4 + n].view(shapes[name])
     return out
 
 

@@ -1133,7 +1133,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     // (griddep_wait) before its first global read
     return run(st, ki, [&] {
         const unsigned grid = (unsigned)ceil_div(T, tc::kBM);
-        launch_maybe_pdl(kern, dim3(grid), dim3(tc::kCosnetThreads), Cfg::kDynamic, st, kProgrammaticLaunch, mA, mB,
+        launch_maybe_pdl(kern, dim3(grid), dim3(Cfg::kThreads), Cfg::kDynamic, st, kProgrammaticLaunch, mA, mB,
                          args);
     });
 }

@@ -74,6 +74,13 @@ struct CosnetCfg {
     static constexpr uint32_t kA = kBM * kBK * 2;
     static constexpr uint32_t kB = B_MN ? kBChunks * kChunkBytes : R * kBK * 2;
     static constexpr uint32_t kStage = kA + kB;
+    // Epilogue warps: two per TMEM lane quarter, four for r >= 128 (more warps
+    // per scheduler hide the latency of the epilogue's dependent steps); a
+    // warp takes the 32-column chunks c with (c / 32) % kColGroups == its group.
+    static constexpr int kEpiWarps = R >= 128 ? 16 : 8;
+    static constexpr int kEpiThreads = 32 * kEpiWarps;
+    static constexpr int kColGroups = kEpiWarps / 4;
+    static constexpr int kThreads = 64 + kEpiThreads;
     static constexpr int kMkb = (R + 63) / 64;            // k-blocks of the r x r operand
     static constexpr int kKSteps = R < 64 ? R / 16 : 4;   // MMA K-steps per k-block
     static constexpr uint32_t kMkbBytes = 2 * R * 128;    // one k-block of M_hi and M_lo
@@ -279,9 +286,8 @@ __device__ __forceinline__ uint4 store_hi_lo_impl(uint8_t *tile, int row, int co
     return hi;
 }
 
-// Warps 0 (TMA) and 1 (MMA, TMEM owner) plus eight epilogue warps: two per
-// TMEM lane quarter, taking alternate 32-column chunks of their 32 rows.
-constexpr int kCosnetThreads = 320;
+// Warps 0 (TMA) and 1 (MMA, TMEM owner) plus CosnetCfg::kEpiWarps epilogue
+// warps, which split the 32-column chunks of their TMEM lane quarter's rows.
 
 // Bottleneck activation of the kernel: the CosNet of Eq. 2 (default), or the
 // variants of the ablation in Section 4.4 (Table 5): a single cosine
@@ -296,7 +302,7 @@ constexpr int kSigCosnet = 0, kSigCos1 = 1, kSigIdentity = 2, kSigAct1 = 3, kSig
 __host__ __device__ constexpr bool sig_two_layers(int sig) { return sig == kSigCosnet || sig == kSigAct2; }
 
 template <int R, bool BWD, int SIG = kSigCosnet>
-__global__ void __launch_bounds__(kCosnetThreads, 1)
+__global__ void __launch_bounds__(CosnetCfg<R, BWD>::kThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
                    const CosnetArgs args)
 {
@@ -344,13 +350,6 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
     // launched as a programmatic dependent: the set-up above overlaps the
     // previous kernel of the stream; nothing it wrote is read before this
     ptx::griddep_wait();
-    for (int i = threadIdx.x; i < R; i += blockDim.x) {
-        // parameters a variant does not use may be NULL
-        prm[i] = args.om1 ? args.om1[i] : 0.f;
-        prm[R + i] = args.ph1 ? args.ph1[i] : 0.f;
-        prm[2 * R + i] = args.om2 ? args.om2[i] : 0.f;
-        prm[3 * R + i] = args.ph2 ? args.ph2[i] : 0.f;
-    }
     ptx::tc_fence_before();
     __syncthreads();
     ptx::tc_fence_after();
@@ -410,10 +409,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             ptx::mbar_wait(tmem_full, 0, nullptr);
         }
     } else {
-        // ---------------- epilogue: 8 warps; a thread owns one token row and
-        // the 32-column chunks c with (c / 32) % 2 == half
+        // ---------------- epilogue: kEpiWarps warps; a thread owns one token
+        // row and the 32-column chunks c with (c / 32) % kColGroups == grp
+        constexpr int NE = C::kEpiThreads, CSTEP = 32 * C::kColGroups;
         const int quarter = warp % 4;
-        const int half = (warp - 2) / 4;
+        const int grp = (warp - 2) / 4;
         const int row = quarter * 32 + lane;
         const int64_t t = m0 + row;
         const bool live = t < args.T;
@@ -421,17 +421,26 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
         const uint32_t acc2 = lane_addr + C::kRCols;
         const float *om1 = prm, *ph1 = prm + R, *om2 = prm + 2 * R, *ph2 = prm + 3 * R;
+        // frequencies and phases into shared memory (parameters a variant does
+        // not use may be NULL); read after the barrier that follows the main
+        // loop, so the copies above start without waiting for these loads
+        for (int i = threadIdx.x - 64; i < R; i += NE) {
+            prm[i] = args.om1 ? args.om1[i] : 0.f;
+            prm[R + i] = args.ph1 ? args.ph1[i] : 0.f;
+            prm[2 * R + i] = args.om2 ? args.om2[i] : 0.f;
+            prm[3 * R + i] = args.ph2 ? args.ph2[i] : 0.f;
+        }
         uint8_t *tile = smem;  // the ring is free once the main accumulator is complete
         // The mixing matrix, bf16 high and low parts, K-major in the SW128
         // layout: group gi covers operand row n (an output column) and k-columns
         // [c, c + 8) of k-block j of a pass.  n runs fastest, so a warp reads
         // whole 128-byte rows of M in the forward.
-        const int et = threadIdx.x - 64;  // 0..255
+        const int et = threadIdx.x - 64;  // 0..NE-1
         constexpr int kGroups = R * 8 * C::kChunkKb;
-        constexpr int kIters = (kGroups + 255) / 256;
+        constexpr int kIters = (kGroups + NE - 1) / NE;
         float mraw[kIters][8];
         auto m_group = [&](int it, int pass, int &j, int &n, int &cg, int &c) {
-            const int gi = et + it * 256;
+            const int gi = et + it * NE;
             j = gi / (R * 8);
             n = gi % R;
             cg = ((gi / R) % 8) * 8;
@@ -483,31 +492,32 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         // the tile's saved h and b rows are read after the main loop: they are
         // brought into L2 some k-blocks before its end (earlier, the streamed
         // dy would evict them again), or at once without a dbias loop
-        auto prefetch_saved = [&] {
+        auto prefetch_saved = [&](int idx, int nthreads) {
             const int64_t rows = min((int64_t)kBM, args.T - m0);
             const int64_t nbytes = (rows > 0 ? rows : 0) * R * 4;
             const uint8_t *hrow = reinterpret_cast<const uint8_t *>(args.h_in + m0 * R);
             const uint8_t *brow = reinterpret_cast<const uint8_t *>(args.b_in + m0 * R);
-            for (int64_t off = (int64_t)et * 128; off < nbytes; off += 256 * 128) {
+            for (int64_t off = (int64_t)idx * 128; off < nbytes; off += (int64_t)nthreads * 128) {
                 asm volatile("prefetch.global.L2 [%0];" ::"l"(hrow + off));
                 asm volatile("prefetch.global.L2 [%0];" ::"l"(brow + off));
             }
         };
         constexpr int kPrefetchAhead = 16;  // k-blocks, several microseconds of the main loop
         if constexpr (BWD)
-            if (!args.bias_part) prefetch_saved();
+            if (!args.bias_part) prefetch_saved(et, NE);
         bool bias_ok = true;
         if constexpr (BWD) {
             if (args.bias_part) {
                 // dbias partials while the main loop runs: epilogue warp ew owns
                 // columns [8 ew, 8 ew + 8) of each dy stage and sums all 128 rows
                 // (stage_colsum8, a fixed order), so no warp waits for another
-                // before the stage goes back to the producer
+                // before the stage goes back to the producer; with sixteen
+                // epilogue warps the first eight take part
                 const int ew = warp - 2;
-                for (int i = 0; i < args.kb; ++i) {
+                for (int i = 0; ew < 8 && i < args.kb; ++i) {
                     const int s = i % STAGES;
                     const uint32_t ph = (i / STAGES) & 1;
-                    if (i == max(0, args.kb - kPrefetchAhead)) prefetch_saved();
+                    if (i == max(0, args.kb - kPrefetchAhead)) prefetch_saved(et, 256);
                     bias_ok = __all_sync(0xffffffffu, bias_ok && ptx::mbar_wait(full_bar(s), ph, args.status));
                     if (!bias_ok) break;
                     const float v = stage_colsum8(smem + s * C::kStage, ew, lane);
@@ -522,7 +532,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
         }
         bool ok = bias_ok && ptx::mbar_wait(tmem_full, 0, args.status);
-        ok = ptx::named_barrier_and(3, 256, ok);  // uniform over the epilogue warps
+        ok = ptx::named_barrier_and(3, NE, ok);  // uniform over the epilogue warps
         if (ok) {
             // the ring is free once the main accumulator is complete
             if constexpr (sig_two_layers(SIG)) m_store(0);
@@ -531,7 +541,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 // single-cosine or identity bottleneck: c (forward) or dh
                 // (backward) straight from the first accumulator
 #pragma unroll 1
-                for (int c = 32 * half; c < R; c += 64) {
+                for (int c = 32 * grp; c < R; c += CSTEP) {
                     float v[32];
                     if constexpr (R >= 32) {
                         ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
@@ -621,7 +631,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             } else {
             // ---- phase 1: first accumulator -> bf16 operand tile (+ outputs)
 #pragma unroll 1
-            for (int c = 32 * half; c < R; c += 64) {
+            for (int c = 32 * grp; c < R; c += CSTEP) {
                 float v[32];
                 if constexpr (R >= 32) {
                     ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
@@ -709,13 +719,13 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 if (pass > 0) {
                     // the previous pass's MMAs have read the operand blocks
                     ok = ptx::mbar_wait(m_empty, (pass - 1) & 1, args.status);
-                    ok = ptx::named_barrier_and(3, 256, ok);
+                    ok = ptx::named_barrier_and(3, NE, ok);
                     if (!ok) break;
                     m_load(pass);
                     m_store(pass);
                 }
                 ptx::fence_proxy_async_smem();
-                ptx::named_barrier_sync(1, 256);
+                ptx::named_barrier_sync(1, NE);
                 if (threadIdx.x == 64) {
                     ptx::tc_fence_after();
                     const uint32_t acc = tmem + C::kRCols;
@@ -743,14 +753,14 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             // the tile and the accumulator are given up
             if (threadIdx.x == 64) ptx::mma_commit(mma2_done);
             const bool done = ptx::mbar_wait(mma2_done, 0, args.status);
-            ok = ptx::named_barrier_and(3, 256, ok && done);
+            ok = ptx::named_barrier_and(3, NE, ok && done);
             }  // two layers
         }
         if (ok) {
             ptx::tc_fence_after();
             // ---- phase 2: second accumulator
 #pragma unroll 1
-            for (int c = 32 * half; sig_two_layers(SIG) && c < R; c += 64) {
+            for (int c = 32 * grp; sig_two_layers(SIG) && c < R; c += CSTEP) {
                 float v[32];
                 if constexpr (R >= 32) {
                     ptx::tmem_ld_32x32b_x32(acc2 + c, v);
@@ -839,8 +849,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
             if constexpr (BWD) {
                 // per-CTA column sums: the four warps added in warp order
-                ptx::named_barrier_sync(1, 256);
-                for (int k = threadIdx.x - 64; k < 4 * R; k += 256) {
+                ptx::named_barrier_sync(1, NE);
+                for (int k = threadIdx.x - 64; k < 4 * R; k += NE) {
                     const int q = k / R, col = k % R;
                     float s = 0.f;
 #pragma unroll

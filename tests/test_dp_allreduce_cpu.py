@@ -114,6 +114,22 @@ def test_bucket_layout(built):
         binding.noble_linear_grad_bucket(binding.make_desc(16, 100, 128, 16, "bf16"))
 
 
+def test_bucket_views_alias_the_slots(built):
+    import torch
+    from paper_2603_06492_gb300 import binding
+    d_in, d_out, r = 200, 264, 16
+    lay = binding.noble_linear_grad_bucket(binding.make_desc(300, d_in, d_out, r, "fp32", binding.NOBLE_FLAG_SIGMA_COS3))
+    bucket = torch.zeros(lay["total_bytes"] // 4)
+    views = binding.bucket_views(bucket, lay, binding.grad_shapes(d_in, d_out, r))
+    assert set(views) == set(binding.BUCKET_SLOTS)
+    for i, name in enumerate(binding.BUCKET_SLOTS):
+        off, n = lay[name]
+        assert tuple(views[name].shape) == binding.grad_shapes(d_in, d_out, r)[name]
+        views[name].fill_(i + 1)
+        assert torch.all(bucket[off // 4: off // 4 + n] == i + 1)
+    assert int((bucket != 0).sum()) == sum(lay[k][1] for k in binding.BUCKET_SLOTS)
+
+
 def test_allreduce_of_token_shards_equals_full_batch_gradients(built):
     import torch.multiprocessing as mp
     from paper_2603_06492_gb300 import binding
