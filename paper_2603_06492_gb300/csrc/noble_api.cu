@@ -937,12 +937,14 @@ noble_status tc_pair_group(cudaStream_t st, const char *name, int n, const ProbS
             using OutT = typename Epi::out_type;
             constexpr int64_t es = sizeof(OutT);
             const auto &e = eps[i];
+            // a transposed store writes C with rows n and columns m
+            const int64_t outM = e.transpose ? P.N : P.M, outN = e.transpose ? P.M : P.N;
             const bool ok = !e.col0 && reinterpret_cast<uintptr_t>(e.C) % 16 == 0 &&
-                            (e.ldc * es) % 16 == 0 && P.N % 4 == 0 &&
+                            (e.ldc * es) % 16 == 0 && outN % 4 == 0 &&
                             (P.nsplit == 1 || (e.split_stride * es) % 16 == 0);
             q.ep.tma = ok ? 1 : 0;
             if (ok)
-                NOBLE_TRY(make_store_map(&maps.m[np][4], e.C, es == 4, P.M, P.N, e.ldc, P.nsplit, e.split_stride));
+                NOBLE_TRY(make_store_map(&maps.m[np][4], e.C, es == 4, outM, outN, e.ldc, P.nsplit, e.split_stride));
         }
         tiles += (int)ceil_div(q.tiles_m, 2) * q.tiles_n * q.nsplit;
         const double K = (double)P.s0.K + (P.s1 ? (double)P.s1->K : 0.0);
@@ -1358,13 +1360,14 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         wgrad_shapes(d, mn);
         int which[kWgradKinds];
         int n = 0;
-        auto add = [&](int k, ProbSpec ps, float *out, int64_t ldc, bool col0) {
+        auto add = [&](int k, ProbSpec ps, float *out, int64_t ldc, bool col0, bool transpose = false) {
             // dW_down (dh), dM (a, db), dbias (the ones operand), dM2 (a2, db2) read
             // what earlier kernels of this call wrote; dW and dW_up read the inputs
             ps.dep = (k == 1 || k == 3 || k == 4 || k == 5) ? 1 : 0;
             P[n] = ps;
             E[n] = {out, ldc, nullptr, 0};
             E[n].col0 = col0 ? 1 : 0;
+            E[n].transpose = transpose ? 1 : 0;
             final_out[n] = out;
             which[n++] = k;
         };
@@ -1372,7 +1375,9 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
         // CTAs that drew fewer full tiles with the small ones
         add(0, ProbSpec{dout, di, TcSeg{dy, x, T}, nullptr, 256}, dW, di, false);
         if (r > 0) {
-            add(1, ProbSpec{r, di, TcSeg{dh, x, T}, nullptr, 256}, dW_down, di, false);
+            // dW_down^T = x^T dh (d_in x r), stored transposed: M = d_in fills
+            // whole 256-row pair tiles where M = r would leave half of each empty
+            add(1, ProbSpec{di, r, TcSeg{x, dh, T}, nullptr, r < 128 ? 128 : (int)r}, dW_down, di, false, true);
             add(2, ProbSpec{dout, r, TcSeg{dy, c, T}, nullptr, r < 128 ? 128 : (int)r}, dW_up, r, false);
             if (sg.two_layers())
                 add(3, ProbSpec{r, r, TcSeg{a, db, T}, nullptr, r < 128 ? 128 : (int)r}, dM, r, false);

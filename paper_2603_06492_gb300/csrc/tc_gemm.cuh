@@ -59,6 +59,7 @@ struct EpiStore {
         int64_t split_stride;  // elements between blockIdx.z partial outputs
         int col0 = 0;          // store only column 0 of each row, to C[row * ldc]
         int tma = 0;           // pair kernel: store through a 3-D TMA map of C (run_tma)
+        int transpose = 0;     // fp32: store the tile transposed, (m, n) to C[n * ldc + m]
     };
 
     // 32 accumulator columns [c, c+32) of this thread's row -> C (+ bias)
@@ -103,6 +104,22 @@ struct EpiStore {
             if (row < M && n0 == 0) *out = (OutT)v[0];
             return;
         }
+        if (p.transpose) {
+            // column n of the tile is row n of C: for each n the warp's lanes
+            // (consecutive m) write one contiguous 128-byte segment
+            OutT *outT = p.C + (int64_t)z * p.split_stride + row;
+#pragma unroll 1
+            for (int c = c0; c < bn; c += cstep) {
+                if (n0 + c >= N) break;
+                float v[32];
+                ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
+                if (row < M)
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (n0 + c + j < N) __stcs(outT + (n0 + c + j) * p.ldc, (OutT)v[j]);
+            }
+            return;
+        }
 #pragma unroll 1
         for (int c = c0; c < bn; c += cstep) {
             if (n0 + c >= N) break;  // warp-uniform: whole chunk past the edge
@@ -125,6 +142,34 @@ struct EpiStore {
                                    int z, int half)
     {
         const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
+        if constexpr (sizeof(OutT) == 4) {
+            if (p.transpose) {
+                // a 32 x 32 block transposed through the staging buffer: lane
+                // (tile row m) writes its column n into staging row n, word m
+                // (one 4-byte store per n, 32 distinct banks per store); the
+                // map describes C with rows n and columns m
+#pragma unroll 1
+                for (int c = 32 * half; c < bn; c += 64) {
+                    if (n0 + c >= N) break;
+                    if (lane == 0) ptx::bulk_wait_read_all();
+                    __syncwarp();
+                    float v[32];
+                    ptx::tmem_ld_32x32b_x32(lane_addr + c, v);
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        *reinterpret_cast<float *>(stg_ptr + j * 128 + ((((lane >> 2) ^ (j & 7))) << 4) + (lane & 3) * 4) =
+                            v[j];
+                    ptx::fence_proxy_async_smem();
+                    __syncwarp();
+                    if (lane == 0) {
+                        ptx::tma_store_3d_hint(map, stg, (int)(m0 + quarter * 32), (int)(n0 + c), z,
+                                               ptx::l2_policy_evict_first());
+                        ptx::bulk_commit_group();
+                    }
+                }
+                return;
+            }
+        }
         uint8_t *my_row = stg_ptr + lane * 128;
 #pragma unroll 1
         for (int c = half * kBoxCols; c < bn; c += 2 * kBoxCols) {
