@@ -127,6 +127,11 @@ struct Cos3 {
     float *dM2, *dom3, *dph3;
 };
 bool is_cos3(const noble_linear_desc *d) { return (d->flags & kFlagSigmaCos3) != 0 && d->r > 0; }
+bool use_tc(const noble_linear_desc *d);
+// The three-layer cosine on the tensor-core path runs in the bottleneck
+// kernel (both r x r products as tensor-core MMAs) for r <= 128; r = 256 keeps
+// the CUDA-core rows (its mixing matrices do not fit shared memory at once).
+bool cos3_tc(const noble_linear_desc *d) { return is_cos3(d) && use_tc(d) && d->r <= 128; }
 
 // Bottleneck activation selected by the descriptor: CosNet (Eq. 2), or a
 // variant of the ablation (Section 4.4, Table 5): single cosine, identity, or
@@ -334,7 +339,23 @@ WorkLayout work_layout(const noble_linear_desc *d)
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align_up(off + bytes, 256); return o; };
     L.dh = take(tr * esize(d));
-    if (is_cos3(d)) {
+    if (cos3_tc(d)) {
+        // three-layer cosine in the bottleneck kernel: a, db, a2, db2 (bf16),
+        // six column sums and the dbias partials per CTA (128-token tile)
+        L.a = take(tr * 2);
+        L.db = take(tr * 2);
+        L.a2 = take(tr * 2);
+        L.db2 = take(tr * 2);
+        L.n_cos_blocks = ceil_div(T, 128);
+        L.cos_part = take((size_t)L.n_cos_blocks * 6 * r * 4);
+        L.bias_part = take((size_t)L.n_cos_blocks * d->d_out * 4);
+        L.split = wgrad_split(d);
+        if (L.split > 1) {
+            int64_t mn[kWgradKinds][2];
+            wgrad_shapes(d, mn);
+            for (int i = 0; i < kWgradKinds; ++i) L.wsplit[i] = take((size_t)L.split * mn[i][0] * mn[i][1] * 4);
+        }
+    } else if (is_cos3(d)) {
         // three-layer cosine: dc (fp32) from a GEMM, the CUDA-core chain rule
         // writes a, db, a2, db2 (bf16 operands of the tensor-core weight
         // gradients, fp32 on the CUDA-core path) and partials per block
@@ -1013,6 +1034,18 @@ noble_status with_rank_tile(int64_t r, F &&f)
     }
     return fail(NOBLE_ERR_UNSUPPORTED, "rank %lld", (long long)r);
 }
+// The same for r <= 128 (kernels that hold a whole r x r operand in shared memory).
+template <class F>
+noble_status with_rank_tile_max128(int64_t r, F &&f)
+{
+    switch (r) {
+    case 16: return f(std::integral_constant<int, 16>{});
+    case 32: return f(std::integral_constant<int, 32>{});
+    case 64: return f(std::integral_constant<int, 64>{});
+    case 128: return f(std::integral_constant<int, 128>{});
+    }
+    return fail(NOBLE_ERR_UNSUPPORTED, "rank %lld", (long long)r);
+}
 
 // The all-ones [T][kOnesCols] bf16 operand of the backward without a branch
 // (dbias = dy^T 1 as extra weight-gradient columns).
@@ -1032,11 +1065,11 @@ noble_status fill_ones(cudaStream_t st, int64_t n, bf16 *ones)
 // Fixed-order sums of partial results: out_j[i] = sum_z part_j[z * stride_j + i]
 // (z ascending) for up to five outputs in one launch.
 struct SplitJobs {
-    const float *part[5];
-    float *out[5];
-    int64_t n[5], stride[5], begin[6];  // stride: elements between consecutive partials
+    const float *part[8];
+    float *out[8];
+    int64_t n[8], stride[8], begin[9];  // stride: elements between consecutive partials
     int nparts;
-    int jparts[5];  // partials of job j when non-zero (else nparts; reduce_split_kernel only)
+    int jparts[8];  // partials of job j when non-zero (else nparts; reduce_split_kernel only)
     int njobs;
 };
 // Block = 8 warps over 32 consecutive outputs: warp w adds partials
@@ -1166,9 +1199,24 @@ noble_status fwd_tc(const noble_linear_desc *d, const bf16 *x, const bf16 *W, co
     const SavedLayout SL = saved_layout(d);
     float *h = (float *)(saved + SL.h), *b = (float *)(saved + SL.b);
     bf16 *c = (bf16 *)(saved + SL.c);
+    if (c3 && cos3_tc(d)) {
+        // three-layer cosine in the bottleneck kernel: h, b, b2 (saved) and c
+        tc::CosnetArgs a{};
+        a.om1 = om1, a.ph1 = ph1, a.om2 = om2, a.ph2 = ph2, a.M = M;
+        a.M2 = c3->M2, a.om3 = c3->om3, a.ph3 = c3->ph3;
+        a.h_out = h, a.b_out = b, a.b2_out = (float *)(saved + SL.b2), a.c_out = c;
+        NOBLE_TRY(with_rank_tile_max128(r, [&](auto bn) {
+            constexpr int R = decltype(bn)::value;
+            return cosnet_launch<R, false, tc::kSigCos3>(st, "tc_down_cosnet_fwd", T, x, di, W_down, a);
+        }));
+        const TcSeg up{c, W_up, r};
+        ProbSpec P{T, dout, main, &up, 256};
+        P.dep = 2;  // c, written by the bottleneck kernel
+        return tc_pair_group<false, false, tc::EpiStore<bf16>>(st, "tc_main_up_fwd", 1, &P, &py);
+    }
     if (c3) {
-        // three-layer cosine: h = x W_down^T on the tensor cores (fp32 out), the
-        // cosines and r x r products on the CUDA cores, then the output GEMM
+        // three-layer cosine, r = 256: h = x W_down^T on the tensor cores (fp32
+        // out), the cosines and r x r products on the CUDA cores, then the output GEMM
         const ProbSpec Ph{T, r, TcSeg{x, W_down, di}, nullptr, r <= 128 ? 128 : 256};
         const tc::EpiStore<float>::Params Eh{h, r, nullptr, 0};
         NOBLE_TRY((tc_pair_group<false, false, tc::EpiStore<float>>(st, "tc_h_gemm", 1, &Ph, &Eh)));
@@ -1237,32 +1285,35 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
     bf16 *dh = (bf16 *)(ws + WL.dh), *a = (bf16 *)(ws + WL.a), *db = (bf16 *)(ws + WL.db);
     bf16 *ones = (bf16 *)(ws + WL.ones);
     const bool fused = fuse_bwd(d);
-    const bool ones_dbias = dbias && (r == 0 || c3);
+    const bool c3k = c3 && cos3_tc(d);  // three-layer cosine in the bottleneck kernel
+    const bool ones_dbias = dbias && (r == 0 || (c3 && !c3k));
     const Sigma sg = sigma_of(d);
     if (ones_dbias) NOBLE_TRY(fill_ones(st, T * kOnesCols, ones));
     // domega1, dphi1, domega2, dphi2 (and dbias) from per-CTA or per-32-token partials
+    // (and domega3, dphi3 of the three-layer cosine in the bottleneck kernel)
     auto reduce_cosnet = [&](const float *cpart, const float *bpart) {
         SplitJobs J{};
-        float *outs[4] = {dom1, dph1, dom2, dph2};
+        float *outs[6] = {dom1, dph1, dom2, dph2, c3k ? c3->dom3 : nullptr, c3k ? c3->dph3 : nullptr};
+        const int nq = c3k ? 6 : 4;
         J.nparts = (int)WL.n_cos_blocks;
         J.begin[0] = 0;
-        for (int q = 0; q < 4; ++q) {
+        for (int q = 0; q < nq; ++q) {
             J.part[q] = cpart + q * r;
             J.out[q] = outs[q];
             J.n[q] = r;
-            J.stride[q] = 4 * r;
+            J.stride[q] = nq * r;
             J.begin[q + 1] = J.begin[q] + r;
         }
-        J.njobs = 4;
+        J.njobs = nq;
         if (bpart) {
-            J.part[4] = bpart;
-            J.out[4] = dbias;
-            J.n[4] = dout;
-            J.stride[4] = dout;
-            J.begin[5] = J.begin[4] + dout;
-            J.njobs = 5;
+            J.part[nq] = bpart;
+            J.out[nq] = dbias;
+            J.n[nq] = dout;
+            J.stride[nq] = dout;
+            J.begin[nq + 1] = J.begin[nq] + dout;
+            J.njobs = nq + 1;
             // the fused launch keeps dbias partials per 128 tokens
-            if (fused) J.jparts[4] = (int)WL.n_bias_chunks;
+            if (fused) J.jparts[nq] = (int)WL.n_bias_chunks;
         }
         const int64_t total = J.begin[J.njobs];
         const KernelInfo kr{"reduce_partials", kBoundHbm, (double)total * J.nparts, 4.0 * total * (J.nparts + 1)};
@@ -1271,9 +1322,29 @@ noble_status bwd_tc(const noble_linear_desc *d, const bf16 *dy, const bf16 *x, c
             launch_maybe_pdl(reduce_split_kernel, dim3((unsigned)ceil_div(total, 32)), dim3(256), 0, st, pdl, J);
         });
     };
-    if (r > 0 && c3) {
-        // three-layer cosine: dc = dy W_up on the tensor cores (fp32 out), the
-        // chain rule on the CUDA cores (bf16 a, db, a2, db2 for the weight gradients)
+    if (r > 0 && c3k) {
+        // three-layer cosine in the bottleneck kernel: dc = dy W_up, the chain
+        // rule through the three layers (both r x r products as tensor-core
+        // MMAs), dh, a, db, a2, db2 and the six column sums
+        float *cpart = (float *)(ws + WL.cos_part);
+        float *bpart = (float *)(ws + WL.bias_part);
+        tc::CosnetArgs ca{};
+        ca.om1 = om1, ca.ph1 = ph1, ca.om2 = om2, ca.ph2 = ph2, ca.M = M;
+        ca.M2 = c3->M2, ca.om3 = c3->om3, ca.ph3 = c3->ph3;
+        ca.h_in = (const float *)(saved + SL.h), ca.b_in = (const float *)(saved + SL.b);
+        ca.b2_in = (const float *)(saved + SL.b2);
+        ca.dh_out = dh, ca.a_out = a, ca.db_out = db, ca.part = cpart;
+        ca.a2_out = (bf16 *)(ws + WL.a2), ca.db2_out = (bf16 *)(ws + WL.db2);
+        ca.bias_part = dbias ? bpart : nullptr;
+        ca.kdim = dout;
+        NOBLE_TRY(with_rank_tile_max128(r, [&](auto bn) {
+            constexpr int R = decltype(bn)::value;
+            return cosnet_launch<R, true, tc::kSigCos3>(st, "tc_dc_cosnet_bwd", T, dy, dout, W_up, ca);
+        }));
+        NOBLE_TRY(reduce_cosnet(cpart, dbias ? bpart : nullptr));
+    } else if (r > 0 && c3) {
+        // three-layer cosine, r = 256: dc = dy W_up on the tensor cores (fp32 out),
+        // the chain rule on the CUDA cores (bf16 a, db, a2, db2 for the weight gradients)
         float *dc = (float *)(ws + WL.dc);
         const ProbSpec Pc{T, r, TcSeg{dy, W_up, dout}, nullptr, r <= 128 ? 128 : 256};
         const tc::EpiStore<float>::Params Ec{dc, r, nullptr, 0};

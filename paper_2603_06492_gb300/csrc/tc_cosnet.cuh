@@ -45,13 +45,20 @@ struct CosnetArgs {
     // backward inputs / outputs
     const float *h_in, *b_in;
     __nv_bfloat16 *dh_out, *a_out, *db_out;
-    float *part;         // [gridDim.x][4][r]
+    float *part;         // [gridDim.x][4][r] ([6][r] for the three-layer cosine)
     // backward, optional: column sums of dy over this CTA's tokens,
     // [gridDim.x][kdim], accumulated from the dy tiles of the main loop
     float *bias_part;
     int64_t kdim;
     int act;             // kSigAct1 / kSigAct2: the activation (act::kTanh, kLeaky, kGelu)
     uint32_t *status;
+    // three-layer cosine (kSigCos3): the second mixing matrix, the third
+    // frequency and phase; the forward also writes b2, the backward reads it
+    // and writes a2 = cos(omega2 b + phi2) and db2 (part then holds six sums)
+    const float *M2, *om3, *ph3;
+    float *b2_out;
+    const float *b2_in;
+    __nv_bfloat16 *a2_out, *db2_out;
 };
 
 // B_MN: the main loop's B operand is MN-major (W_up [d_out][r] as stored, in
@@ -85,7 +92,9 @@ struct CosnetCfg {
     static constexpr int kKSteps = R < 64 ? R / 16 : 4;   // MMA K-steps per k-block
     static constexpr uint32_t kMkbBytes = 2 * R * 128;    // one k-block of M_hi and M_lo
     static constexpr uint32_t kTileBytes = kMkb * kBM * 128;  // epilogue row-operand tile, bf16
-    static constexpr uint32_t kExtra = 4 * R * 4 + 4 * 4 * R * 4 + 256;  // params, column sums, barriers
+    // frequencies and phases (up to six vectors), per-quarter column sums (up
+    // to six per column), barriers
+    static constexpr uint32_t kExtra = 6 * R * 4 + 4 * 6 * R * 4 + 256;
     static constexpr uint32_t kFit = (227u * 1024u - 1024u - kExtra) / kStage;
     static constexpr int kStages = kFit > 8 ? 8 : (int)kFit;
     static_assert(kStages >= 2, "pipeline depth");
@@ -97,9 +106,9 @@ struct CosnetCfg {
     static_assert(kChunkKb >= 1 && kMkb % kChunkKb == 0, "mixing matrix passes");
     static constexpr int kPasses = kMkb / kChunkKb;
     static constexpr uint32_t kMOff = 2 * kTileBytes;  // 1024-aligned
-    static constexpr uint32_t kParamOff = kRing;        // omega/phi copies, 4 x R floats
-    static constexpr uint32_t kPartOff = kParamOff + 4 * R * 4;  // [4 warps][4][R] floats
-    static constexpr uint32_t kBarOff = kPartOff + 4 * 4 * R * 4;
+    static constexpr uint32_t kParamOff = kRing;        // omega/phi copies, 6 x R floats
+    static constexpr uint32_t kPartOff = kParamOff + 6 * R * 4;  // [4 quarters][6][R] floats
+    static constexpr uint32_t kBarOff = kPartOff + 4 * 6 * R * 4;
     static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 3) + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
@@ -298,8 +307,16 @@ __device__ __forceinline__ uint4 store_hi_lo_impl(uint8_t *tile, int row, int co
 // so their epilogue ends after the first accumulator; the two-layer ones run
 // the CosNet epilogue with f in place of the cosines and no frequencies or
 // phases (their partial sums are written as zeros).
-constexpr int kSigCosnet = 0, kSigCos1 = 1, kSigIdentity = 2, kSigAct1 = 3, kSigAct2 = 4;
-__host__ __device__ constexpr bool sig_two_layers(int sig) { return sig == kSigCosnet || sig == kSigAct2; }
+//
+// kSigCos3, the three-layer cosine of the same ablation, adds a second
+// mixing matrix and a third cosine: a2 = cos(omega2 b + phi2), b2 = a2 M2,
+// c = cos(omega3 b2 + phi3).  Its epilogue runs a middle phase and a second
+// r x r product between the CosNet's two (r <= 128: one pass per matrix).
+constexpr int kSigCosnet = 0, kSigCos1 = 1, kSigIdentity = 2, kSigAct1 = 3, kSigAct2 = 4, kSigCos3 = 5;
+__host__ __device__ constexpr bool sig_two_layers(int sig)
+{
+    return sig == kSigCosnet || sig == kSigAct2 || sig == kSigCos3;
+}
 
 template <int R, bool BWD, int SIG = kSigCosnet>
 __global__ void __launch_bounds__(CosnetCfg<R, BWD>::kThreads, 1)
@@ -421,6 +438,13 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         const uint32_t lane_addr = tmem + ((uint32_t)(quarter * 32) << 16);
         const uint32_t acc2 = lane_addr + C::kRCols;
         const float *om1 = prm, *ph1 = prm + R, *om2 = prm + 2 * R, *ph2 = prm + 3 * R;
+        const float *om3 = prm + 4 * R, *ph3 = prm + 5 * R;
+        // the three-layer cosine: sums per column for three layers, and the
+        // outermost layer of the backward's first phase is the third one
+        constexpr bool C3 = SIG == kSigCos3;
+        static_assert(!C3 || C::kPasses == 1, "three-layer cosine: one pass per mixing matrix (r <= 128)");
+        constexpr int NQ = C3 ? 6 : 4;
+        const float *omL = C3 ? om3 : om2, *phL = C3 ? ph3 : ph2;  // the last layer's frequency and phase
         // frequencies and phases into shared memory (parameters a variant does
         // not use may be NULL); read after the barrier that follows the main
         // loop, so the copies above start without waiting for these loads
@@ -429,6 +453,10 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             prm[R + i] = args.ph1 ? args.ph1[i] : 0.f;
             prm[2 * R + i] = args.om2 ? args.om2[i] : 0.f;
             prm[3 * R + i] = args.ph2 ? args.ph2[i] : 0.f;
+            if constexpr (SIG == kSigCos3) {
+                prm[4 * R + i] = args.om3[i];
+                prm[5 * R + i] = args.ph3[i];
+            }
         }
         uint8_t *tile = smem;  // the ring is free once the main accumulator is complete
         // The mixing matrix, bf16 high and low parts, K-major in the SW128
@@ -449,19 +477,23 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         };
         // loads only: the values are first used in m_store, so the loads stay
         // in flight across whatever runs in between
-        auto m_load = [&](int pass) {
+        // the matrices of the r x r products in order: M (forward; the
+        // three-layer cosine's backward starts with M2, the forward ends with it)
+        const float *mat1 = (C3 && BWD) ? args.M2 : args.M;
+        const float *mat2 = (C3 && BWD) ? args.M : args.M2;
+        auto m_load = [&](int pass, const float *Mp) {
 #pragma unroll
             for (int it = 0; it < kIters; ++it) {
                 int j, n, cg, c;
                 if (!m_group(it, pass, j, n, cg, c)) continue;
                 if constexpr (BWD) {
-                    const float4 *src = reinterpret_cast<const float4 *>(args.M + (int64_t)n * R + c);  // M[n][c+q]
+                    const float4 *src = reinterpret_cast<const float4 *>(Mp + (int64_t)n * R + c);  // M[n][c+q]
                     const float4 u = __ldg(src), w = __ldg(src + 1);
                     mraw[it][0] = u.x, mraw[it][1] = u.y, mraw[it][2] = u.z, mraw[it][3] = u.w;
                     mraw[it][4] = w.x, mraw[it][5] = w.y, mraw[it][6] = w.z, mraw[it][7] = w.w;
                 } else {
 #pragma unroll
-                    for (int q = 0; q < 8; ++q) mraw[it][q] = __ldg(args.M + (int64_t)(c + q) * R + n);  // M[c+q][n]
+                    for (int q = 0; q < 8; ++q) mraw[it][q] = __ldg(Mp + (int64_t)(c + q) * R + n);  // M[c+q][n]
                 }
             }
         };
@@ -488,7 +520,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
         };
         // the first pass's part of M is read while the main loop runs
-        if constexpr (sig_two_layers(SIG)) m_load(0);
+        if constexpr (sig_two_layers(SIG)) m_load(0, mat1);
         // the tile's saved h and b rows are read after the main loop: they are
         // brought into L2 some k-blocks before its end (earlier, the streamed
         // dy would evict them again), or at once without a dbias loop
@@ -621,10 +653,10 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         const float s0 = warp_colsum32(q0);
                         const float s1 = warp_colsum32(q1);
                         if (c + lane < R) {
-                            cpart[(quarter * 4 + 0) * R + c + lane] = s0;
-                            cpart[(quarter * 4 + 1) * R + c + lane] = s1;
-                            cpart[(quarter * 4 + 2) * R + c + lane] = 0.f;  // no second layer
-                            cpart[(quarter * 4 + 3) * R + c + lane] = 0.f;
+                            cpart[(quarter * NQ + 0) * R + c + lane] = s0;
+                            cpart[(quarter * NQ + 1) * R + c + lane] = s1;
+                            cpart[(quarter * NQ + 2) * R + c + lane] = 0.f;  // no second layer
+                            cpart[(quarter * NQ + 3) * R + c + lane] = 0.f;
                         }
                     }
                 }
@@ -670,14 +702,17 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     for (int i = 0; i < 32; ++i) bv[i] = 0.f;
                     {
                         uint32_t w[W / 4][4];
-                        load_segments<W / 4>(w, args.b_in + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        load_segments<W / 4>(w, (C3 ? args.b2_in : args.b_in) + t0 * R + c, (int64_t)R * 4, t0,
+                                             args.T);
 #pragma unroll
                         for (int i = 0; i < W / 4; ++i)
 #pragma unroll
                             for (int q = 0; q < 4; ++q) bv[4 * i + q] = __uint_as_float(w[i][q]);
                     }
                     // the column-sum operands replace their inputs in place
-                    // (bv: du2 b, v: du2), which keeps the register count low
+                    // (bv: du2 b, v: du2), which keeps the register count low;
+                    // for the three-layer cosine this is its third layer (b2,
+                    // omega3, phi3: du3, db2)
                     uint32_t wdb[W / 8][4];
 #pragma unroll
                     for (int i = W; i < 32; ++i) bv[i] = 0.f, v[i] = 0.f;
@@ -693,8 +728,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                                 bv[j] = 0.f;
                                 v[j] = 0.f;
                             } else {
-                                const float du2 = live ? -sin_reduced(fmaf(om2[k], bv[j], ph2[k])) * v[j] : 0.f;
-                                o[i] = om2[k] * du2;
+                                const float du2 = live ? -sin_reduced(fmaf(omL[k], bv[j], phL[k])) * v[j] : 0.f;
+                                o[i] = omL[k] * du2;
                                 bv[j] *= du2;
                                 v[j] = du2;
                             }
@@ -702,12 +737,13 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         const uint4 q = store_hi_lo(tile, row, c + 8 * g, o);
                         wdb[g][0] = q.x, wdb[g][1] = q.y, wdb[g][2] = q.z, wdb[g][3] = q.w;
                     }
-                    store_segments<W / 8>(wdb, args.db_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                    store_segments<W / 8>(wdb, (C3 ? args.db2_out : args.db_out) + t0 * R + c, (int64_t)R * 2, t0,
+                                          args.T);
                     const float s2 = warp_colsum32(bv);
                     const float s3 = warp_colsum32(v);
                     if (c + lane < R) {
-                        cpart[(quarter * 4 + 2) * R + c + lane] = s2;
-                        cpart[(quarter * 4 + 3) * R + c + lane] = s3;
+                        cpart[(quarter * NQ + (C3 ? 4 : 2)) * R + c + lane] = s2;
+                        cpart[(quarter * NQ + (C3 ? 5 : 3)) * R + c + lane] = s3;
                     }
                 }
             }
@@ -721,7 +757,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     ok = ptx::mbar_wait(m_empty, (pass - 1) & 1, args.status);
                     ok = ptx::named_barrier_and(3, NE, ok);
                     if (!ok) break;
-                    m_load(pass);
+                    m_load(pass, mat1);
                     m_store(pass);
                 }
                 ptx::fence_proxy_async_smem();
@@ -754,25 +790,145 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             if (threadIdx.x == 64) ptx::mma_commit(mma2_done);
             const bool done = ptx::mbar_wait(mma2_done, 0, args.status);
             ok = ptx::named_barrier_and(3, NE, ok && done);
+            if constexpr (C3) {
+                // ---- middle phase (three-layer cosine): the first product's
+                // accumulator becomes the second product's row operand; that
+                // product (with the other matrix) goes into the first
+                // accumulator, whose h or dc phase 1 has consumed
+                if (ok) {
+                    m_load(0, mat2);
+                    m_store(0);
+                    ptx::tc_fence_after();
+#pragma unroll 1
+                    for (int c = 32 * grp; c < R; c += CSTEP) {
+                        float v[32];
+                        if constexpr (R >= 32) {
+                            ptx::tmem_ld_32x32b_x32(acc2 + c, v);
+                        } else {
+                            float w[16];
+                            ptx::tmem_ld_32x32b_x16(acc2 + c, w);
+#pragma unroll
+                            for (int i = 0; i < 16; ++i) v[i] = w[i], v[i + 16] = 0.f;
+                        }
+                        constexpr int W = R < 32 ? R : 32;
+                        if constexpr (!BWD) {
+                            // v = b: store b, operand a2 = cos(omega2 b + phi2)
+                            {
+                                uint32_t w[W / 4][4];
+#pragma unroll
+                                for (int i = 0; i < W / 4; ++i)
+#pragma unroll
+                                    for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
+                                if (args.b_out)
+                                    store_segments<W / 4>(w, args.b_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                            }
+#pragma unroll
+                            for (int g = 0; g < W / 8; ++g) {
+                                float o[8];
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) {
+                                    const int k = c + 8 * g + i;
+                                    o[i] = cos_reduced(fmaf(om2[k], v[8 * g + i], ph2[k]));
+                                }
+                                store_hi_lo(tile, row, c + 8 * g, o);
+                            }
+                        } else {
+                            // v = da2; with b of this row: du2 = -sin(u2) da2,
+                            // operand db = omega2 du2, a2 = cos(u2)
+                            float bv[32];
+#pragma unroll
+                            for (int i = 0; i < 32; ++i) bv[i] = 0.f;
+                            {
+                                uint32_t w[W / 4][4];
+                                load_segments<W / 4>(w, args.b_in + t0 * R + c, (int64_t)R * 4, t0, args.T);
+#pragma unroll
+                                for (int i = 0; i < W / 4; ++i)
+#pragma unroll
+                                    for (int q = 0; q < 4; ++q) bv[4 * i + q] = __uint_as_float(w[i][q]);
+                            }
+                            uint32_t wdb[W / 8][4], wa2[W / 8][4];
+#pragma unroll
+                            for (int i = W; i < 32; ++i) bv[i] = 0.f, v[i] = 0.f;
+#pragma unroll
+                            for (int g = 0; g < W / 8; ++g) {
+                                float o[8], a2v[8];
+#pragma unroll
+                                for (int i = 0; i < 8; ++i) {
+                                    const int k = c + 8 * g + i, j = 8 * g + i;
+                                    float s2, c2;
+                                    sincos_reduced(fmaf(om2[k], bv[j], ph2[k]), &s2, &c2);
+                                    const float du2 = live ? -s2 * v[j] : 0.f;
+                                    o[i] = om2[k] * du2;
+                                    a2v[i] = c2;
+                                    bv[j] *= du2;  // the column-sum operands, in place
+                                    v[j] = du2;
+                                }
+                                const uint4 q = store_hi_lo(tile, row, c + 8 * g, o);
+                                wdb[g][0] = q.x, wdb[g][1] = q.y, wdb[g][2] = q.z, wdb[g][3] = q.w;
+#pragma unroll
+                                for (int q2 = 0; q2 < 4; ++q2) wa2[g][q2] = ptx::pack_bf16x2(a2v[2 * q2], a2v[2 * q2 + 1]);
+                            }
+                            store_segments<W / 8>(wdb, args.db_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                            store_segments<W / 8>(wa2, args.a2_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                            const float s2 = warp_colsum32(bv);
+                            const float s3 = warp_colsum32(v);
+                            if (c + lane < R) {
+                                cpart[(quarter * NQ + 2) * R + c + lane] = s2;
+                                cpart[(quarter * NQ + 3) * R + c + lane] = s3;
+                            }
+                        }
+                    }
+                    // the first accumulator's loads are complete before the
+                    // product overwrites it
+                    ptx::tc_fence_before();
+                    ptx::fence_proxy_async_smem();
+                    ptx::named_barrier_sync(1, NE);
+                    if (threadIdx.x == 64) {
+                        ptx::tc_fence_after();
+#pragma unroll
+                        for (int kb = 0; kb < C::kMkb; ++kb) {
+#pragma unroll
+                            for (int kk = 0; kk < C::kKSteps; ++kk) {
+                                const uint32_t a_hi = sbase + kb * (kBM * 128) + kk * 32;
+                                const uint32_t a_lo = a_hi + C::kTileBytes;
+                                const uint32_t m_hi = sbase + C::kMOff + kb * C::kMkbBytes + kk * 32;
+                                const uint32_t m_lo = m_hi + R * 128;
+                                const uint64_t dah = ptx::smem_desc_sw128(a_hi, 16, 1024);
+                                const uint64_t dal = ptx::smem_desc_sw128(a_lo, 16, 1024);
+                                const uint64_t dmh = ptx::smem_desc_sw128(m_hi, 16, 1024);
+                                const uint64_t dml = ptx::smem_desc_sw128(m_lo, 16, 1024);
+                                ptx::mma_bf16(tmem, dah, dmh, idesc, (kb > 0 || kk > 0) ? 1u : 0u);
+                                ptx::mma_bf16(tmem, dal, dmh, idesc, 1u);
+                                ptx::mma_bf16(tmem, dah, dml, idesc, 1u);
+                            }
+                        }
+                        ptx::mma_commit(mma2_done);
+                    }
+                    const bool done2 = ptx::mbar_wait(mma2_done, 1, args.status);
+                    ok = ptx::named_barrier_and(3, NE, ok && done2);
+                }
+            }
             }  // two layers
         }
         if (ok) {
             ptx::tc_fence_after();
             // ---- phase 2: second accumulator
 #pragma unroll 1
+            // (the three-layer cosine's last product is in the first accumulator)
+            const uint32_t accL = C3 ? lane_addr : acc2;
             for (int c = 32 * grp; sig_two_layers(SIG) && c < R; c += CSTEP) {
                 float v[32];
                 if constexpr (R >= 32) {
-                    ptx::tmem_ld_32x32b_x32(acc2 + c, v);
+                    ptx::tmem_ld_32x32b_x32(accL + c, v);
                 } else {
                     float w[16];
-                    ptx::tmem_ld_32x32b_x16(acc2 + c, w);
+                    ptx::tmem_ld_32x32b_x16(accL + c, w);
 #pragma unroll
                     for (int i = 0; i < 16; ++i) v[i] = w[i], v[i + 16] = 0.f;
                 }
                 constexpr int W = R < 32 ? R : 32;
                 if constexpr (!BWD) {
-                    // v = b
+                    // v = b (the three-layer cosine: b2, with omega3 and phi3)
                     uint32_t wc[W / 8][4];
 #pragma unroll
                     for (int g = 0; g < W / 8; ++g) {
@@ -780,7 +936,7 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                         for (int i = 0; i < 8; ++i)
                             cc[i] = SIG == kSigAct2 ? act::f(args.act, v[8 * g + i])
-                                                    : cos_reduced(fmaf(om2[c + 8 * g + i], v[8 * g + i], ph2[c + 8 * g + i]));
+                                                    : cos_reduced(fmaf(omL[c + 8 * g + i], v[8 * g + i], phL[c + 8 * g + i]));
 #pragma unroll
                         for (int q = 0; q < 4; ++q) wc[g][q] = ptx::pack_bf16x2(cc[2 * q], cc[2 * q + 1]);
                     }
@@ -790,7 +946,8 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         for (int i = 0; i < W / 4; ++i)
 #pragma unroll
                             for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
-                        if (args.b_out) store_segments<W / 4>(w, args.b_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        float *bo = C3 ? args.b2_out : args.b_out;
+                        if (bo) store_segments<W / 4>(w, bo + t0 * R + c, (int64_t)R * 4, t0, args.T);
                     }
                     store_segments<W / 8>(wc, args.c_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                 } else {
@@ -842,20 +999,21 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                     const float s0 = warp_colsum32(hv);
                     const float s1 = warp_colsum32(v);
                     if (c + lane < R) {
-                        cpart[(quarter * 4 + 0) * R + c + lane] = s0;
-                        cpart[(quarter * 4 + 1) * R + c + lane] = s1;
+                        cpart[(quarter * NQ + 0) * R + c + lane] = s0;
+                        cpart[(quarter * NQ + 1) * R + c + lane] = s1;
                     }
                 }
             }
             if constexpr (BWD) {
-                // per-CTA column sums: the four warps added in warp order
+                // per-CTA column sums: the four lane quarters added in order
+                // (NQ sums per column: four, six for the three-layer cosine)
                 ptx::named_barrier_sync(1, NE);
-                for (int k = threadIdx.x - 64; k < 4 * R; k += NE) {
+                for (int k = threadIdx.x - 64; k < NQ * R; k += NE) {
                     const int q = k / R, col = k % R;
                     float s = 0.f;
 #pragma unroll
-                    for (int w = 0; w < 4; ++w) s += cpart[(w * 4 + q) * R + col];
-                    args.part[(int64_t)blockIdx.x * 4 * R + k] = s;
+                    for (int w = 0; w < 4; ++w) s += cpart[(w * NQ + q) * R + col];
+                    args.part[(int64_t)blockIdx.x * NQ * R + k] = s;
                 }
             }
         }

@@ -2,7 +2,8 @@
 the ablation in Section 4.4, Table 5) on the GPU through
 noble_linear_fwd_cos3 / noble_linear_bwd_cos3, against the oracle's fwd3 /
 bwd3 (pinned by tests/test_oracle_cos3.py), in fp32 and bf16 at ragged
-shapes for every rank, and on the CUDA-core path."""
+shapes for every rank (bf16, r <= 128: the tensor-core bottleneck kernel;
+r = 256: CUDA-core rows), and on the CUDA-core path."""
 import numpy as np
 import pytest
 
@@ -57,7 +58,8 @@ def inputs(layer, seed):
 
 @pytest.mark.parametrize("dtype", ["fp32", "bf16"])
 @pytest.mark.parametrize("shape", [(300, 200, 264, 16), (257, 192, 328, 64), (200, 256, 136, 128),
-                                   (130, 264, 256, 256)], ids=lambda s: "x".join(map(str, s)))
+                                   (130, 264, 256, 256), (777, 136, 200, 32), (1000, 512, 520, 128)],
+                         ids=lambda s: "x".join(map(str, s)))
 def test_cos3_matches_oracle(dtype, shape):
     layer = Layer("cos3", *shape, dtype)
     inp = inputs(layer, 61)
