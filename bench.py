@@ -620,6 +620,36 @@ def main():
                 "plain_ms": t_p, "plain_tflops": world * layer.plain().flops() / (t_p * 1e-3) / 1e12,
                 "overhead_vs_plain": t_n / t_p - 1.0}
 
+    # data parallel over N ranks (only under torchrun with N > 1): the same step
+    # followed by the sum-all-reduce of every layer's gradient bucket, each
+    # started as soon as that layer's backward is enqueued (NCCL overlaps it
+    # with the next layer); and the all-reduces alone.  The headline above is
+    # the replica step; these two report what the exchange adds.
+    dp = None
+    if dist is not None:
+        from paper_2603_06492_gb300.dp import GradAllReduce
+        ar = GradAllReduce()
+
+        def dp_step():
+            for d, b in zip(dev_inputs, bufs):
+                binding.forward(b, d["x"], d, stream)
+                binding.backward(b, d["x"], d["dy"], d, stream)
+                ar.launch(b.bucket)
+            ar.wait()
+
+        def allreduce_only():
+            for b in bufs:
+                ar.launch(b.bucket)
+            ar.wait()
+
+        dp_step()
+        ms_dp = timed(dp_step, args.steps) / args.steps
+        ms_ar = timed(allreduce_only, args.steps) / args.steps
+        dp = {"step_ms": ms_dp, "allreduce_ms_per_step": ms_ar,
+              "bucket_bytes_per_step": sum(b.layout["total_bytes"] for b in bufs),
+              "tflops": job_throughput(world, flops_step, ms_dp),
+              "note": "tokens sharded over ranks; one sum-all-reduce per layer's gradient bucket (NCCL)"}
+
     # cuBLAS reference timing of the plain layer (torch.matmul x3), context only
     def cublas_step():
         for d in dev_inputs:
@@ -679,6 +709,7 @@ def main():
             "overhead_vs_cublas_plain": ms_noble_med / args.steps / ms_cublas - 1.0,
             "roofline": roof, "cpu_baseline": cpu, "e2e": e2e, "per_layer": per_layer,
             "gpu_launches": launches,
+            "data_parallel": dp,
             "profiled_ms_per_step": ms_profiled / args.steps,
             "optimizer_step": adamw,
             "kernel_breakdown": {k: {"ms_per_step": v["ms"] / args.steps,

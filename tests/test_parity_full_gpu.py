@@ -1,9 +1,11 @@
 """Parity at the measured layer shapes (configs 1-4), in the same launch
 configuration bench.py times, on outputs the oracle can compute one by one:
 
-  * y and dx on sampled tokens (tokens are independent, so the oracle runs on
-    just those rows);
-  * sampled elements of dW and all of dbias (each is one sum over tokens);
+  * y and dx on one sampled token of every 128-token tile (up to 256 tiles)
+    and the last token (tokens are independent, so the oracle runs on just
+    those rows);
+  * one element of dW in every 256 x 256 tile, 1024 more at random, and all
+    of dbias (each is one sum over tokens);
   * every branch gradient (dW_down, dW_up, dM, domega, dphi) in full, from one
     full-batch oracle pass of the r-wide branch.
 """
@@ -63,8 +65,12 @@ def check_full_size(layer, seed, rng_seed, ctx, init="config", branch_delta=Fals
     rng = np.random.default_rng(rng_seed)
     tol = TOL[layer.dtype]
 
-    rows = np.sort(rng.choice(layer.T, 48, replace=False))
-    rows[-1] = layer.T - 1  # the ragged tail tile
+    # one token from each 128-token tile (at most 256 tiles), and the last token
+    # (the ragged tail tile): every row tile of every kernel is checked
+    nblk = -(-layer.T // 128)
+    blks = np.sort(rng.choice(nblk, min(nblk, 256), replace=False))
+    rows = np.minimum(blks * 128 + rng.integers(0, 128, blks.size), layer.T - 1)
+    rows = np.unique(np.append(rows, layer.T - 1))
     sub = {k: (v[rows] if k in ("x", "dy") else v) for k, v in p.items()}
     y_ref = oracle.fwd(sub["x"], sub["W"], sub["bias"], sub["W_down"], sub["omega1"], sub["phi1"],
                        sub["M"], sub["omega2"], sub["phi2"], sub["W_up"])
@@ -79,10 +85,14 @@ def check_full_size(layer, seed, rng_seed, ctx, init="config", branch_delta=Fals
                            sub["M"], sub["omega2"], sub["phi2"], np.zeros_like(sub["W_up"]))
         errs["branch"] = rel_err(got["y"][rows] - plain, y_ref - plain)
 
-    n = 512
-    o_idx = rng.integers(0, layer.d_out, n)
-    i_idx = rng.integers(0, layer.d_in, n)
-    o_idx[0], i_idx[0] = layer.d_out - 1, layer.d_in - 1
+    # dW: one element in each 256 x 256 output tile of the weight-gradient
+    # launch, 1024 more at random, and the far corner
+    tm, tn = -(-layer.d_out // 256), -(-layer.d_in // 256)
+    gm, gn = np.meshgrid(np.arange(tm), np.arange(tn), indexing="ij")
+    o_idx = np.minimum(gm.ravel() * 256 + rng.integers(0, 256, gm.size), layer.d_out - 1)
+    i_idx = np.minimum(gn.ravel() * 256 + rng.integers(0, 256, gn.size), layer.d_in - 1)
+    o_idx = np.concatenate([o_idx, rng.integers(0, layer.d_out, 1024), [layer.d_out - 1]])
+    i_idx = np.concatenate([i_idx, rng.integers(0, layer.d_in, 1024), [layer.d_in - 1]])
     dW_ref = oracle.outer_elems(p["dy"], p["x"], o_idx, i_idx)
     errs["dW"] = rel_err(got["dW"][o_idx, i_idx], dW_ref)
     ones = np.ones((layer.T, 1))
