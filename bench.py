@@ -413,19 +413,50 @@ def main():
     lib.noble_profile_enable(0)
     prof = binding.profile_read()
 
-    # overhead against the plain (r = 0) layer of this library: NOBLE and
-    # plain runs alternate five times, medians compared (clock and thermal
-    # drift between two single runs is of the size of the effect); each run's
-    # clock is sampled so that a clock-normalised overhead (time x median SM
-    # clock, i.e. SM cycles) can be given beside the raw one
+    # overhead against the plain (r = 0) layer of this library, in the two
+    # clock regimes of a GB300 under this load:
+    #  * burst (the reported overhead): NOBLE and plain runs of the timed steps
+    #    alternate five times, each after an idle second, so that both arms run
+    #    at the maximum SM clock as the headline steps do (a run that follows
+    #    another at once starts under the power cap the first one raised);
+    #    medians compared, each run's clock sampled, and a clock-normalised
+    #    overhead (time x median SM clock, i.e. SM cycles) given beside it;
+    #  * sustained: blocks of back-to-back runs per arm (NOBLE, plain, NOBLE,
+    #    plain) long enough to settle under the power cap, the median of each
+    #    block's later runs, with that block's clock
     reps_n, reps_p, clk_n, clk_p = [], [], [], []
+    sustained = {"noble": [], "plain": [], "noble_mhz": [], "plain_mhz": []}
     with ClockSampler(local_rank) as clk_ovh:
         for _ in range(5):
             for arm, reps, clks in ((False, reps_n, clk_n), (True, reps_p, clk_p)):
+                time.sleep(1.0)
                 m0 = clk_ovh.mark()
                 reps.append(timed(lambda: step(plain_bufs if arm else bufs, plain=arm), args.steps))
                 clks.append(clk_ovh.summary(m0, clk_ovh.mark()))
+        sus_k = max(1, args.steps // 2)
+        for _ in range(2):
+            for arm in (False, True):
+                key = "plain" if arm else "noble"
+                ts, m_begin = [], None
+                for i in range(40):
+                    if i == 25:
+                        m_begin = clk_ovh.mark()
+                    t = timed(lambda: step(plain_bufs if arm else bufs, plain=arm), sus_k) / sus_k
+                    if i >= 25:
+                        ts.append(t)
+                sustained[key].append(statistics.median(ts))
+                sustained[key + "_mhz"].append(clk_ovh.summary(m_begin, clk_ovh.mark()).get("sm_mhz"))
     ms_noble_med, ms_plain = statistics.median(reps_n), statistics.median(reps_p)
+    sus_n, sus_p = statistics.median(sustained["noble"]), statistics.median(sustained["plain"])
+    mhz_n = [m for m in sustained["noble_mhz"] if m]
+    mhz_p = [m for m in sustained["plain_mhz"] if m]
+    overhead_sustained = {
+        "noble_ms_per_step": sus_n, "plain_ms_per_step": sus_p, "overhead": sus_n / sus_p - 1.0,
+        "noble_sm_mhz": statistics.median(mhz_n) if mhz_n else None,
+        "plain_sm_mhz": statistics.median(mhz_p) if mhz_p else None,
+        "overhead_clock_normalised": (sus_n * statistics.median(mhz_n) / (sus_p * statistics.median(mhz_p)) - 1.0)
+        if mhz_n and mhz_p else None,
+        "method": "2 blocks per arm of 40 back-to-back runs of steps/2 steps; median of runs 26-40"}
 
     def med_mhz(clks):
         v = [c["sm_mhz"] for c in clks if c.get("sm_mhz")]
@@ -690,7 +721,9 @@ def main():
             "plain_ms_per_step": ms_plain / args.steps,
             "plain_tflops": world * flops_plain / (ms_plain / args.steps * 1e-3) / 1e12,
             "overhead_vs_plain": ms_noble_med / ms_plain - 1.0,
-            "overhead_method": "median of 5 alternating NOBLE / plain runs of the timed steps",
+            "overhead_method": "median of 5 alternating NOBLE / plain runs of the timed steps, each after an "
+                               "idle second (both arms at the maximum SM clock, as the headline)",
+            "overhead_sustained": overhead_sustained,
             "overhead_reps_ms_per_step": {"noble": [round(v / args.steps, 4) for v in reps_n],
                                           "plain": [round(v / args.steps, 4) for v in reps_p]},
             "overhead_clock_normalised": (cyc_n / cyc_p - 1.0) if cyc_n and cyc_p else None,
