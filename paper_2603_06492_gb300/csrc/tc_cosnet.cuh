@@ -14,6 +14,9 @@
 //   writes dh, a, db (bf16, [T][r]) and per-CTA column sums
 //             part[cta][0] = sum du1*h, [1] = sum du1, [2] = sum du2*b, [3] = sum du2
 //   (each [r]), reduced over the 128 tokens of the tile in a fixed order.
+//   The saved h and b rows are read straight from memory after the main
+//   loop: an L2 prefetch of them during the loop cost the streaming more than
+//   it saved the epilogue.
 //
 // The mixing matrix enters as a bf16 K-major operand that the epilogue
 // threads build in shared memory from the fp32 M once the main loop is done:
@@ -521,22 +524,6 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         };
         // the first pass's part of M is read while the main loop runs
         if constexpr (sig_two_layers(SIG)) m_load(0, mat1);
-        // the tile's saved h and b rows are read after the main loop: they are
-        // brought into L2 some k-blocks before its end (earlier, the streamed
-        // dy would evict them again), or at once without a dbias loop
-        auto prefetch_saved = [&](int idx, int nthreads) {
-            const int64_t rows = min((int64_t)kBM, args.T - m0);
-            const int64_t nbytes = (rows > 0 ? rows : 0) * R * 4;
-            const uint8_t *hrow = reinterpret_cast<const uint8_t *>(args.h_in + m0 * R);
-            const uint8_t *brow = reinterpret_cast<const uint8_t *>(args.b_in + m0 * R);
-            for (int64_t off = (int64_t)idx * 128; off < nbytes; off += (int64_t)nthreads * 128) {
-                asm volatile("prefetch.global.L2 [%0];" ::"l"(hrow + off));
-                asm volatile("prefetch.global.L2 [%0];" ::"l"(brow + off));
-            }
-        };
-        constexpr int kPrefetchAhead = 16;  // k-blocks, several microseconds of the main loop
-        if constexpr (BWD)
-            if (!args.bias_part) prefetch_saved(et, NE);
         bool bias_ok = true;
         if constexpr (BWD) {
             if (args.bias_part) {
@@ -549,7 +536,6 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                 for (int i = 0; ew < 8 && i < args.kb; ++i) {
                     const int s = i % STAGES;
                     const uint32_t ph = (i / STAGES) & 1;
-                    if (i == max(0, args.kb - kPrefetchAhead)) prefetch_saved(et, 256);
                     bias_ok = __all_sync(0xffffffffu, bias_ok && ptx::mbar_wait(full_bar(s), ph, args.status));
                     if (!bias_ok) break;
                     const float v = stage_colsum8(smem + s * C::kStage, ew, lane);
