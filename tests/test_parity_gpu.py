@@ -78,14 +78,35 @@ def test_fused_bottleneck(shape, separate):
     assert_close(got, ref, "bf16", ctx=f"{shape} {'separate' if separate else 'fused'}")
 
 
+def _bf16_ulp(v):
+    # spacing of bf16 numbers at |v| (8 significant bits)
+    e = np.floor(np.log2(np.maximum(np.abs(v), np.finfo(np.float32).tiny)))
+    return np.exp2(e - 7)
+
+
+def _is_bf16(v):
+    import torch
+    return np.array_equal(v, torch.from_numpy(v).to(torch.bfloat16).double().numpy())
+
+
 def test_fused_matches_separate():
-    # same arithmetic up to summation order: far tighter than the oracle bound
+    # same arithmetic up to summation order: far tighter than the oracle bound.
+    # Both runs accumulate in fp32 in different orders, so an output stored in
+    # bf16 may round the other way: there an element may differ by one bf16
+    # step of its own magnitude, and few elements may differ at all.
     layer = Layer("fused", 3000, 256, 520, 128, "bf16")
     inp = make_layer_inputs(layer, 99)
     a = run_gpu(layer, inp, flags=binding.NOBLE_FLAG_FUSED_BRANCH)
     b = run_gpu(layer, inp)
     for k in a:
-        assert rel_err(a[k], b[k]) <= 2e-3, (k, rel_err(a[k], b[k]))
+        if _is_bf16(a[k]) and _is_bf16(b[k]):
+            d = np.abs(a[k] - b[k])
+            step = _bf16_ulp(np.maximum(np.abs(a[k]), np.abs(b[k])))
+            scale = np.max(np.abs(b[k]))
+            assert np.all(d <= np.maximum(step, 2e-3 * scale)), (k, float(np.max(d / step)))
+            assert np.mean(d > 0) <= 0.02, (k, float(np.mean(d > 0)))
+        else:
+            assert rel_err(a[k], b[k]) <= 2e-3, (k, rel_err(a[k], b[k]))
 
 
 @pytest.mark.parametrize("dtype", ["fp32", "bf16"])
