@@ -81,7 +81,6 @@ def config_of(cfg, layers, world, sigma):
         {"name": l.name, "T": l.T, "d_in": l.d_in, "d_out": l.d_out, "r": l.r} for l in layers],
         "l2": "inputs larger than L2: each step streams ~1.8 GB of activations",
         "parallelism": f"replicas x{world}"}
-METRIC = "NOBLE linear fwd+bwd TFLOP/s"
 
 
 def peaks():
@@ -477,16 +476,26 @@ def main():
         for d, b in zip(dev_inputs, bset):
             binding.backward(b, d["x"], d["dy"], {k: d[k] for k in ("W", "bias")} if plain else d, stream)
 
-    ms_fwd, ms_bwd = timed(lambda: fwd_only(bufs), args.steps), timed(lambda: bwd_only(bufs), args.steps)
     # inference forward (NOBLE_FLAG_INFERENCE: h and b not saved)
     inf_bufs = [binding.NobleLinearBuffers(l.T, l.d_in, l.d_out, l.r, l.dtype, with_grads=False,
                                            flags=binding.NOBLE_FLAG_INFERENCE | b.desc.flags)
                 for l, b in zip(layers, bufs)]
     fwd_only(inf_bufs)
-    ms_fwd_inf = timed(lambda: fwd_only(inf_bufs), args.steps)
+    # each run after an idle second, so that every run starts at the maximum
+    # clock like the headline (back to back, the later runs would meet the
+    # power cap and the NOBLE / plain ratios would compare two clocks);
+    # NOBLE and plain alternate, three runs each, medians
+    passes = {"fwd": lambda: fwd_only(bufs), "fwd_p": lambda: fwd_only(plain_bufs, True),
+              "bwd": lambda: bwd_only(bufs), "bwd_p": lambda: bwd_only(plain_bufs, True),
+              "fwd_inf": lambda: fwd_only(inf_bufs)}
+    sep = {k: [] for k in passes}
+    for _ in range(3):
+        for k, fn in passes.items():
+            time.sleep(1.0)
+            sep[k].append(timed(fn, args.steps))
     del inf_bufs
-    ms_fwd_p = timed(lambda: fwd_only(plain_bufs, True), args.steps)
-    ms_bwd_p = timed(lambda: bwd_only(plain_bufs, True), args.steps)
+    ms_fwd, ms_bwd, ms_fwd_p, ms_bwd_p, ms_fwd_inf = (statistics.median(sep[k])
+                                                      for k in ("fwd", "bwd", "fwd_p", "bwd_p", "fwd_inf"))
     binding.noble_get_device_status(None)
 
     ms_step = ms / args.steps
