@@ -719,6 +719,28 @@ noble_status make_store_map(CUtensorMap *m, void *C, bool fp32, int64_t M, int64
     return NOBLE_OK;
 }
 
+// 2-D TMA map for the bottleneck kernel's row outputs [T][r] (fp32 or bf16):
+// box of 32 columns by 32 rows; 128-byte rows (fp32) with the 128-byte
+// swizzle, 64-byte rows (bf16) with the 64-byte swizzle.
+noble_status make_rows_map(CUtensorMap *m, void *p, bool fp32, int64_t T, int64_t r)
+{
+    EncodeTiledFn enc = encode_fn();
+    if (!enc) return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled is unavailable");
+    const cuuint64_t es = fp32 ? 4 : 2;
+    cuuint64_t dims[2] = {(cuuint64_t)r, (cuuint64_t)T};
+    cuuint64_t strides[1] = {(cuuint64_t)r * es};
+    cuuint32_t box[2] = {32, 32};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult res = enc(m, fp32 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT32 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, p, dims,
+                       strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                       fp32 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B, CU_TENSOR_MAP_L2_PROMOTION_NONE,
+                       CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (res != CUDA_SUCCESS)
+        return fail(NOBLE_ERR_CUDA, "cuTensorMapEncodeTiled (rows) failed (%d): T=%lld r=%lld", (int)res,
+                    (long long)T, (long long)r);
+    return NOBLE_OK;
+}
+
 // The current CUDA context (NULL if none or the driver call is unavailable).
 typedef CUresult (*CtxGetCurrentFn)(CUcontext *);
 CUcontext current_context()
@@ -1159,6 +1181,19 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     args.T = T;
     args.kb = (int)ceil_div(K, tc::kBK);
     args.status = status_ptr();
+    // the epilogue's row outputs go out through TMA stores (CosNet, r in {64, 128})
+    tc::CosnetStoreMaps smaps{};
+    if constexpr (SIG == tc::kSigCosnet && Cfg::kStgFits) {
+        if (T > 0 && BWD) {
+            NOBLE_TRY(make_rows_map(&smaps.m[0], args.db_out, false, T, R));
+            NOBLE_TRY(make_rows_map(&smaps.m[1], args.dh_out, false, T, R));
+            NOBLE_TRY(make_rows_map(&smaps.m[2], args.a_out, false, T, R));
+        } else if (T > 0) {
+            if (args.h_out) NOBLE_TRY(make_rows_map(&smaps.m[0], args.h_out, true, T, R));
+            if (args.b_out) NOBLE_TRY(make_rows_map(&smaps.m[1], args.b_out, true, T, R));
+            NOBLE_TRY(make_rows_map(&smaps.m[2], args.c_out, false, T, R));
+        }
+    }
     auto kern = tc::cosnet_gemm_kernel<R, BWD, SIG>;
     if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kDynamic) != cudaSuccess)
         return fail(NOBLE_ERR_CUDA, "%s: cudaFuncSetAttribute: %s", name, cudaGetErrorString(cudaGetLastError()));
@@ -1169,7 +1204,7 @@ noble_status cosnet_launch(cudaStream_t st, const char *name, int64_t T, const b
     return run(st, ki, [&] {
         const unsigned grid = (unsigned)ceil_div(T, tc::kBM);
         launch_maybe_pdl(kern, dim3(grid), dim3(Cfg::kThreads), Cfg::kDynamic, st, kProgrammaticLaunch, mA, mB,
-                         args);
+                         args, smaps);
     });
 }
 

@@ -137,6 +137,16 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap *map, uint32_t sr
                  "r"(src), "r"(c0), "r"(c1), "r"(c2)
                  : "memory");
 }
+// 2-D tiled store shared -> global, tracked by this thread's bulk groups.
+// c0 is the innermost coordinate (elements); it must be a multiple of 16
+// bytes.  Elements outside the tensor's extent are not written.
+__device__ __forceinline__ void tma_store_2d(const CUtensorMap *map, uint32_t src, int c0, int c1)
+{
+    asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%2, %3}], [%1];" ::"l"(
+                     reinterpret_cast<uint64_t>(map)),
+                 "r"(src), "r"(c0), "r"(c1)
+                 : "memory");
+}
 // L2 policy that marks lines to be evicted first (outputs that this kernel
 // does not read back, so that they do not push its operands out of L2).
 __device__ __forceinline__ uint64_t l2_policy_evict_first()

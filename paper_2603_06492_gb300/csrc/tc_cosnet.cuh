@@ -64,6 +64,14 @@ struct CosnetArgs {
     __nv_bfloat16 *a2_out, *db2_out;
 };
 
+// TMA maps for the epilogue's row outputs (CosnetCfg::kStgFits): forward h,
+// b (fp32) and c (bf16); backward db, dh and a (bf16).  Each is a 2-D map over
+// [T][r] with a box of 32 columns by 32 rows (128-byte rows with the 128-byte
+// swizzle for fp32, 64-byte rows with the 64-byte swizzle for bf16).
+struct CosnetStoreMaps {
+    CUtensorMap m[3];
+};
+
 // B_MN: the main loop's B operand is MN-major (W_up [d_out][r] as stored, in
 // the backward), loaded as 64-wide column chunks of 64 K rows each; otherwise
 // it is K-major with R rows (W_down [r][d_in], in the forward).
@@ -112,6 +120,17 @@ struct CosnetCfg {
     static constexpr uint32_t kParamOff = kRing;        // omega/phi copies, 6 x R floats
     static constexpr uint32_t kPartOff = kParamOff + 6 * R * 4;  // [4 quarters][6][R] floats
     static constexpr uint32_t kBarOff = kPartOff + 4 * 6 * R * 4;
+    // Epilogue outputs through TMA stores: each epilogue warp stages its 32
+    // rows of a 32-column chunk and one lane stores them.  Phase 1 (h, or
+    // db) stages behind the mixing matrix, 4 KB per warp; phase 2 (b and c,
+    // or dh and a) from the start of the ring, 6 KB per warp, once the r x r
+    // product has read the operand tile and the matrix.  The two regions do
+    // not overlap, so phase 2 never waits for phase 1's copies.
+    static constexpr uint32_t kStg1Off = kMOff + kChunkKb * kMkbBytes;
+    static constexpr uint32_t kStg1Bytes = 4096, kStg2Bytes = 6144;
+    static constexpr bool kStgFits = kPasses == 1 && (R == 64 || R == 128) &&
+                                     kStg1Off + kEpiWarps * kStg1Bytes <= kRing &&
+                                     kEpiWarps * kStg2Bytes <= kStg1Off;
     static constexpr uint32_t kBytes = kBarOff + 8 * (2 * kStages + 3) + 16;
     static constexpr uint32_t kDynamic = kBytes + 1024;
 };
@@ -214,6 +233,33 @@ __device__ __forceinline__ void load_segments(uint32_t (&w)[P][4], const void *s
 {
     load_segments_raw<P>(w, src, pitch, t0, T);
     transpose_pieces<P>(w);
+}
+
+// The warp's rows of a 32-column chunk through a TMA store.  Lane l holds
+// row l's P 16-byte pieces (P = 8: fp32, P = 4: bf16) and writes them into
+// the warp's slot in the box layout of the map: 128-byte rows with the
+// 128-byte swizzle (piece j at j ^ (l & 7)) or 64-byte rows with the 64-byte
+// swizzle (piece j at j ^ ((l >> 1) & 3)); eight consecutive lanes then
+// cover all 32 banks.  Lane 0 stores the box at (column c, row t0); rows at
+// or past the tensor's end are clipped by the copy.  The slot must not be
+// written again before this lane's bulk group has read it.
+template <int P>
+__device__ __forceinline__ void stage_store(const uint32_t (&w)[P][4], uint8_t *slot, const CUtensorMap *map, int c,
+                                            int64_t t0)
+{
+    static_assert(P == 8 || P == 4, "fp32 or bf16 rows of 32 columns");
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int j = 0; j < P; ++j) {
+        const int pos = P == 8 ? (j ^ (lane & 7)) : (j ^ ((lane >> 1) & 3));
+        *reinterpret_cast<uint4 *>(slot + lane * (P * 16) + pos * 16) = make_uint4(w[j][0], w[j][1], w[j][2], w[j][3]);
+    }
+    ptx::fence_proxy_async_smem();
+    __syncwarp();
+    if (lane == 0) {
+        ptx::tma_store_2d(map, ptx::smem_u32(slot), c, (int)t0);
+        ptx::bulk_commit_group();
+    }
 }
 
 // Column sums of one A stage (128 rows x 64 bf16 columns, K-major, 128-byte
@@ -324,7 +370,7 @@ __host__ __device__ constexpr bool sig_two_layers(int sig)
 template <int R, bool BWD, int SIG = kSigCosnet>
 __global__ void __launch_bounds__(CosnetCfg<R, BWD>::kThreads, 1)
 cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant__ CUtensorMap mB,
-                   const CosnetArgs args)
+                   const CosnetArgs args, const __grid_constant__ CosnetStoreMaps smaps)
 {
     using C = CosnetCfg<R, BWD>;
     constexpr int STAGES = C::kStages;
@@ -462,6 +508,12 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
             }
         }
         uint8_t *tile = smem;  // the ring is free once the main accumulator is complete
+        // TMA stores of the row outputs (CosNet, r in {64, 128}): this warp's
+        // staging slots for phase 1 and phase 2
+        constexpr bool kTma = SIG == kSigCosnet && C::kStgFits;
+        uint8_t *stg1 = smem + C::kStg1Off + (warp - 2) * C::kStg1Bytes;
+        uint8_t *stg2 = smem + (warp - 2) * C::kStg2Bytes;
+        static_assert(!kTma || R == 32 * C::kColGroups, "one 32-column chunk per warp and phase");
         // The mixing matrix, bf16 high and low parts, K-major in the SW128
         // layout: group gi covers operand row n (an output column) and k-columns
         // [c, c + 8) of k-block j of a pass.  n runs fastest, so a warp reads
@@ -668,7 +720,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         for (int i = 0; i < W / 4; ++i)
 #pragma unroll
                             for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
-                        if (args.h_out) store_segments<W / 4>(w, args.h_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        if constexpr (kTma) {
+                            if (args.h_out) stage_store<W / 4>(w, stg1, &smaps.m[0], c, t0);
+                        } else if (args.h_out) {
+                            store_segments<W / 4>(w, args.h_out + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        }
                     }
 #pragma unroll
                     for (int g = 0; g < W / 8; ++g) {
@@ -723,8 +779,11 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                         const uint4 q = store_hi_lo(tile, row, c + 8 * g, o);
                         wdb[g][0] = q.x, wdb[g][1] = q.y, wdb[g][2] = q.z, wdb[g][3] = q.w;
                     }
-                    store_segments<W / 8>(wdb, (C3 ? args.db2_out : args.db_out) + t0 * R + c, (int64_t)R * 2, t0,
-                                          args.T);
+                    if constexpr (kTma)
+                        stage_store<W / 8>(wdb, stg1, &smaps.m[0], c, t0);
+                    else
+                        store_segments<W / 8>(wdb, (C3 ? args.db2_out : args.db_out) + t0 * R + c, (int64_t)R * 2,
+                                              t0, args.T);
                     const float s2 = warp_colsum32(bv);
                     const float s3 = warp_colsum32(v);
                     if (c + lane < R) {
@@ -933,9 +992,16 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
 #pragma unroll
                             for (int q = 0; q < 4; ++q) w[i][q] = __float_as_uint(v[4 * i + q]);
                         float *bo = C3 ? args.b2_out : args.b_out;
-                        if (bo) store_segments<W / 4>(w, bo + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        if constexpr (kTma) {
+                            if (bo) stage_store<W / 4>(w, stg2, &smaps.m[1], c, t0);
+                        } else if (bo) {
+                            store_segments<W / 4>(w, bo + t0 * R + c, (int64_t)R * 4, t0, args.T);
+                        }
                     }
-                    store_segments<W / 8>(wc, args.c_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                    if constexpr (kTma)
+                        stage_store<W / 8>(wc, stg2 + 4096, &smaps.m[2], c, t0);
+                    else
+                        store_segments<W / 8>(wc, args.c_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
                 } else {
                     // v = da; with h of this row: du1, dh = omega1 du1, a = cos(u1)
                     float hv[32];
@@ -980,8 +1046,13 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
                             wa[g][q] = ptx::pack_bf16x2(av[2 * q], av[2 * q + 1]);
                         }
                     }
-                    store_segments<W / 8>(wdh, args.dh_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
-                    store_segments<W / 8>(wa, args.a_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                    if constexpr (kTma) {
+                        stage_store<W / 8>(wdh, stg2, &smaps.m[1], c, t0);
+                        stage_store<W / 8>(wa, stg2 + 2048, &smaps.m[2], c, t0);
+                    } else {
+                        store_segments<W / 8>(wdh, args.dh_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                        store_segments<W / 8>(wa, args.a_out + t0 * R + c, (int64_t)R * 2, t0, args.T);
+                    }
                     const float s0 = warp_colsum32(hv);
                     const float s1 = warp_colsum32(v);
                     if (c + lane < R) {
@@ -1005,6 +1076,10 @@ cosnet_gemm_kernel(const __grid_constant__ CUtensorMap mA, const __grid_constant
         }
     }
 
+    // the epilogue's TMA stores are complete before the shared memory they
+    // read goes away
+    if constexpr (SIG == kSigCosnet && C::kStgFits)
+        if (warp >= 2 && lane == 0) ptx::bulk_wait_all();
     ptx::tc_fence_before();
     __syncthreads();
     if (warp == 1) {
