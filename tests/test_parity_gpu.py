@@ -38,6 +38,8 @@ SMALL = [
     (200, 256, 136, 128),
     (130, 264, 256, 256),
     (1, 128, 128, 64),
+    (33, 128, 136, 128),  # one row in the second 32-row box, the last two boxes past T
+    (31, 64, 72, 128),    # fewer tokens than one 32-row store box; a single k-block
     (127, 72, 40, 16),
     (333, 200, 264, 0),
 ]
